@@ -1,0 +1,371 @@
+"""Throughput of one encoder-slice training step (forward + backward) on GB300.
+
+A step is one pass of the whole hot path over one batch: the forward pass of
+every layer of the slice, then the backward pass in reverse order with all
+weight and input gradients (the per-device unit of work of the paper's
+layer-partitioned training, Sec. III / IV-D).  Default workload: BERT-large
+width, 8 layers, S=512, B=16 (bf16, seeded synthetic inputs standing in for
+the paper's MNLI batches).
+
+Prints one JSON line (rank 0).  `--impl reference` times the float64 CPU
+oracle instead (the reference arm).  With torchrun (N > 1) every rank runs an
+independent replica on its own GPU (the path has no data-path collective) and
+the slowest rank's time is reported.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2202_11836_gb300 import synth  # noqa: E402
+
+METRIC = "encoder-slice fwd+bwd tokens/sec on 1 GB300; % of bf16 tensor-core peak"
+DEFAULT_WORKLOAD = "large-s512"
+L2_BYTES = 129 * 2 ** 20
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"],
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def algorithmic_flops(w, lens):
+    """Matmul FLOPs of one step (forward + backward) over all layers."""
+    T, H, F, S = w.batch * w.seq, w.hidden, w.ffn, w.seq
+    gemm = 3 * 2 * T * (4 * H * H + 2 * H * F)
+    attn = 3 * 4 * H * S * int(np.sum(lens))
+    return w.layers * gemm, w.layers * attn
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.idx = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.idx)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0])); mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------ distributed
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), \
+        int(os.environ.get("LOCAL_RANK", 0))
+
+
+def timed_region(step, steps, warmup, sync, barrier, reduce_max, start_event, stop_event):
+    """W untimed steps, then K steps between a barrier + sync on both sides.
+
+    Returns the slowest rank's elapsed milliseconds for the K steps."""
+    for _ in range(warmup):
+        step()
+    sync()
+    barrier()
+    sync()
+    start_event()
+    for _ in range(steps):
+        step()
+    ms = stop_event()
+    sync()
+    barrier()
+    return reduce_max(ms)
+
+
+# ------------------------------------------------------------- CPU oracle
+def oracle_sample(w, seconds: float):
+    """Times the float64 oracle on one sequence and one layer of workload ``w``
+    (forward + backward) until ``seconds`` have passed; returns tokens/s of
+    the whole slice and a description."""
+    from oracle import encoder_f64 as ORC
+    lens = synth.lengths(w)
+    b = int(np.argmax(lens))
+    X = synth.activations(w, batch=b + 1)[b:b + 1].astype(np.float64)
+    dY = synth.upstream_grad(w, batch=b + 1)[b:b + 1].astype(np.float64)
+    p = synth.layer_params(w.layer_begin, w.hidden, w.ffn, w.dtype)
+    p = {k: v.astype(np.float64) for k, v in p.items()}
+    n, t0 = 0, time.perf_counter()
+    while True:
+        ORC.slice_step(X, lens[b:b + 1], dY, [p], w.heads, 1e-12)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    per_layer_seq = el / n
+    tok_s = w.seq / (per_layer_seq * w.layers)
+    desc = (f"{n} x (1 sequence of S={w.seq} (len {int(lens[b])}), 1 of {w.layers} layers, fwd+bwd,"
+            f" float64 numpy) in {el:.1f} s; scaled to the {w.layers}-layer slice")
+    return tok_s, desc, per_layer_seq
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def run_reference(args, w):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from oracle import encoder_f64 as ORC  # noqa: F401
+    for _ in range(args.warmup):
+        oracle_sample(w, 0.0)
+    vals, times = [], []
+    for _ in range(args.steps):
+        v, desc, t = oracle_sample(w, 0.0)
+        vals.append(v); times.append(t)
+    value = statistics.median(vals)
+    ms = statistics.median(times) * w.layers * w.batch * 1e3
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic", "config": config_of(w),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cpu_cores(),
+                             "kind": "oracle",
+                             "sample": "each step: 1 sequence x 1 layer fwd+bwd of the workload, "
+                                       "scaled to the whole slice"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_of(w):
+    return {"workload": w.name, "layers": w.layers, "hidden": w.hidden, "heads": w.heads,
+            "ffn": w.ffn, "seq": w.seq, "batch": w.batch, "tokens_per_step": w.tokens,
+            "dtype": w.dtype, "l2": "inputs larger than L2 (the step streams a multi-GB "
+            "activation stash; no explicit flush)"}
+
+
+# ---------------------------------------------------------------- GPU arm
+def run_gpu(args, w):
+    import torch
+    import torch.distributed as dist
+    from paper_2202_11836_gb300 import _lib
+    from paper_2202_11836_gb300.slice import EncoderSlice
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local)
+
+    lens = synth.lengths(w)
+    s = EncoderSlice(w.hidden, w.heads, w.ffn, w.layer_begin, w.layer_begin + w.layers,
+                     w.batch, w.seq, w.dtype)
+    for l in range(w.layer_begin, w.layer_begin + w.layers):
+        s.set_params(l, synth.layer_params(l, w.hidden, w.ffn, w.dtype))
+    tdt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    X = synth.activations(w)
+    dY = synth.upstream_grad(w)
+    x = torch.from_numpy(X).to(dev).to(tdt)
+    dy = torch.from_numpy(dY).to(dev).to(tdt)
+    ln = torch.from_numpy(lens).to(dev)
+    y = torch.empty_like(x)
+    dx = torch.empty_like(x)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        s.forward(x, ln, y, stream)
+        s.backward(dy, dx, stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def reduce_max(v):
+        if world > 1:
+            t = torch.tensor([v], dtype=torch.float64, device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            return float(t.item())
+        return v
+
+    ev = {}
+
+    def start():
+        ev["a"] = torch.cuda.Event(enable_timing=True)
+        ev["b"] = torch.cuda.Event(enable_timing=True)
+        ev["a"].record(stream)
+
+    def stop():
+        ev["b"].record(stream)
+        ev["b"].synchronize()
+        return ev["a"].elapsed_time(ev["b"])
+
+    sync = torch.cuda.synchronize
+    # 1. device-resident throughput
+    launches0 = _lib.lib().sky_launch_count()
+    props = torch.cuda.get_device_properties(local)
+    gpu_id = ("GPU-" + str(props.uuid)) if getattr(props, "uuid", None) else str(local)
+    with ClockSampler(gpu_id) as clk:
+        ms = timed_region(step, args.steps, args.warmup, sync, barrier, reduce_max, start, stop)
+    launches = (_lib.lib().sky_launch_count() - launches0)
+    launches_timed = launches * args.steps // (args.steps + args.warmup)
+    s.sync()
+    ms_step = ms / args.steps
+    tokens = w.tokens
+    value = world * tokens * args.steps / (ms / 1e3)
+    gemm_flops, attn_flops = algorithmic_flops(w, lens)
+    pk = peaks()
+
+    # 2. per-kernel CUDA-event timing of the same steps (roofline of the dominant kernel)
+    s.set_profiling(True)
+    ms_prof = timed_region(step, max(3, args.steps // 4), 1, sync, barrier, reduce_max, start, stop)
+    stats = s.kernel_stats()
+    s.set_profiling(False)
+    gemm_ms = sum(v["total_ms"] for k, v in stats.items() if k.startswith("gemm"))
+    gemm_f = sum(v["flops"] for k, v in stats.items() if k.startswith("gemm"))
+    gemm_n = sum(v["launches"] for k, v in stats.items() if k.startswith("gemm"))
+    achieved = gemm_f / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else 0.0
+    kernel_table = {k: {"launches": v["launches"], "ms": round(v["total_ms"], 4),
+                        "share": round(v["total_ms"] / max(1e-9, sum(x["total_ms"] for x in stats.values())), 4),
+                        "tflops": round(v["flops"] / (v["total_ms"] / 1e3) / 1e12, 1) if v["flops"] else None,
+                        "gbs": round(v["bytes"] / (v["total_ms"] / 1e3) / 1e9, 1) if v["bytes"] else None}
+                    for k, v in stats.items()}
+
+    # 3. per-layer cost (the allocator's per-layer time)
+    rec = s.layer_cost(w.batch, w.seq, iters=5)
+    per_layer_ms = statistics.median([r["fwd_ms"] + r["bwd_ms"] for r in rec])
+
+    # 4. end to end through the public API with host buffers
+    xh = torch.from_numpy(X).to(tdt).pin_memory()
+    dyh = torch.from_numpy(dY).to(tdt).pin_memory()
+    lh = torch.from_numpy(lens).pin_memory()
+    yh = torch.empty_like(xh).pin_memory()
+    dxh = torch.empty_like(xh).pin_memory()
+    h2d = xh.numel() * xh.element_size() * 2 + lh.numel() * 4
+    d2h = yh.numel() * yh.element_size() * 2
+
+    def step_e2e():
+        x.copy_(xh, non_blocking=True)
+        dy.copy_(dyh, non_blocking=True)
+        ln.copy_(lh, non_blocking=True)
+        s.forward(x, ln, y, stream)
+        s.backward(dy, dx, stream)
+        yh.copy_(y, non_blocking=True)
+        dxh.copy_(dx, non_blocking=True)
+
+    ms_e2e = timed_region(step_e2e, args.steps, 2, sync, barrier, reduce_max, start, stop)
+    e2e_value = world * tokens * args.steps / (ms_e2e / 1e3)
+    s.sync()
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        v, desc, _ = oracle_sample(w, args.cpu_seconds)
+        cpu = {"value": v, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+               "sample": desc}
+
+    if rank == 0:
+        total_f = gemm_flops + attn_flops
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+            "data": "synthetic", "config": config_of(w),
+            "pct_bf16_peak_end_to_end": round(100 * total_f / (ms_step / 1e3) / 1e12 / pk["bf16"], 2),
+            "tokens_per_s_per_layer": tokens / (per_layer_ms / 1e3),
+            "per_layer_ms": per_layer_ms,
+            "valid_tokens_per_s": world * int(np.sum(lens)) * args.steps / (ms / 1e3),
+            "roofline": {"kernel": "gemm_tc_kernel (all GEMM launches of the step)",
+                         "bound": "tensor", "achieved": round(achieved, 1),
+                         "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+                         "frac": round(achieved / pk["bf16_sus"], 4),
+                         "frac_of_burst_peak": round(achieved / pk["bf16"], 4),
+                         "peak_source": pk["source"] + " (sustained bf16; burst also given)",
+                         "traffic": None, "launches": gemm_n},
+            "kernels": kernel_table,
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": int(launches_timed),
+            "clocks": clk.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    s.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args(argv)
+    assert args.warmup >= 0 and args.steps >= 1
+    w = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_gpu(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,184 @@
+/*
+ * sky_slice.h -- C ABI of the GB300 encoder-slice library.
+ *
+ * The paper (Sky Computing, Sec. III and Sec. IV-D) partitions a deep BERT
+ * encoder by layer index: device i owns the contiguous layers
+ * pi[i] .. pi[i+1]-1, runs their forward pass on the activations it receives
+ * from device i-1, and, after the last device has finished, runs the backward
+ * pass in reverse order, computing the gradients of its own layers locally.
+ * This library is that per-device unit of work on one GPU: a "slice" is the
+ * post-LN BERT encoder layers [layer_begin, layer_end), and the calls below
+ * create it, run its forward and backward pass, and measure what each of its
+ * layers costs (the per-layer time and memory the paper's allocator consumes,
+ * Sec. IV-B).
+ *
+ * One encoder layer (Sec. II-C, Eq. 1), rows of X[T,H] with T = B*S tokens:
+ *   QKV = X Wqkv^T + bqkv                         (Wqkv[3H,H]: rows Q | K | V)
+ *   ctx = softmax(Q K^T / sqrt(D)) V per sequence b and head a, keys j < len[b]
+ *   X1  = LayerNorm(ctx Wo^T + bo + X) * gamma1 + beta1
+ *   Y   = LayerNorm(GELU(X1 W1^T + b1) W2^T + b2 + X1) * gamma2 + beta2
+ * GELU(z) = z * Phi(z) (exact erf form); LayerNorm uses the biased variance.
+ *
+ * Conventions for every call:
+ *   - Every function returns a sky_status and never aborts or throws across
+ *     the ABI.  After a failure, sky_last_error() holds a message (per thread).
+ *   - Activations are row-major [B, S, H] in the slice's dtype (bf16 bits or
+ *     fp32).  Lengths are int32[B] in device memory.  Padded positions
+ *     (s >= len[b]) are computed and returned; as keys they get probability 0.
+ *   - Device pointers passed in stay owned by the caller and must stay valid
+ *     until the work enqueued on the given stream has finished.
+ *   - All GPU work goes on the caller's stream (a cudaStream_t passed as
+ *     void*; NULL is the legacy default stream).  No call synchronises except
+ *     where stated.
+ *   - The library is not thread-safe per handle: calls on one handle must not
+ *     overlap.  Distinct handles are independent.
+ */
+#ifndef SKY_SLICE_H
+#define SKY_SLICE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SKY_OK = 0,
+  SKY_ERR_INVALID_ARG = 1,  /* bad size, null pointer, length outside [1,S] */
+  SKY_ERR_OOM = 2,          /* device memory for the slice does not fit     */
+  SKY_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed            */
+  SKY_ERR_STATE = 4,        /* e.g. backward without a matching forward     */
+  SKY_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up           */
+  SKY_ERR_UNSUPPORTED = 6   /* valid but not implemented (e.g. D != 64 bf16)*/
+} sky_status;
+
+typedef enum { SKY_DTYPE_BF16 = 0, SKY_DTYPE_FP32 = 1 } sky_dtype;
+
+/* Slice description.  layer_begin/layer_end are the partition indices
+ * [pi[i], pi[i+1]) of Sec. IV-D; they name global layer indices and only
+ * matter for reporting (parameters are set per layer by the caller).
+ * max_batch * max_seq sizes the activation stash and workspace, which are
+ * allocated once, at create.  bf16 slices need head dim D = width/heads = 64. */
+typedef struct {
+  int32_t width;        /* H */
+  int32_t heads;        /* A, width % heads == 0 */
+  int32_t ffn;          /* F */
+  int32_t layer_begin;  /* l0 */
+  int32_t layer_end;    /* l1 > l0 */
+  int32_t max_batch;    /* largest B a forward may use */
+  int32_t max_seq;      /* largest S a forward may use */
+  sky_dtype dtype;      /* storage type of activations and parameters */
+  float ln_eps;         /* LayerNorm epsilon (BERT uses 1e-12) */
+} sky_slice_config;
+
+/* Per-layer cost record (Sec. IV-B: the model benchmark's per-layer FLOPs
+ * lf_j and memory lm_j, and the device's measured time for them). */
+typedef struct {
+  int32_t layer;              /* global layer index */
+  int32_t _pad;
+  double fwd_ms, bwd_ms;      /* median measured time of this layer */
+  double fwd_flops, bwd_flops;/* algorithmic matmul FLOPs of this layer */
+  uint64_t param_bytes;       /* 12 parameter tensors, slice dtype */
+  uint64_t grad_bytes;        /* 12 gradient tensors, fp32 */
+  uint64_t stash_bytes;       /* activations kept from forward for backward */
+  uint64_t workspace_bytes;   /* this layer's share of the shared workspace */
+} sky_layer_cost;
+
+/* Per-kernel timing record (profiling, see sky_slice_set_profiling). */
+typedef struct {
+  char name[32];        /* kernel family, e.g. "gemm", "attn_fwd", "ln_fwd" */
+  int64_t launches;     /* launches timed since profiling was enabled */
+  double total_ms;      /* sum of CUDA-event durations of those launches */
+  double flops;         /* algorithmic FLOPs of those launches (0 if n/a) */
+  double bytes;         /* algorithmic HBM bytes of those launches */
+} sky_kernel_stat;
+
+typedef struct sky_slice sky_slice;  /* opaque, owned by the library */
+
+/* Order of the 12 per-layer tensors in set/get calls (layouts [out, in]):
+ *  0 Wqkv[3H,H] 1 bqkv[3H] 2 Wo[H,H] 3 bo[H] 4 gamma1[H] 5 beta1[H]
+ *  6 W1[F,H]    7 b1[F]    8 W2[H,F] 9 b2[H] 10 gamma2[H] 11 beta2[H]   */
+#define SKY_NUM_PARAMS 12
+
+/* Creates a slice and allocates its parameters, gradients, stash and
+ * workspace on the current CUDA device.  Parameters start at zero.
+ * Errors: INVALID_ARG (non-positive sizes, width % heads, l0 >= l1),
+ * UNSUPPORTED (bf16 with head dim != 64, or width % 8), OOM (the arena does
+ * not fit, or exceeds the cap of sky_debug_set_alloc_cap), CUDA. */
+sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out);
+
+/* Frees everything the slice owns.  NULL is accepted.  Synchronises the device. */
+sky_status sky_slice_destroy(sky_slice* s);
+
+/* Copies the 12 parameter tensors of global layer `layer` into the slice.
+ * tensors[k] points to tensor k in the slice dtype (host memory if
+ * on_device == 0, device memory otherwise).  Synchronous. */
+sky_status sky_slice_set_params(sky_slice* s, int32_t layer, const void* const* tensors,
+                                int on_device);
+
+/* Copies the 12 parameter tensors of `layer` out (slice dtype).  Synchronous. */
+sky_status sky_slice_get_params(sky_slice* s, int32_t layer, void* const* tensors, int on_device);
+
+/* Copies the 12 fp32 gradient tensors of `layer` (from the last backward)
+ * out.  Synchronous; also reports a pending device status (see sky_slice_sync). */
+sky_status sky_slice_get_grads(sky_slice* s, int32_t layer, void* const* tensors, int on_device);
+
+/* Forward pass of all layers of the slice: y = layer_{l1-1}(...layer_{l0}(x)).
+ * x, y: device [B,S,H] in the slice dtype (may not alias); d_len: device
+ * int32[B], each in [1,S] (checked on the device: a bad length is clamped,
+ * and reported as INVALID_ARG by the next synchronising call).  x is copied
+ * into the stash, so the caller may reuse it once the stream has passed it.
+ * Enqueues work on `stream`; no host synchronisation.
+ * Errors: INVALID_ARG (B > max_batch, S > max_seq, B or S < 1, null). */
+sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,
+                             int32_t S, void* y, void* stream);
+
+/* Backward pass of the slice for the most recent forward: given dy = dL/dy
+ * (device [B,S,H], slice dtype) writes dx = dL/dx and overwrites the fp32
+ * gradients of every layer.  Must follow a forward on the same handle (the
+ * forward's d_len must still be valid).  Enqueues on `stream`.
+ * Errors: STATE (no forward since create), INVALID_ARG (null). */
+sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stream);
+
+/* Measures every layer of the slice: runs `iters` forward+backward passes at
+ * [B,S] with full-length sequences and synthetic data already on the device
+ * (parameters as set), records CUDA events around each layer, and writes the
+ * median per-layer times with the analytic FLOPs and the byte counts.
+ * n_out must equal layer_end - layer_begin.  Synchronous; overwrites grads. */
+sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, int32_t iters,
+                                sky_layer_cost* out, int32_t n_out);
+
+/* Waits for the slice's enqueued work and reports device-side status:
+ * INVALID_ARG if a length was outside [1,S], TIMEOUT if a bounded wait gave
+ * up, CUDA on an asynchronous CUDA error.  Clears the status word. */
+sky_status sky_slice_sync(sky_slice* s);
+
+/* Enables (1) or disables (0) per-kernel CUDA-event timing of the slice's
+ * launches; enabling resets the counters. */
+sky_status sky_slice_set_profiling(sky_slice* s, int enable);
+
+/* Reads the per-kernel records accumulated while profiling was on
+ * (synchronises).  Writes at most n_out records and the count to *n_written. */
+sky_status sky_slice_kernel_stats(sky_slice* s, sky_kernel_stat* out, int32_t n_out,
+                                  int32_t* n_written);
+
+/* Bytes the slice allocated at create (parameters, grads, stash, workspace). */
+sky_status sky_slice_memory(const sky_slice* s, uint64_t* param_bytes, uint64_t* grad_bytes,
+                            uint64_t* stash_bytes, uint64_t* workspace_bytes);
+
+/* Host-side cap (bytes) on what sky_slice_create may allocate; 0 = no cap.
+ * Lets the out-of-memory path be tested without exhausting a device. */
+void sky_debug_set_alloc_cap(uint64_t bytes);
+
+/* Total number of kernels the library has launched in this process (all
+ * handles and threads), for accounting of GPU work. */
+int64_t sky_launch_count(void);
+
+const char* sky_status_string(sky_status st);
+const char* sky_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SKY_SLICE_H */

@@ -1,0 +1,76 @@
+// Shared host/device helpers of the encoder-slice library.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <cstdio>
+#include <string>
+
+#include "../../include/sky_ops.h"
+#include "../../include/sky_slice.h"
+
+namespace sky {
+
+// Device status word bits (sky_ops.h: d_status).
+constexpr int32_t kStatusBadLength = 1;
+constexpr int32_t kStatusTimeout = 2;
+
+// Records the thread-local error message returned by sky_last_error().
+void set_error(const char* fmt, ...);
+sky_status cuda_fail(cudaError_t e, const char* what);
+
+#define SKY_CUDA(call)                                        \
+  do {                                                        \
+    cudaError_t e_ = (call);                                  \
+    if (e_ != cudaSuccess) return ::sky::cuda_fail(e_, #call); \
+  } while (0)
+
+#define SKY_CHECK(cond, status, ...)   \
+  do {                                 \
+    if (!(cond)) {                     \
+      ::sky::set_error(__VA_ARGS__);   \
+      return (status);                 \
+    }                                  \
+  } while (0)
+
+// bf16 <-> fp32 conversions usable for both storage types.
+template <typename T> __device__ __forceinline__ float to_f32(T v);
+template <> __device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) {
+  return __bfloat162float(v);
+}
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
+  return __float2bfloat16_rn(v);
+}
+
+// GELU(h) = h * Phi(h) and its derivative Phi(h) + h * phi(h), via CUDA's
+// normcdff / expf (exact-erf form, no tanh approximation).
+__device__ __forceinline__ float gelu_f(float h) { return h * normcdff(h); }
+__device__ __forceinline__ float gelu_grad_f(float h) {
+  const float inv_sqrt_2pi = 0.3989422804014327f;
+  return normcdff(h) + h * inv_sqrt_2pi * expf(-0.5f * h * h);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+inline int ceil_div(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
+
+int sm_count();  // cached per device
+
+// Number of kernels this library has launched (all threads, all devices).
+void count_launches(int n);
+
+}  // namespace sky

@@ -1,0 +1,27 @@
+// Internal GEMM launchers (bf16 tensor-core and fp32 SIMT).
+#pragma once
+#include <cuda_runtime.h>
+
+#include "../../include/sky_ops.h"
+
+namespace sky {
+namespace gemm {
+
+// bf16 inputs on tcgen05; C is bf16 unless out_f32.
+sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
+                       void* C, bool out_f32, int epi, const void* bias, const void* aux,
+                       void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
+                       cudaStream_t stream);
+size_t workspace_bytes(sky_gemm_form form, int M, int N, int K, bool out_f32);
+int choose_splits(int tiles, int k_blocks, int sms);
+// Debug controls: per-wait timeout (0 = default 2 s) and the fault-injection
+// switch that makes the TMA producer skip its loads (waits then time out).
+void set_debug(uint64_t timeout_ns, int skip_loads);
+
+// fp32 SIMT path (exact fp32 FMA accumulation); same forms and epilogues.
+sky_status launch_f32(sky_gemm_form form, int M, int N, int K, const float* A, const float* B,
+                      float* C, int epi, const float* bias, const float* aux, float* aux_out,
+                      cudaStream_t stream);
+
+}  // namespace gemm
+}  // namespace sky

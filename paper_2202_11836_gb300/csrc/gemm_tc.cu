@@ -1,0 +1,471 @@
+// bf16 GEMMs of the encoder layer on the 5th-generation tensor cores.
+//
+// The linear maps of Sec. II-C (Q/K/V projection, attention-output dense,
+// intermediate and output layers) and their input and weight gradients are
+// the dense contractions of the slice.  One persistent, warp-specialised
+// kernel serves all three contraction forms:
+//   warp 0      TMA producer: 128-byte-swizzled tiles of A and B into a
+//               STAGES-deep shared-memory ring (mbarrier complete_tx),
+//   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=256,
+//               K=16) into a TMEM accumulator; two accumulators (512 TMEM
+//               columns) let the epilogue of one tile overlap the next,
+//   warps 2..5  epilogue: tcgen05.ld of the accumulator, fused bias / GELU /
+//               GELU' / residual, store to global memory.
+// K-major operands (x and W in y = x W^T) and MN-major operands (W in
+// dy W, and both operands of dy^T x) are read directly through the
+// descriptors' major-ness bit, so no transpose pass exists.  Weight gradients
+// (fp32 output) may split the token dimension over CTAs; partials go to a
+// workspace and are summed in a fixed order, so results are deterministic.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "gemm.h"
+#include "ptx.cuh"
+
+namespace sky {
+namespace gemm {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;        // 16 KiB
+constexpr int B_BYTES = BN * BK * 2;        // 32 KiB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int TMEM_COLS = 2 * BN;           // two fp32 accumulators of 128 x 256
+constexpr int NUM_THREADS = 192;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
+
+struct Params {
+  int M, N, K;
+  int m_tiles, n_tiles, splits, kb_per_split, k_blocks;
+  int epi;
+  int out_f32;
+  void* C;                        // bf16 [M,N], fp32 [M,N], or fp32 [splits][M][N]
+  const __nv_bfloat16* bias;      // [N] or null
+  const __nv_bfloat16* aux;       // [M,N] GELU input (GELU_BWD) or null
+  const float* aux32;             // [M,N] fp32 residual (RESIDUAL) or null
+  __nv_bfloat16* aux_out;         // [M,N] or null
+  int32_t* status;
+  uint64_t timeout_ns;
+  int skip_loads;                 // fault injection: producer never issues TMA
+};
+
+template <bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA,
+                   const __grid_constant__ CUtensorMap tmB, const Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_addr = ptx::smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      ptx::mbar_init(&tfull[a], 1);
+      ptx::mbar_init(&tempty[a], 128);
+    }
+    ptx::mbar_init(done, 1);
+    ptx::fence_mbar_init();
+    ptx::fence_proxy_async_smem();
+    ptx::prefetch_tensormap(&tmA);
+    ptx::prefetch_tensormap(&tmB);
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(tmem_slot, TMEM_COLS);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int tiles = p.m_tiles * p.n_tiles;
+  const int units = tiles * p.splits;
+  const uint64_t lim = p.timeout_ns;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const int split = u / tiles, rem = u % tiles;
+        const int m0 = (rem / p.n_tiles) * BM, n0 = (rem % p.n_tiles) * BN;
+        const int kb0 = split * p.kb_per_split;
+        const int kb1 = min(p.k_blocks, kb0 + p.kb_per_split);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, lim, p.status)) { ok = false; break; }
+          uint8_t* sa = smem + stage * STAGE_BYTES;
+          uint8_t* sb = sa + A_BYTES;
+          ptx::mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+          if (!p.skip_loads) {
+            const int k0 = kb * BK;
+            if (A_MN) {
+              ptx::tma_load_2d(sa, &tmA, &full[stage], m0, k0);
+              ptx::tma_load_2d(sa + MN_CHUNK_BYTES, &tmA, &full[stage], m0 + 64, k0);
+            } else {
+              ptx::tma_load_2d(sa, &tmA, &full[stage], k0, m0);
+            }
+            if (B_MN) {
+#pragma unroll
+              for (int j = 0; j < BN / 64; ++j)
+                ptx::tma_load_2d(sb + j * MN_CHUNK_BYTES, &tmB, &full[stage], n0 + 64 * j, k0);
+            } else {
+              ptx::tma_load_2d(sb, &tmB, &full[stage], k0, n0);
+            }
+          }
+          ++issued;
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // Drain: wait (bounded) for the loads still in flight before exiting.
+      const int n_tail = issued < STAGES ? issued : STAGES;
+      for (int i = 0; i < n_tail; ++i) {
+        if (--stage < 0) { stage = STAGES - 1; phase ^= 1u; }
+        ptx::mbar_wait(&full[stage], phase, lim, p.status);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- MMA issue
+    if (lane == 0) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, BN, A_MN, B_MN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t aphase = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const int split = u / tiles;
+        const int kb0 = split * p.kb_per_split;
+        const int kb1 = min(p.k_blocks, kb0 + p.kb_per_split);
+        if (!ptx::mbar_wait(&tempty[acc], aphase ^ 1u, lim, p.status)) break;
+        ptx::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!ptx::mbar_wait(&full[stage], phase, lim, p.status)) { ok = false; break; }
+          ptx::tc_fence_after();
+          const uint32_t sa = ptx::smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sa + A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t ad = A_MN ? ptx::smem_desc_sw128(sa + kk * 2048, MN_CHUNK_BYTES, 1024)
+                                     : ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
+            const uint64_t bd = B_MN ? ptx::smem_desc_sw128(sb + kk * 2048, MN_CHUNK_BYTES, 1024)
+                                     : ptx::smem_desc_sw128(sb + kk * 32, 16, 1024);
+            ptx::tc_mma_f16(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+          }
+          ptx::tc_commit(&empty[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        ptx::tc_commit(&tfull[acc]);
+        if (++acc == 2) { acc = 0; aphase ^= 1u; }
+      }
+      // All issued MMAs must finish before TMEM is released.
+      ptx::tc_commit(done);
+      ptx::mbar_wait(done, 0, lim, p.status);
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    int acc = 0;
+    uint32_t aphase = 0;
+    for (int u = blockIdx.x; u < units; u += gridDim.x) {
+      const int split = u / tiles, rem = u % tiles;
+      const int m0 = (rem / p.n_tiles) * BM, n0 = (rem % p.n_tiles) * BN;
+      if (!ptx::mbar_wait(&tfull[acc], aphase, lim, p.status)) break;
+      ptx::tc_fence_after();
+      const int row = m0 + q * 32 + lane;
+      const bool row_ok = row < p.M;
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        uint32_t r[32];
+        __syncwarp();
+        ptx::tmem_ld_32x32b_x32(taddr + c, r);
+        ptx::tmem_ld_wait();
+        const int n = n0 + c;
+        if (!row_ok || n >= p.N) continue;
+        const bool full_chunk = n + 32 <= p.N;
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+        const int64_t off = static_cast<int64_t>(row) * p.N + n;
+        const int nv = full_chunk ? 32 : p.N - n;
+        if (p.bias) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (j < nv) v[j] += __bfloat162float(p.bias[n + j]);
+        }
+        if (p.epi == SKY_EPI_GELU_BWD) {
+          __nv_bfloat16 a[32];
+          if (full_chunk) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 8)
+              *reinterpret_cast<uint4*>(&a[j]) = *reinterpret_cast<const uint4*>(p.aux + off + j);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) a[j] = j < nv ? p.aux[off + j] : __float2bfloat16(0.f);
+          }
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] *= gelu_grad_f(__bfloat162float(a[j]));
+        } else if (p.epi == SKY_EPI_RESIDUAL) {
+          if (full_chunk) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              const float4 q = *reinterpret_cast<const float4*>(p.aux32 + off + j);
+              v[j] += q.x; v[j + 1] += q.y; v[j + 2] += q.z; v[j + 3] += q.w;
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j < nv) v[j] += p.aux32[off + j];
+          }
+        }
+        if (p.out_f32) {
+          float* out = static_cast<float*>(p.C) +
+                       static_cast<int64_t>(split) * p.M * static_cast<int64_t>(p.N) + off;
+          if (full_chunk) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4)
+              *reinterpret_cast<float4*>(out + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+          } else {
+            for (int j = 0; j < nv; ++j) out[j] = v[j];
+          }
+          continue;
+        }
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.C) + off;
+        uint32_t packed[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) packed[j] = ptx::pack_bf16(v[2 * j], v[2 * j + 1]);
+        if (full_chunk) {
+#pragma unroll
+          for (int j = 0; j < 16; j += 4)
+            *reinterpret_cast<uint4*>(out + 2 * j) =
+                make_uint4(packed[j], packed[j + 1], packed[j + 2], packed[j + 3]);
+        } else {
+          for (int j = 0; j < nv; ++j) out[j] = __float2bfloat16_rn(v[j]);
+        }
+        if (p.epi == SKY_EPI_BIAS_GELU) {
+          __nv_bfloat16* g = p.aux_out + off;
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            packed[j] = ptx::pack_bf16(gelu_f(v[2 * j]), gelu_f(v[2 * j + 1]));
+          if (full_chunk) {
+#pragma unroll
+            for (int j = 0; j < 16; j += 4)
+              *reinterpret_cast<uint4*>(g + 2 * j) =
+                  make_uint4(packed[j], packed[j + 1], packed[j + 2], packed[j + 3]);
+          } else {
+            for (int j = 0; j < nv; ++j) g[j] = __float2bfloat16_rn(gelu_f(v[j]));
+          }
+        }
+      }
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&tempty[acc]);
+      if (++acc == 2) { acc = 0; aphase ^= 1u; }
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+// Fixed-order sum of split-K partials: out[i] = sum_s ws[s][i].
+__global__ void splitk_reduce_kernel(const float* __restrict__ ws, int splits, int64_t n,
+                                     float* __restrict__ out) {
+  const int64_t n4 = n / 4;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    float4 acc = reinterpret_cast<const float4*>(ws)[i];
+    for (int s = 1; s < splits; ++s) {
+      const float4 v = reinterpret_cast<const float4*>(ws + s * n)[i];
+      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    }
+    reinterpret_cast<float4*>(out)[i] = acc;
+  }
+  for (int64_t i = n4 * 4 + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    float acc = ws[i];
+    for (int s = 1; s < splits; ++s) acc += ws[s * n + i];
+    out[i] = acc;
+  }
+}
+
+// ------------------------------------------------------------------- host
+namespace {
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix, box {64, box_rows},
+// 128-byte swizzle; out-of-range elements read as zero.
+bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1u, 1u};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <bool A_MN, bool B_MN>
+cudaError_t set_smem_attr() {
+  static cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<A_MN, B_MN>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              SMEM_BYTES);
+  return e;
+}
+
+uint64_t g_timeout_ns = 2000000000ull;  // 2 s per wait
+int g_skip_loads = 0;
+}  // namespace
+
+void set_debug(uint64_t timeout_ns, int skip_loads) {
+  g_timeout_ns = timeout_ns ? timeout_ns : 2000000000ull;
+  g_skip_loads = skip_loads;
+}
+
+int choose_splits(int tiles, int k_blocks, int sms) {
+  // Estimated makespan (in k-block units) of `tiles * s` units on `sms` CTAs
+  // plus a small per-unit cost; the fixed-order reduce is charged per split.
+  int best = 1;
+  double best_cost = 1e30;
+  for (int s = 1; s <= 32 && s <= k_blocks; ++s) {
+    const int per = ceil_div(k_blocks, s);
+    const int s_eff = ceil_div(k_blocks, per);
+    const int waves = ceil_div((int64_t)tiles * s_eff, sms);
+    const double cost = waves * (per + 4.0) + (s_eff > 1 ? 2.0 + 0.5 * s_eff : 0.0);
+    if (cost < best_cost - 1e-9) { best_cost = cost; best = s_eff; }
+  }
+  return best;
+}
+
+size_t workspace_bytes(sky_gemm_form form, int M, int N, int K, bool out_f32) {
+  if (!out_f32) return 0;
+  const int tiles = ceil_div(M, BM) * ceil_div(N, BN);
+  const int kb = ceil_div(K, BK);
+  const int s = choose_splits(tiles, kb, sm_count() > 0 ? sm_count() : 148);
+  (void)form;
+  return s > 1 ? static_cast<size_t>(s) * M * N * sizeof(float) : 0;
+}
+
+sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
+                       void* C, bool out_f32, int epi, const void* bias, const void* aux,
+                       void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
+                       cudaStream_t stream) {
+  // TMA row pitches and the 16-byte epilogue stores need the contiguous
+  // dimensions to be multiples of 8 elements; the token dimension is free.
+  const bool dims_ok = N % 8 == 0 && (form == SKY_GEMM_XTW ? M % 8 == 0 : K % 8 == 0);
+  SKY_CHECK(dims_ok, SKY_ERR_UNSUPPORTED,
+            "bf16 GEMM form %d: contiguous dimensions must be multiples of 8 (M=%d N=%d K=%d)",
+            (int)form, M, N, K);
+  SKY_CHECK(M > 0 && N > 0 && K > 0, SKY_ERR_INVALID_ARG, "GEMM sizes must be positive");
+  SKY_CHECK((reinterpret_cast<uintptr_t>(A) & 15) == 0 && (reinterpret_cast<uintptr_t>(B) & 15) == 0,
+            SKY_ERR_UNSUPPORTED, "bf16 GEMM operands must be 16-byte aligned");
+  SKY_CHECK(reinterpret_cast<uintptr_t>(C) % 16 == 0, SKY_ERR_UNSUPPORTED,
+            "GEMM output must be 16-byte aligned");
+  SKY_CHECK(!out_f32 || epi == SKY_EPI_STORE || epi == SKY_EPI_RESIDUAL, SKY_ERR_UNSUPPORTED,
+            "fp32-output GEMM supports the STORE and RESIDUAL epilogues");
+  SKY_CHECK(epi != SKY_EPI_BIAS_GELU || (bias && aux_out), SKY_ERR_INVALID_ARG,
+            "BIAS_GELU epilogue needs bias and aux_out");
+  SKY_CHECK(epi != SKY_EPI_GELU_BWD && epi != SKY_EPI_RESIDUAL || aux, SKY_ERR_INVALID_ARG,
+            "epilogue needs aux");
+  const int sms = sm_count();
+  SKY_CHECK(sms > 0, SKY_ERR_CUDA, "no CUDA device");
+
+  CUtensorMap ta, tb;
+  const bool a_mn = form == SKY_GEMM_XTW;
+  const bool b_mn = form != SKY_GEMM_XWT;
+  bool ok = a_mn ? make_map(&ta, A, K, M, 64) : make_map(&ta, A, M, K, BM);
+  ok = ok && (b_mn ? make_map(&tb, B, K, N, 64) : make_map(&tb, B, N, K, BN));
+  SKY_CHECK(ok, SKY_ERR_CUDA, "cuTensorMapEncodeTiled failed (M=%d N=%d K=%d)", M, N, K);
+
+  Params p{};
+  p.M = M; p.N = N; p.K = K;
+  p.m_tiles = ceil_div(M, BM);
+  p.n_tiles = ceil_div(N, BN);
+  p.k_blocks = ceil_div(K, BK);
+  const bool may_split = out_f32 && epi == SKY_EPI_STORE && bias == nullptr;
+  p.splits = may_split ? choose_splits(p.m_tiles * p.n_tiles, p.k_blocks, sms) : 1;
+  if (p.splits > 1) {  // never more partials than the workspace holds
+    const size_t cap = ws_bytes / (static_cast<size_t>(M) * N * sizeof(float));
+    p.splits = cap < 2 ? 1 : (p.splits < (int)cap ? p.splits : (int)cap);
+  }
+  p.kb_per_split = ceil_div(p.k_blocks, p.splits);
+  p.splits = ceil_div(p.k_blocks, p.kb_per_split);
+  p.epi = epi;
+  p.out_f32 = out_f32 ? 1 : 0;
+  const size_t need = p.splits > 1 ? static_cast<size_t>(p.splits) * M * N * sizeof(float) : 0;
+  SKY_CHECK(ws_bytes >= need && (need == 0 || ws), SKY_ERR_INVALID_ARG,
+            "GEMM workspace too small (%zu < %zu)", ws_bytes, need);
+  p.C = p.splits > 1 ? ws : C;
+  p.bias = static_cast<const __nv_bfloat16*>(bias);
+  p.aux = epi == SKY_EPI_GELU_BWD ? static_cast<const __nv_bfloat16*>(aux) : nullptr;
+  p.aux32 = epi == SKY_EPI_RESIDUAL ? static_cast<const float*>(aux) : nullptr;
+  p.aux_out = static_cast<__nv_bfloat16*>(aux_out);
+  p.status = status;
+  p.timeout_ns = g_timeout_ns;
+  p.skip_loads = g_skip_loads;
+
+  const int units = p.m_tiles * p.n_tiles * p.splits;
+  const int grid = units < sms ? units : sms;
+  cudaError_t e;
+  if (form == SKY_GEMM_XWT) {
+    SKY_CUDA((set_smem_attr<false, false>()));
+    gemm_tc_kernel<false, false><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
+  } else if (form == SKY_GEMM_XW) {
+    SKY_CUDA((set_smem_attr<false, true>()));
+    gemm_tc_kernel<false, true><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
+  } else {
+    SKY_CUDA((set_smem_attr<true, true>()));
+    gemm_tc_kernel<true, true><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
+  }
+  count_launches(1);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "gemm_tc_kernel launch");
+  if (p.splits > 1) {
+    const int64_t n = static_cast<int64_t>(M) * N;
+    const int blocks = static_cast<int>(std::min<int64_t>(ceil_div(n / 4 + 1, 256), sms * 8));
+    splitk_reduce_kernel<<<blocks, 256, 0, stream>>>(static_cast<const float*>(ws), p.splits, n,
+                                                     static_cast<float*>(C));
+    count_launches(1);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "splitk_reduce launch");
+  }
+  return SKY_OK;
+}
+
+}  // namespace gemm
+}  // namespace sky

@@ -1,0 +1,435 @@
+// Row-wise and element-wise kernels of the encoder layer: residual +
+// LayerNorm forward and backward (post-LN placement, biased variance),
+// bias + GELU forward and GELU backward, and deterministic column sums (the
+// bias / gamma / beta gradients).
+//
+// All are HBM-bound.  One warp owns one row; every lane moves 16-byte vectors
+// (8 bf16 or 4 fp32) so a warp touches 512 contiguous bytes per access; row
+// statistics are fp32, two-pass in registers, reduced with warp shuffles.
+// Column sums never use floating-point atomics: each CTA writes per-column
+// partials, and a second pass adds them in a fixed order.
+#include "common.cuh"
+#include "rowwise.h"
+
+namespace sky {
+namespace rw {
+
+// 8 consecutive elements <-> fp32 registers (one 16-byte bf16 vector or two
+// 16-byte fp32 vectors).
+__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0], b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
+  const uint4 raw = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&raw);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = __bfloat162float(e[i]);
+}
+__device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
+  reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+__device__ __forceinline__ void store8(__nv_bfloat16* p, const float (&v)[8]) {
+  uint4 raw;
+  __nv_bfloat16* e = reinterpret_cast<__nv_bfloat16*>(&raw);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) e[i] = __float2bfloat16_rn(v[i]);
+  *reinterpret_cast<uint4*>(p) = raw;
+}
+
+constexpr int LN_WARPS = 8;
+constexpr int V = 8;  // elements per lane per chunk; chunk c of a lane starts at (c*32+lane)*8
+
+// y = gamma * (u - mean) * rstd + beta on the fp32 residual sum u.
+template <typename T, int NV>
+__global__ void __launch_bounds__(LN_WARPS * 32) ln_fwd_kernel(
+    const float* __restrict__ u, const T* __restrict__ gamma, const T* __restrict__ beta,
+    int rows, int H, float eps, float* __restrict__ y32, T* __restrict__ yT,
+    float* __restrict__ mean_out, float* __restrict__ rstd_out) {
+  const int lane = threadIdx.x & 31;
+  const int warp = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
+  const int nwarps = gridDim.x * LN_WARPS;
+  float gm[NV][V], bt[NV][V];
+#pragma unroll
+  for (int c = 0; c < NV; ++c) {
+    const int col = (c * 32 + lane) * V;
+    if (col < H) {
+      load8(gamma + col, gm[c]);
+      load8(beta + col, bt[c]);
+    }
+  }
+  const float invH = 1.f / H;
+  for (int row = warp; row < rows; row += nwarps) {
+    float x[NV][V];
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < NV; ++c) {
+      const int col = (c * 32 + lane) * V;
+      if (col < H) {
+        load8(u + (int64_t)row * H + col, x[c]);
+#pragma unroll
+        for (int i = 0; i < V; ++i) s += x[c][i];
+      }
+    }
+    const float mu = warp_sum(s) * invH;
+    float q = 0.f;
+#pragma unroll
+    for (int c = 0; c < NV; ++c) {
+      const int col = (c * 32 + lane) * V;
+      if (col < H) {
+#pragma unroll
+        for (int i = 0; i < V; ++i) {
+          const float d = x[c][i] - mu;
+          q += d * d;
+        }
+      }
+    }
+    const float rs = rsqrtf(warp_sum(q) * invH + eps);
+#pragma unroll
+    for (int c = 0; c < NV; ++c) {
+      const int col = (c * 32 + lane) * V;
+      if (col < H) {
+        float o[V];
+#pragma unroll
+        for (int i = 0; i < V; ++i) o[i] = gm[c][i] * ((x[c][i] - mu) * rs) + bt[c][i];
+        if (y32) store8(y32 + (int64_t)row * H + col, o);
+        if (yT) store8(yT + (int64_t)row * H + col, o);
+      }
+    }
+    if (lane == 0) {
+      mean_out[row] = mu;
+      rstd_out[row] = rs;
+    }
+  }
+}
+
+// Writes this CTA's column sums of `acc` (one per warp, added in warp order)
+// to part[k][blockIdx.x][:].
+template <int NV>
+__device__ __forceinline__ void ln_flush_partial(const float (&acc)[NV][V], int k, float* red,
+                                                 float* __restrict__ part, int H) {
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+#pragma unroll
+  for (int c = 0; c < NV; ++c) {
+    const int col = (c * 32 + lane) * V;
+    if (col < H) {
+#pragma unroll
+      for (int i = 0; i < V; ++i) red[wib * H + col + i] = acc[c][i];
+    }
+  }
+  __syncthreads();
+  for (int col = threadIdx.x; col < H; col += blockDim.x) {
+    float s = 0.f;
+    for (int w = 0; w < LN_WARPS; ++w) s += red[w * H + col];
+    part[((int64_t)k * gridDim.x + blockIdx.x) * H + col] = s;
+  }
+  __syncthreads();
+}
+
+// du = rstd * (g - mean(g) - xhat * mean(g * xhat)), g = dy * gamma, and the
+// per-CTA column partials of dy * xhat, dy and du.
+template <typename TDY, typename T, int NV>
+__global__ void __launch_bounds__(LN_WARPS * 32) ln_bwd_kernel(
+    const TDY* __restrict__ dy, const float* __restrict__ u, const T* __restrict__ gamma,
+    const float* __restrict__ mean, const float* __restrict__ rstd, int rows, int H,
+    float* __restrict__ du32, T* __restrict__ duT, float* __restrict__ part) {
+  extern __shared__ float red[];  // [LN_WARPS][H]
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const int warp = blockIdx.x * LN_WARPS + wib;
+  const int nwarps = gridDim.x * LN_WARPS;
+  float gm[NV][V];
+  float pg[NV][V] = {}, pb[NV][V] = {}, pu[NV][V] = {};
+#pragma unroll
+  for (int c = 0; c < NV; ++c) {
+    const int col = (c * 32 + lane) * V;
+    if (col < H) load8(gamma + col, gm[c]);
+  }
+  const float invH = 1.f / H;
+  for (int row = warp; row < rows; row += nwarps) {
+    const float mu = mean[row], rs = rstd[row];
+    float xh[NV][V], dyv[NV][V];
+    float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+    for (int c = 0; c < NV; ++c) {
+      const int col = (c * 32 + lane) * V;
+      if (col < H) {
+        const int64_t off = (int64_t)row * H + col;
+        load8(u + off, xh[c]);
+        load8(dy + off, dyv[c]);
+#pragma unroll
+        for (int i = 0; i < V; ++i) {
+          xh[c][i] = (xh[c][i] - mu) * rs;
+          const float g = dyv[c][i] * gm[c][i];
+          s1 += g;
+          s2 += g * xh[c][i];
+        }
+      }
+    }
+    const float mg = warp_sum(s1) * invH, mgx = warp_sum(s2) * invH;
+#pragma unroll
+    for (int c = 0; c < NV; ++c) {
+      const int col = (c * 32 + lane) * V;
+      if (col < H) {
+        float o[V];
+#pragma unroll
+        for (int i = 0; i < V; ++i) {
+          o[i] = rs * (dyv[c][i] * gm[c][i] - mg - xh[c][i] * mgx);
+          pg[c][i] += dyv[c][i] * xh[c][i];
+          pb[c][i] += dyv[c][i];
+          pu[c][i] += o[i];
+        }
+        if (du32) store8(du32 + (int64_t)row * H + col, o);
+        if (duT) store8(duT + (int64_t)row * H + col, o);
+      }
+    }
+  }
+  // CTA column partials: [3][gridDim.x][H], summed over the CTA's warps in order
+  ln_flush_partial<NV>(pg, 0, red, part, H);
+  ln_flush_partial<NV>(pb, 1, red, part, H);
+  ln_flush_partial<NV>(pu, 2, red, part, H);
+}
+
+template <typename T>
+__global__ void to_f32_kernel(const T* __restrict__ x, int64_t n, float* __restrict__ out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = to_f32(x[i]);
+}
+
+// out_k[n] = sum_b part[k][b][n] for the non-null outputs (fixed order).
+__global__ void reduce_partials(const float* __restrict__ part, int nblk, int N, float* out0,
+                                float* out1, float* out2) {
+  const int n = blockIdx.x * blockDim.x + threadIdx.x;
+  const int k = blockIdx.y;
+  float* out = k == 0 ? out0 : (k == 1 ? out1 : out2);
+  if (n >= N || out == nullptr) return;
+  const float* p = part + (int64_t)k * nblk * N + n;
+  float s = 0.f;
+  for (int b = 0; b < nblk; ++b) s += p[(int64_t)b * N];
+  out[n] = s;
+}
+
+// Column partial sums of x[T, N]: part[y][n] over rows y, y + gridDim.y, ...
+template <typename T>
+__global__ void colsum_partial(const T* __restrict__ x, int rows, int N, float* __restrict__ part) {
+  const int n = blockIdx.x * blockDim.x + threadIdx.x;
+  if (n >= N) return;
+  float s = 0.f;
+  for (int r = blockIdx.y; r < rows; r += gridDim.y) s += to_f32(x[(int64_t)r * N + n]);
+  part[(int64_t)blockIdx.y * N + n] = s;
+}
+
+template <typename T>
+__global__ void bias_gelu_kernel(const T* __restrict__ z, const T* __restrict__ bias, int64_t n,
+                                 int N, T* __restrict__ hpre, T* __restrict__ g) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const float h = to_f32(z[i]) + (bias ? to_f32(bias[i % N]) : 0.f);
+    hpre[i] = from_f32<T>(h);
+    g[i] = from_f32<T>(gelu_f(h));
+  }
+}
+
+template <typename T>
+__global__ void gelu_bwd_kernel(const T* __restrict__ dg, const T* __restrict__ hpre, int64_t n,
+                                T* __restrict__ dh) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    dh[i] = from_f32<T>(to_f32(dg[i]) * gelu_grad_f(to_f32(hpre[i])));
+}
+
+int ln_blocks(int rows) {
+  const int want = ceil_div(rows, LN_WARPS);
+  const int cap = 4 * (sm_count() > 0 ? sm_count() : 148);
+  return want < cap ? want : cap;
+}
+
+template <typename T, int NV>
+void ln_fwd_launch(const float* u, const void* gm, const void* bt, int rows, int H, float eps,
+                   float* y32, void* y, float* mean, float* rstd, cudaStream_t st) {
+  ln_fwd_kernel<T, NV><<<ln_blocks(rows), LN_WARPS * 32, 0, st>>>(
+      u, static_cast<const T*>(gm), static_cast<const T*>(bt), rows, H, eps, y32,
+      static_cast<T*>(y), mean, rstd);
+}
+template <typename TDY, typename T, int NV>
+void ln_bwd_launch(const void* dy, const float* u, const void* gm, const float* mean,
+                   const float* rstd, int rows, int H, float* du32, void* du, float* part,
+                   int nblk, cudaStream_t st) {
+  const size_t smem = (size_t)LN_WARPS * H * sizeof(float);
+  if (smem > 48 * 1024)
+    cudaFuncSetAttribute(ln_bwd_kernel<TDY, T, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+  ln_bwd_kernel<TDY, T, NV><<<nblk, LN_WARPS * 32, smem, st>>>(
+      static_cast<const TDY*>(dy), u, static_cast<const T*>(gm), mean, rstd, rows, H, du32,
+      static_cast<T*>(du), part);
+}
+
+}  // namespace rw
+
+// ------------------------------------------------------------------- host
+namespace {
+constexpr int kMaxNV = 8;
+int lane_vectors(int H) { return ceil_div(H, 32 * rw::V); }
+}  // namespace
+
+#define SKY_NV_DISPATCH(NVV, CALL) \
+  switch (NVV) {                   \
+    case 1: CALL(1); break;        \
+    case 2: CALL(2); break;        \
+    case 3: CALL(3); break;        \
+    case 4: CALL(4); break;        \
+    case 5: CALL(5); break;        \
+    case 6: CALL(6); break;        \
+    case 7: CALL(7); break;        \
+    default: CALL(8); break;       \
+  }
+
+sky_status layernorm_fwd(const float* u, const void* gamma, const void* beta, int rows, int H,
+                         float eps, sky_dtype dt, float* y32, void* y, float* mean, float* rstd,
+                         cudaStream_t st) {
+  SKY_CHECK(H % rw::V == 0 && lane_vectors(H) <= kMaxNV && (dt == SKY_DTYPE_BF16 || H <= 1024),
+            SKY_ERR_UNSUPPORTED, "LayerNorm width %d unsupported", H);
+  SKY_CHECK(y32 || y, SKY_ERR_INVALID_ARG, "LayerNorm forward needs an output");
+  const int nv = lane_vectors(H);
+  if (dt == SKY_DTYPE_BF16) {
+#define LNF(NV) rw::ln_fwd_launch<__nv_bfloat16, NV>(u, gamma, beta, rows, H, eps, y32, y, mean, rstd, st)
+    SKY_NV_DISPATCH(nv, LNF)
+#undef LNF
+  } else {
+    // fp32 slices: the dtype output is itself fp32, so one store suffices
+    float* only = y32 ? y32 : static_cast<float*>(y);
+#define LNF(NV) rw::ln_fwd_launch<float, NV>(u, gamma, beta, rows, H, eps, only, nullptr, mean, rstd, st)
+    SKY_NV_DISPATCH(nv, LNF)
+#undef LNF
+    if (y32 && y && y != y32)
+      SKY_CUDA(cudaMemcpyAsync(y, y32, (size_t)rows * H * 4, cudaMemcpyDeviceToDevice, st));
+  }
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm forward launch");
+}
+
+size_t layernorm_bwd_ws(int rows, int H) {
+  return (size_t)3 * rw::ln_blocks(rows) * H * sizeof(float);
+}
+
+sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* u, const void* gamma,
+                         const float* mean, const float* rstd, int rows, int H, sky_dtype dt,
+                         float* du32, void* du, float* dgamma, float* dbeta, float* dbias,
+                         void* ws, size_t ws_bytes, cudaStream_t st) {
+  SKY_CHECK(H % rw::V == 0 && lane_vectors(H) <= kMaxNV && (dt == SKY_DTYPE_BF16 || H <= 1024),
+            SKY_ERR_UNSUPPORTED, "LayerNorm width %d unsupported", H);
+  SKY_CHECK(du32 || du, SKY_ERR_INVALID_ARG, "LayerNorm backward needs an output");
+  const int nblk = rw::ln_blocks(rows);
+  SKY_CHECK(ws && ws_bytes >= (size_t)3 * nblk * H * sizeof(float), SKY_ERR_INVALID_ARG,
+            "LayerNorm backward workspace too small");
+  float* part = static_cast<float*>(ws);
+  const int nv = lane_vectors(H);
+  if (dt == SKY_DTYPE_BF16) {
+    if (dy_dt == SKY_DTYPE_BF16) {
+#define LNB(NV) rw::ln_bwd_launch<__nv_bfloat16, __nv_bfloat16, NV>(dy, u, gamma, mean, rstd, rows, H, du32, du, part, nblk, st)
+      SKY_NV_DISPATCH(nv, LNB)
+#undef LNB
+    } else {
+#define LNB(NV) rw::ln_bwd_launch<float, __nv_bfloat16, NV>(dy, u, gamma, mean, rstd, rows, H, du32, du, part, nblk, st)
+      SKY_NV_DISPATCH(nv, LNB)
+#undef LNB
+    }
+  } else {
+    float* only = du32 ? du32 : static_cast<float*>(du);
+#define LNB(NV) rw::ln_bwd_launch<float, float, NV>(dy, u, gamma, mean, rstd, rows, H, only, nullptr, part, nblk, st)
+    SKY_NV_DISPATCH(nv, LNB)
+#undef LNB
+    if (du32 && du && du != du32)
+      SKY_CUDA(cudaMemcpyAsync(du, du32, (size_t)rows * H * 4, cudaMemcpyDeviceToDevice, st));
+  }
+  dim3 grid(ceil_div(H, 256), 3);
+  rw::reduce_partials<<<grid, 256, 0, st>>>(part, nblk, H, dgamma, dbeta, dbias);
+  count_launches(2);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward launch");
+}
+
+sky_status to_f32(const void* x, int64_t n, sky_dtype dt, float* out, cudaStream_t st) {
+  if (n <= 0) return SKY_OK;
+  const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
+  if (dt == SKY_DTYPE_BF16)
+    rw::to_f32_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(x), n, out);
+  else
+    rw::to_f32_kernel<float><<<blocks, 256, 0, st>>>(static_cast<const float*>(x), n, out);
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "widen launch");
+}
+
+namespace {
+int colsum_row_groups(int rows, int N) {
+  const int cb = ceil_div(N, 256);
+  int g = 4 * (sm_count() > 0 ? sm_count() : 148) / cb;
+  if (g < 1) g = 1;
+  if (g > rows) g = rows;
+  return g;
+}
+}  // namespace
+
+size_t column_sum_ws(int rows, int N) {
+  return (size_t)colsum_row_groups(rows, N) * N * sizeof(float);
+}
+
+sky_status column_sum(const void* x, int rows, int N, sky_dtype dt, float* out, void* ws,
+                      size_t ws_bytes, cudaStream_t st) {
+  const int groups = colsum_row_groups(rows, N);
+  SKY_CHECK(ws && ws_bytes >= (size_t)groups * N * sizeof(float), SKY_ERR_INVALID_ARG,
+            "column-sum workspace too small");
+  float* part = static_cast<float*>(ws);
+  dim3 grid(ceil_div(N, 256), groups);
+  if (dt == SKY_DTYPE_BF16)
+    rw::colsum_partial<__nv_bfloat16><<<grid, 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(x), rows, N, part);
+  else
+    rw::colsum_partial<float><<<grid, 256, 0, st>>>(static_cast<const float*>(x), rows, N, part);
+  rw::reduce_partials<<<dim3(ceil_div(N, 256), 1), 256, 0, st>>>(part, groups, N, out, nullptr,
+                                                                 nullptr);
+  count_launches(2);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "column sum launch");
+}
+
+sky_status bias_gelu_fwd(const void* z, const void* bias, int rows, int N, sky_dtype dt,
+                         void* hpre, void* g, cudaStream_t st) {
+  const int64_t n = (int64_t)rows * N;
+  const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
+  if (dt == SKY_DTYPE_BF16)
+    rw::bias_gelu_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(z), static_cast<const __nv_bfloat16*>(bias), n, N,
+        static_cast<__nv_bfloat16*>(hpre), static_cast<__nv_bfloat16*>(g));
+  else
+    rw::bias_gelu_kernel<float><<<blocks, 256, 0, st>>>(static_cast<const float*>(z),
+                                                        static_cast<const float*>(bias), n, N,
+                                                        static_cast<float*>(hpre),
+                                                        static_cast<float*>(g));
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "bias+GELU launch");
+}
+
+sky_status gelu_bwd(const void* dg, const void* hpre, int rows, int N, sky_dtype dt, void* dh,
+                    cudaStream_t st) {
+  const int64_t n = (int64_t)rows * N;
+  const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
+  if (dt == SKY_DTYPE_BF16)
+    rw::gelu_bwd_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(dg), static_cast<const __nv_bfloat16*>(hpre), n,
+        static_cast<__nv_bfloat16*>(dh));
+  else
+    rw::gelu_bwd_kernel<float><<<blocks, 256, 0, st>>>(static_cast<const float*>(dg),
+                                                       static_cast<const float*>(hpre), n,
+                                                       static_cast<float*>(dh));
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "GELU backward launch");
+}
+
+}  // namespace sky

@@ -1,0 +1,33 @@
+// Internal launchers of the attention and row-wise kernels.
+#pragma once
+#include <cuda_runtime.h>
+
+#include "../../include/sky_ops.h"
+
+namespace sky {
+
+sky_status attention_fwd(const void* qkv, const int32_t* lens, int B, int S, int H, int A,
+                         sky_dtype dt, void* ctx, float* lse, int32_t* status, cudaStream_t st);
+size_t attention_bwd_ws(int B, int S, int A);
+sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, const float* lse,
+                         const int32_t* lens, int B, int S, int H, int A, sky_dtype dt, void* dqkv,
+                         float* delta, int32_t* status, cudaStream_t st);
+
+sky_status layernorm_fwd(const float* u, const void* gamma, const void* beta, int rows, int H,
+                         float eps, sky_dtype dt, float* y32, void* y, float* mean, float* rstd,
+                         cudaStream_t st);
+size_t layernorm_bwd_ws(int rows, int H);
+sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* u, const void* gamma,
+                         const float* mean, const float* rstd, int rows, int H, sky_dtype dt,
+                         float* du32, void* du, float* dgamma, float* dbeta, float* dbias,
+                         void* ws, size_t ws_bytes, cudaStream_t st);
+sky_status to_f32(const void* x, int64_t n, sky_dtype dt, float* out, cudaStream_t st);
+size_t column_sum_ws(int rows, int N);
+sky_status column_sum(const void* x, int rows, int N, sky_dtype dt, float* out, void* ws,
+                      size_t ws_bytes, cudaStream_t st);
+sky_status bias_gelu_fwd(const void* z, const void* bias, int rows, int N, sky_dtype dt,
+                         void* hpre, void* g, cudaStream_t st);
+sky_status gelu_bwd(const void* dg, const void* hpre, int rows, int N, sky_dtype dt, void* dh,
+                    cudaStream_t st);
+
+}  // namespace sky

@@ -1,0 +1,916 @@
+// Slice runtime and the C ABI (sky_slice.h, sky_ops.h).
+//
+// A slice owns the layers [l0, l1) of the encoder (the partition unit of
+// Sec. IV-D).  At create it makes one device allocation holding, per layer,
+// the 12 parameters (slice dtype), their fp32 gradients and the activation
+// stash the backward pass needs (Sec. IV-B counts exactly these: inputs,
+// weights, gradients and outputs), plus one shared workspace.  forward runs
+// the layers in order and leaves each layer's intermediates in its stash;
+// backward walks the layers in reverse (Sec. III) reading that stash.  Every
+// launch goes on the caller's stream; nothing synchronises the host except the
+// calls documented as synchronous.
+#include <algorithm>
+#include <atomic>
+#include <cstdarg>
+#include <cstring>
+#include <exception>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "gemm.h"
+#include "rowwise.h"
+
+namespace sky {
+
+namespace {
+thread_local std::string g_last_error;
+uint64_t g_alloc_cap = 0;
+std::atomic<int64_t> g_launches{0};
+}  // namespace
+
+void count_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+void set_error(const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+}
+
+sky_status cuda_fail(cudaError_t e, const char* what) {
+  set_error("%s: %s", what, cudaGetErrorString(e));
+  return e == cudaErrorMemoryAllocation ? SKY_ERR_OOM : SKY_ERR_CUDA;
+}
+
+int sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  static int cache[64] = {0};
+  if (dev < 0 || dev >= 64) return 0;
+  if (cache[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    cache[dev] = n;
+  }
+  return cache[dev];
+}
+
+// ---------------------------------------------------------------- profiling
+struct ProfRecord {
+  int cat;
+  cudaEvent_t start, stop;
+  double flops, bytes;
+};
+enum ProfCat { P_GEMM_FWD, P_GEMM_DGRAD, P_GEMM_WGRAD, P_ATTN_FWD, P_ATTN_BWD, P_LN_FWD,
+               P_LN_BWD, P_COLSUM, P_COPY, P_NCAT };
+static const char* kCatNames[P_NCAT] = {"gemm_fwd", "gemm_dgrad", "gemm_wgrad", "attn_fwd",
+                                        "attn_bwd", "ln_fwd", "ln_bwd", "colsum", "copy"};
+
+// Per-layer parameters, gradients and the activation stash.  The residual
+// stream (layer input X, the residual sums U1 and U2, the LayerNorm output X1)
+// is kept in fp32; tensors that feed a bf16 contraction have a copy in the
+// slice dtype (for fp32 slices the two are the same buffer).
+struct LayerBufs {
+  void* p[SKY_NUM_PARAMS];
+  float* g[SKY_NUM_PARAMS];
+  void *Xb, *QKV, *ctx, *X1b, *Hpre, *G;
+  float *X32, *U1, *X1_32, *U2;
+  float *lse, *mean1, *rstd1, *mean2, *rstd2;
+};
+
+}  // namespace sky
+
+struct sky_slice {
+  sky_slice_config cfg;
+  int L, H, A, F, D;
+  size_t esz;
+  int64_t maxT;
+  int device;
+  void* arena = nullptr;
+  uint64_t param_bytes = 0, grad_bytes = 0, stash_bytes = 0, ws_bytes_total = 0;
+  std::vector<sky::LayerBufs> layers;
+  float *g32a, *g32b, *dU2_32, *dX1_32, *dU1_32;  // fp32 gradient stream
+  void *dU2b, *dU1b, *dH, *dctx, *dqkv;           // dtype copies / branch gradients
+  float* delta;
+  void* ws;
+  size_t ws_bytes;
+  int32_t* d_status;
+  // state of the most recent forward
+  bool have_fwd = false;
+  int B = 0, S = 0;
+  const int32_t* d_len = nullptr;
+  cudaStream_t last_stream = nullptr;
+  // profiling
+  bool prof = false;
+  std::vector<sky::ProfRecord> recs;
+  std::vector<cudaEvent_t> event_pool;
+  size_t event_next = 0;
+  double cat_ms[sky::P_NCAT] = {0};
+  double cat_flops[sky::P_NCAT] = {0};
+  double cat_bytes[sky::P_NCAT] = {0};
+  int64_t cat_n[sky::P_NCAT] = {0};
+};
+
+namespace sky {
+namespace {
+
+size_t param_elems(const sky_slice* s, int k) {
+  const size_t H = s->H, F = s->F;
+  switch (k) {
+    case 0: return 3 * H * H;
+    case 1: return 3 * H;
+    case 2: return H * H;
+    case 6: return F * H;
+    case 7: return F;
+    case 8: return H * F;
+    default: return H;
+  }
+}
+
+size_t align_up(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Scratch needed by the backward pass at T tokens (shared by all steps).
+size_t workspace_need(const sky_slice* s, int64_t T) {
+  const int H = s->H, F = s->F;
+  size_t need = 0;
+  if (s->cfg.dtype == SKY_DTYPE_BF16) {
+    const int64_t shapes[4][2] = {{3 * H, H}, {H, H}, {F, H}, {H, F}};
+    for (auto& sh : shapes)
+      need = std::max(need, gemm::workspace_bytes(SKY_GEMM_XTW, (int)sh[0], (int)sh[1], (int)T, true));
+  }
+  need = std::max(need, layernorm_bwd_ws((int)T, H));
+  need = std::max(need, column_sum_ws((int)T, F));
+  need = std::max(need, column_sum_ws((int)T, 3 * H));
+  return need;
+}
+
+cudaEvent_t next_event(sky_slice* s) {
+  if (s->event_next == s->event_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    s->event_pool.push_back(e);
+  }
+  return s->event_pool[s->event_next++];
+}
+
+// Brackets one launch with CUDA events when profiling is on.
+struct Timed {
+  sky_slice* s;
+  cudaStream_t st;
+  ProfRecord r{};
+  Timed(sky_slice* s_, cudaStream_t st_, int cat, double flops, double bytes) : s(s_), st(st_) {
+    if (!s->prof) return;
+    r.cat = cat; r.flops = flops; r.bytes = bytes;
+    r.start = next_event(s);
+    r.stop = next_event(s);
+    if (r.start) cudaEventRecord(r.start, st);
+  }
+  ~Timed() {
+    if (!s->prof || !r.start || !r.stop) return;
+    cudaEventRecord(r.stop, st);
+    s->recs.push_back(r);
+  }
+};
+
+sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, int M, int N,
+                    int K, const void* A, const void* Bm, void* C, bool out_f32, int epi,
+                    const void* bias, const void* aux, void* aux_out) {
+  Timed t(s, st, cat, 2.0 * M * N * K, 0);
+  if (s->cfg.dtype == SKY_DTYPE_BF16)
+    return gemm::launch_bf16(form, M, N, K, A, Bm, C, out_f32, epi, bias, aux, aux_out, s->ws,
+                             s->ws_bytes, s->d_status, st);
+  return gemm::launch_f32(form, M, N, K, static_cast<const float*>(A),
+                          static_cast<const float*>(Bm), static_cast<float*>(C), epi,
+                          static_cast<const float*>(bias), static_cast<const float*>(aux),
+                          static_cast<float*>(aux_out), st);
+}
+
+#define SKY_TRY(call)                   \
+  do {                                  \
+    sky_status st_ = (call);            \
+    if (st_ != SKY_OK) return st_;      \
+  } while (0)
+
+// ------------------------------------------------------------------ forward
+// One layer, steps a1..a8.  y_out == nullptr: write the next layer's Xb/X32.
+sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
+  LayerBufs& Lb = s->layers[i];
+  const int B = s->B, S = s->S, H = s->H, A = s->A, F = s->F;
+  const int T = B * S;
+  const sky_dtype dt = s->cfg.dtype;
+  const double e = (double)s->esz;
+  // a1: QKV = X Wqkv^T + bqkv
+  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, 3 * H, H, Lb.Xb, Lb.p[0], Lb.QKV, false,
+                   SKY_EPI_STORE, Lb.p[1], nullptr, nullptr));
+  // a2: masked scaled dot-product attention (Eq. 1)
+  {
+    Timed t(s, st, P_ATTN_FWD, 4.0 * H * S * (double)T, e * T * 4.0 * H);
+    SKY_TRY(attention_fwd(Lb.QKV, s->d_len, B, S, H, A, dt, Lb.ctx, Lb.lse, s->d_status, st));
+  }
+  // a3 + residual: U1 = ctx Wo^T + bo + X  (fp32)
+  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, H, Lb.ctx, Lb.p[2], Lb.U1, true,
+                   SKY_EPI_RESIDUAL, Lb.p[3], Lb.X32, nullptr));
+  // a4: X1 = LN(U1)
+  {
+    Timed t(s, st, P_LN_FWD, 0, 4.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_fwd(Lb.U1, Lb.p[4], Lb.p[5], T, H, s->cfg.ln_eps, dt,
+                          dt == SKY_DTYPE_BF16 ? Lb.X1_32 : nullptr, Lb.X1b, Lb.mean1, Lb.rstd1,
+                          st));
+  }
+  // a5 + a6: Hpre = X1 W1^T + b1, G = GELU(Hpre) (fused epilogue)
+  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, F, H, Lb.X1b, Lb.p[6], Lb.Hpre, false,
+                   SKY_EPI_BIAS_GELU, Lb.p[7], nullptr, Lb.G));
+  // a7 + residual: U2 = G W2^T + b2 + X1  (fp32)
+  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, F, Lb.G, Lb.p[8], Lb.U2, true,
+                   SKY_EPI_RESIDUAL, Lb.p[9], Lb.X1_32, nullptr));
+  // a8: Y = LN(U2) -> next layer's input (fp32 + dtype copy) or the caller's y
+  {
+    Timed t(s, st, P_LN_FWD, 0, 4.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
+    if (y_out) {
+      SKY_TRY(layernorm_fwd(Lb.U2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, nullptr, y_out,
+                            Lb.mean2, Lb.rstd2, st));
+    } else {
+      LayerBufs& Nx = s->layers[i + 1];
+      SKY_TRY(layernorm_fwd(Lb.U2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt,
+                            dt == SKY_DTYPE_BF16 ? Nx.X32 : nullptr, Nx.Xb, Lb.mean2, Lb.rstd2,
+                            st));
+    }
+  }
+  return SKY_OK;
+}
+
+// ----------------------------------------------------------------- backward
+// One layer, steps a9..a16.  dY: dtype (top layer, from the caller) or fp32;
+// dX: fp32 stream buffer, or the caller's dx (dtype) for the first layer.
+sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, void* dX,
+                          bool dx_f32, cudaStream_t st) {
+  LayerBufs& Lb = s->layers[i];
+  const int B = s->B, S = s->S, H = s->H, A = s->A, F = s->F;
+  const int T = B * S;
+  const sky_dtype dt = s->cfg.dtype;
+  const bool bf = dt == SKY_DTYPE_BF16;
+  const double e = (double)s->esz;
+  const double dye = dy_dt == SKY_DTYPE_BF16 ? 2.0 : 4.0;
+  // a9: LN2 backward -> dU2 (fp32 + dtype), dgamma2, dbeta2, db2
+  {
+    Timed t(s, st, P_LN_BWD, 0, (dye + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_bwd(dY, dy_dt, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
+                          bf ? s->dU2_32 : nullptr, s->dU2b, Lb.g[10], Lb.g[11], Lb.g[9], s->ws,
+                          s->ws_bytes, st));
+  }
+  // a10 + a11: dHpre = (dU2 W2) * GELU'(Hpre);  dW2 = dU2^T G
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
+                   SKY_EPI_GELU_BWD, nullptr, Lb.Hpre, nullptr));
+  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  {
+    Timed t(s, st, P_COLSUM, 0, e * T * F);
+    SKY_TRY(column_sum(s->dH, T, F, dt, Lb.g[7], s->ws, s->ws_bytes, st));
+  }
+  // a12: dX1 = dHpre W1 + dU2 (fp32);  dW1 = dHpre^T X1
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dX1_32, true,
+                   SKY_EPI_RESIDUAL, nullptr, s->dU2_32, nullptr));
+  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, F, H, T, s->dH, Lb.X1b, Lb.g[6], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  // a13: LN1 backward -> dU1 (fp32 + dtype), dgamma1, dbeta1, dbo
+  {
+    Timed t(s, st, P_LN_BWD, 0, (4.0 + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_bwd(s->dX1_32, SKY_DTYPE_FP32, Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H,
+                          dt, bf ? s->dU1_32 : nullptr, s->dU1b, Lb.g[4], Lb.g[5], Lb.g[3], s->ws,
+                          s->ws_bytes, st));
+  }
+  // a14: dctx = dU1 Wo;  dWo = dU1^T ctx
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, H, s->dU1b, Lb.p[2], s->dctx, false,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, H, T, s->dU1b, Lb.ctx, Lb.g[2], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  // a15: attention backward -> dQKV
+  {
+    Timed t(s, st, P_ATTN_BWD, 8.0 * H * S * (double)T, e * T * 8.0 * H);
+    SKY_TRY(attention_bwd(Lb.QKV, Lb.ctx, s->dctx, Lb.lse, s->d_len, B, S, H, A, dt, s->dqkv,
+                          s->delta, s->d_status, st));
+  }
+  {
+    Timed t(s, st, P_COLSUM, 0, e * T * 3.0 * H);
+    SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], s->ws, s->ws_bytes, st));
+  }
+  // a16: dX = dQKV Wqkv + dU1;  dWqkv = dQKV^T X
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, 3 * H, s->dqkv, Lb.p[0], dX, dx_f32,
+                   SKY_EPI_RESIDUAL, nullptr, bf ? s->dU1_32 : s->dU1b, nullptr));
+  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, 3 * H, H, T, s->dqkv, Lb.Xb, Lb.g[0], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  return SKY_OK;
+}
+
+sky_status forward_all(sky_slice* s, const void* x, void* y, cudaStream_t st,
+                       std::vector<cudaEvent_t>* marks) {
+  const int64_t n = (int64_t)s->B * s->S * s->H;
+  {
+    Timed t(s, st, P_COPY, 0, (2.0 * s->esz + (s->esz == 2 ? 6.0 : 0.0)) * n);
+    SKY_CUDA(cudaMemcpyAsync(s->layers[0].Xb, x, n * s->esz, cudaMemcpyDeviceToDevice, st));
+    if (s->cfg.dtype == SKY_DTYPE_BF16)
+      SKY_TRY(to_f32(x, n, s->cfg.dtype, s->layers[0].X32, st));
+  }
+  for (int i = 0; i < s->L; ++i) {
+    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i], st));
+    SKY_TRY(forward_layer(s, i, i + 1 < s->L ? nullptr : y, st));
+    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
+  }
+  return SKY_OK;
+}
+
+sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
+                        std::vector<cudaEvent_t>* marks) {
+  const void* cur = dy;
+  sky_dtype cur_dt = s->cfg.dtype;
+  for (int i = s->L - 1; i >= 0; --i) {
+    const bool last = i == 0;
+    void* out = last ? dx : ((s->L - 1 - i) % 2 == 0 ? (void*)s->g32a : (void*)s->g32b);
+    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i], st));
+    SKY_TRY(backward_layer(s, i, cur, cur_dt, out, !last, st));
+    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
+    cur = out;
+    cur_dt = SKY_DTYPE_FP32;
+  }
+  return SKY_OK;
+}
+
+int layer_index(const sky_slice* s, int32_t layer) {
+  if (layer < s->cfg.layer_begin || layer >= s->cfg.layer_end) return -1;
+  return layer - s->cfg.layer_begin;
+}
+
+__global__ void fill_pattern(void* p, int64_t n, int bf16, float scale, uint32_t seed) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    uint32_t h = (uint32_t)i * 2654435761u ^ seed;
+    h ^= h >> 15; h *= 2246822519u; h ^= h >> 13; h *= 3266489917u; h ^= h >> 16;
+    const float v = scale * ((h & 0xFFFFFF) / 8388608.0f - 1.0f);
+    if (bf16) static_cast<__nv_bfloat16*>(p)[i] = __float2bfloat16_rn(v);
+    else static_cast<float*>(p)[i] = v;
+  }
+}
+__global__ void fill_int(int32_t* p, int n, int v) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) p[i] = v;
+}
+
+}  // namespace
+}  // namespace sky
+
+using namespace sky;
+
+#define ABI_GUARD_BEGIN try {
+#define ABI_GUARD_END                                              \
+  }                                                                \
+  catch (const std::bad_alloc&) {                                  \
+    set_error("host allocation failed");                           \
+    return SKY_ERR_OOM;                                            \
+  }                                                                \
+  catch (const std::exception& ex) {                               \
+    set_error("internal error: %s", ex.what());                    \
+    return SKY_ERR_CUDA;                                           \
+  }                                                                \
+  catch (...) {                                                    \
+    set_error("internal error");                                   \
+    return SKY_ERR_CUDA;                                           \
+  }
+
+extern "C" {
+
+void sky_debug_set_alloc_cap(uint64_t bytes) { g_alloc_cap = bytes; }
+
+int64_t sky_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+const char* sky_status_string(sky_status st) {
+  switch (st) {
+    case SKY_OK: return "SKY_OK";
+    case SKY_ERR_INVALID_ARG: return "SKY_ERR_INVALID_ARG";
+    case SKY_ERR_OOM: return "SKY_ERR_OOM";
+    case SKY_ERR_CUDA: return "SKY_ERR_CUDA";
+    case SKY_ERR_STATE: return "SKY_ERR_STATE";
+    case SKY_ERR_TIMEOUT: return "SKY_ERR_TIMEOUT";
+    case SKY_ERR_UNSUPPORTED: return "SKY_ERR_UNSUPPORTED";
+  }
+  return "SKY_ERR_UNKNOWN";
+}
+
+const char* sky_last_error(void) { return g_last_error.c_str(); }
+
+int32_t sky_device_sm_count(void) { return sm_count(); }
+
+// Sizes of the arena carved at create, computed on the host only.
+static sky_status plan_slice(sky_slice* s, size_t* total) {
+  const sky_slice_config& c = s->cfg;
+  const int64_t T = (int64_t)c.max_batch * c.max_seq;
+  s->maxT = T;
+  size_t pb = 0, gb = 0;
+  for (int k = 0; k < SKY_NUM_PARAMS; ++k) {
+    pb += align_up(param_elems(s, k) * s->esz);
+    gb += align_up(param_elems(s, k) * 4);
+  }
+  const size_t th = align_up((size_t)T * s->H * s->esz);
+  const size_t t32 = align_up((size_t)T * s->H * 4);
+  const bool bf = c.dtype == SKY_DTYPE_BF16;
+  const size_t lse = align_up((size_t)c.max_batch * s->A * c.max_seq * 4);
+  // Xb ctx X1b | QKV | Hpre G | U1 U2 (+ X32 X1_32 for bf16) | lse | 4 stats
+  const size_t stash = 3 * th + align_up((size_t)T * 3 * s->H * s->esz) +
+                       2 * align_up((size_t)T * s->F * s->esz) + (bf ? 4 : 2) * t32 + lse +
+                       4 * align_up((size_t)T * 4);
+  s->param_bytes = pb * s->L;
+  s->grad_bytes = gb * s->L;
+  s->stash_bytes = stash * s->L;
+  s->ws_bytes = align_up(workspace_need(s, T));
+  // g32a g32b dU2_32 dX1_32 dU1_32 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | status
+  const size_t wk = 5 * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
+                    align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes + 256;
+  s->ws_bytes_total = wk;
+  *total = s->param_bytes + s->grad_bytes + s->stash_bytes + wk;
+  return SKY_OK;
+}
+
+sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(cfg && out, SKY_ERR_INVALID_ARG, "null argument");
+  *out = nullptr;
+  const sky_slice_config& c = *cfg;
+  SKY_CHECK(c.width > 0 && c.heads > 0 && c.ffn > 0 && c.max_batch > 0 && c.max_seq > 0,
+            SKY_ERR_INVALID_ARG, "sizes must be positive");
+  SKY_CHECK(c.width % c.heads == 0, SKY_ERR_INVALID_ARG, "width %d not divisible by heads %d",
+            c.width, c.heads);
+  SKY_CHECK(c.layer_begin >= 0 && c.layer_begin < c.layer_end, SKY_ERR_INVALID_ARG,
+            "need 0 <= layer_begin < layer_end");
+  SKY_CHECK(c.dtype == SKY_DTYPE_BF16 || c.dtype == SKY_DTYPE_FP32, SKY_ERR_INVALID_ARG,
+            "unknown dtype");
+  SKY_CHECK(c.ln_eps >= 0.f, SKY_ERR_INVALID_ARG, "ln_eps must be >= 0");
+  const int D = c.width / c.heads;
+  if (c.dtype == SKY_DTYPE_BF16) {
+    SKY_CHECK(D == 64, SKY_ERR_UNSUPPORTED, "bf16 slices need head dim 64 (got %d)", D);
+    SKY_CHECK(c.width % 8 == 0 && c.ffn % 8 == 0, SKY_ERR_UNSUPPORTED,
+              "bf16 slices need width and ffn multiples of 8");
+    SKY_CHECK(c.width <= 2048, SKY_ERR_UNSUPPORTED, "width above 2048 not supported");
+  } else {
+    SKY_CHECK(D <= 128 && c.width % 4 == 0 && c.width <= 1024, SKY_ERR_UNSUPPORTED,
+              "fp32 slices need head dim <= 128 and width <= 1024, multiple of 4");
+  }
+  SKY_CHECK((int64_t)c.max_batch * c.max_seq <= (int64_t)1 << 30, SKY_ERR_INVALID_ARG,
+            "max_batch * max_seq too large");
+  auto* s = new sky_slice();
+  s->cfg = c;
+  s->L = c.layer_end - c.layer_begin;
+  s->H = c.width; s->A = c.heads; s->F = c.ffn; s->D = D;
+  s->esz = c.dtype == SKY_DTYPE_BF16 ? 2 : 4;
+  size_t total = 0;
+  plan_slice(s, &total);
+  if (g_alloc_cap && total > g_alloc_cap) {
+    set_error("slice needs %zu bytes, above the allocation cap %llu", total,
+              (unsigned long long)g_alloc_cap);
+    delete s;
+    return SKY_ERR_OOM;
+  }
+  if (cudaGetDevice(&s->device) != cudaSuccess) {
+    set_error("no CUDA device");
+    delete s;
+    return SKY_ERR_CUDA;
+  }
+  cudaError_t e = cudaMalloc(&s->arena, total);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    set_error("cudaMalloc(%zu): %s", total, cudaGetErrorString(e));
+    delete s;
+    return e == cudaErrorMemoryAllocation ? SKY_ERR_OOM : SKY_ERR_CUDA;
+  }
+  e = cudaMemset(s->arena, 0, total);
+  if (e != cudaSuccess) {
+    cudaFree(s->arena);
+    delete s;
+    return cuda_fail(e, "cudaMemset");
+  }
+  char* p = static_cast<char*>(s->arena);
+  auto take = [&](size_t bytes) {
+    void* r = p;
+    p += align_up(bytes);
+    return r;
+  };
+  const int64_t T = s->maxT;
+  const size_t th = (size_t)T * s->H * s->esz;
+  const size_t t32 = (size_t)T * s->H * 4;
+  const bool bf = c.dtype == SKY_DTYPE_BF16;
+  const size_t lse_b = (size_t)c.max_batch * s->A * c.max_seq * 4;
+  s->layers.resize(s->L);
+  for (auto& Lb : s->layers) {
+    for (int k = 0; k < SKY_NUM_PARAMS; ++k) Lb.p[k] = take(param_elems(s, k) * s->esz);
+    for (int k = 0; k < SKY_NUM_PARAMS; ++k) Lb.g[k] = static_cast<float*>(take(param_elems(s, k) * 4));
+    Lb.Xb = take(th); Lb.ctx = take(th); Lb.X1b = take(th);
+    Lb.QKV = take((size_t)T * 3 * s->H * s->esz);
+    Lb.Hpre = take((size_t)T * s->F * s->esz);
+    Lb.G = take((size_t)T * s->F * s->esz);
+    Lb.U1 = static_cast<float*>(take(t32));
+    Lb.U2 = static_cast<float*>(take(t32));
+    Lb.X32 = bf ? static_cast<float*>(take(t32)) : static_cast<float*>(Lb.Xb);
+    Lb.X1_32 = bf ? static_cast<float*>(take(t32)) : static_cast<float*>(Lb.X1b);
+    Lb.lse = static_cast<float*>(take(lse_b));
+    Lb.mean1 = static_cast<float*>(take((size_t)T * 4));
+    Lb.rstd1 = static_cast<float*>(take((size_t)T * 4));
+    Lb.mean2 = static_cast<float*>(take((size_t)T * 4));
+    Lb.rstd2 = static_cast<float*>(take((size_t)T * 4));
+  }
+  s->g32a = static_cast<float*>(take(t32));
+  s->g32b = static_cast<float*>(take(t32));
+  s->dU2_32 = static_cast<float*>(take(t32));
+  s->dX1_32 = static_cast<float*>(take(t32));
+  s->dU1_32 = static_cast<float*>(take(t32));
+  s->dU2b = bf ? take(th) : s->dU2_32;
+  s->dU1b = bf ? take(th) : s->dU1_32;
+  s->dctx = take(th);
+  s->dH = take((size_t)T * s->F * s->esz);
+  s->dqkv = take((size_t)T * 3 * s->H * s->esz);
+  s->delta = static_cast<float*>(take(lse_b));
+  s->ws = take(s->ws_bytes);
+  s->d_status = static_cast<int32_t*>(take(4));
+  *out = s;
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_destroy(sky_slice* s) {
+  ABI_GUARD_BEGIN
+  if (!s) return SKY_OK;
+  cudaDeviceSynchronize();
+  for (auto e : s->event_pool) cudaEventDestroy(e);
+  if (s->arena) cudaFree(s->arena);
+  delete s;
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+static sky_status copy_tensors(sky_slice* s, int32_t layer, const void* const* src,
+                               void* const* dst, int on_device, bool to_slice, bool grads) {
+  SKY_CHECK(s && (to_slice ? (const void*)src : (const void*)dst), SKY_ERR_INVALID_ARG,
+            "null argument");
+  const int li = layer_index(s, layer);
+  SKY_CHECK(li >= 0, SKY_ERR_INVALID_ARG, "layer %d outside [%d, %d)", layer,
+            s->cfg.layer_begin, s->cfg.layer_end);
+  if (s->last_stream) SKY_CUDA(cudaStreamSynchronize(s->last_stream));
+  SKY_CUDA(cudaDeviceSynchronize());
+  LayerBufs& Lb = s->layers[li];
+  for (int k = 0; k < SKY_NUM_PARAMS; ++k) {
+    const size_t bytes = param_elems(s, k) * (grads ? 4 : s->esz);
+    void* dev = grads ? (void*)Lb.g[k] : Lb.p[k];
+    if (to_slice) {
+      SKY_CHECK(src[k], SKY_ERR_INVALID_ARG, "tensor %d is null", k);
+      SKY_CUDA(cudaMemcpy(dev, src[k], bytes,
+                          on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice));
+    } else {
+      SKY_CHECK(dst[k], SKY_ERR_INVALID_ARG, "tensor %d is null", k);
+      SKY_CUDA(cudaMemcpy(dst[k], dev, bytes,
+                          on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost));
+    }
+  }
+  return SKY_OK;
+}
+
+sky_status sky_slice_set_params(sky_slice* s, int32_t layer, const void* const* tensors,
+                                int on_device) {
+  ABI_GUARD_BEGIN
+  return copy_tensors(s, layer, tensors, nullptr, on_device, true, false);
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_get_params(sky_slice* s, int32_t layer, void* const* tensors, int on_device) {
+  ABI_GUARD_BEGIN
+  return copy_tensors(s, layer, nullptr, tensors, on_device, false, false);
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_sync(sky_slice* s) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s, SKY_ERR_INVALID_ARG, "null handle");
+  if (s->last_stream) SKY_CUDA(cudaStreamSynchronize(s->last_stream));
+  SKY_CUDA(cudaDeviceSynchronize());
+  int32_t st = 0;
+  SKY_CUDA(cudaMemcpy(&st, s->d_status, 4, cudaMemcpyDeviceToHost));
+  SKY_CUDA(cudaMemset(s->d_status, 0, 4));
+  if (st & kStatusTimeout) {
+    set_error("a bounded device wait timed out");
+    return SKY_ERR_TIMEOUT;
+  }
+  if (st & kStatusBadLength) {
+    set_error("a sequence length was outside [1, S]");
+    return SKY_ERR_INVALID_ARG;
+  }
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_get_grads(sky_slice* s, int32_t layer, void* const* tensors, int on_device) {
+  ABI_GUARD_BEGIN
+  SKY_TRY(copy_tensors(s, layer, nullptr, tensors, on_device, false, true));
+  return sky_slice_sync(s);
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,
+                             int32_t S, void* y, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s && x && d_len && y, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(B >= 1 && S >= 1, SKY_ERR_INVALID_ARG, "B and S must be >= 1 (got %d, %d)", B, S);
+  SKY_CHECK(B <= s->cfg.max_batch && S <= s->cfg.max_seq, SKY_ERR_INVALID_ARG,
+            "B=%d S=%d exceed max_batch=%d max_seq=%d", B, S, s->cfg.max_batch, s->cfg.max_seq);
+  SKY_CHECK(x != y, SKY_ERR_INVALID_ARG, "x and y must not alias");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s->B = B; s->S = S; s->d_len = d_len; s->last_stream = st;
+  s->have_fwd = false;
+  SKY_TRY(forward_all(s, x, y, st, nullptr));
+  s->have_fwd = true;
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s && dy && dx, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(s->have_fwd, SKY_ERR_STATE, "backward needs a forward on this slice first");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s->last_stream = st;
+  return backward_all(s, dy, dx, st, nullptr);
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, int32_t iters,
+                                sky_layer_cost* out, int32_t n_out) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s && out, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(n_out == s->L, SKY_ERR_INVALID_ARG, "n_out must be %d", s->L);
+  SKY_CHECK(iters >= 1 && B >= 1 && S >= 1 && B <= s->cfg.max_batch && S <= s->cfg.max_seq,
+            SKY_ERR_INVALID_ARG, "bad B/S/iters");
+  const size_t xb = (size_t)B * S * s->H * s->esz;
+  void *x = nullptr, *y = nullptr, *dy = nullptr, *dx = nullptr;
+  int32_t* len = nullptr;
+  SKY_CUDA(cudaMalloc(&x, xb));
+  SKY_CUDA(cudaMalloc(&y, xb));
+  SKY_CUDA(cudaMalloc(&dy, xb));
+  SKY_CUDA(cudaMalloc(&dx, xb));
+  SKY_CUDA(cudaMalloc(&len, B * sizeof(int32_t)));
+  cudaStream_t st;
+  SKY_CUDA(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
+  const int64_t n = (int64_t)B * S * s->H;
+  const int bf = s->cfg.dtype == SKY_DTYPE_BF16;
+  fill_pattern<<<256, 256, 0, st>>>(x, n, bf, 1.0f, 1u);
+  fill_pattern<<<256, 256, 0, st>>>(dy, n, bf, 1e-3f, 2u);
+  fill_int<<<ceil_div(B, 256), 256, 0, st>>>(len, B, S);
+  count_launches(3);
+  std::vector<cudaEvent_t> fm(2 * s->L), bm(2 * s->L);
+  for (auto& e : fm) SKY_CUDA(cudaEventCreate(&e));
+  for (auto& e : bm) SKY_CUDA(cudaEventCreate(&e));
+  std::vector<std::vector<double>> ft(s->L), bt(s->L);
+  s->B = B; s->S = S; s->d_len = len; s->last_stream = st;
+  const bool prof = s->prof;
+  s->prof = false;
+  sky_status rc = SKY_OK;
+  const int warm = 2;
+  for (int it = 0; it < warm + iters && rc == SKY_OK; ++it) {
+    rc = forward_all(s, x, y, st, &fm);
+    if (rc == SKY_OK) rc = backward_all(s, dy, dx, st, &bm);
+    if (rc != SKY_OK) break;
+    if (cudaStreamSynchronize(st) != cudaSuccess) { rc = cuda_fail(cudaGetLastError(), "sync"); break; }
+    if (it < warm) continue;
+    for (int i = 0; i < s->L; ++i) {
+      float a = 0, b = 0;
+      cudaEventElapsedTime(&a, fm[2 * i], fm[2 * i + 1]);
+      cudaEventElapsedTime(&b, bm[2 * i], bm[2 * i + 1]);
+      ft[i].push_back(a);
+      bt[i].push_back(b);
+    }
+  }
+  s->prof = prof;
+  s->have_fwd = false;
+  s->last_stream = nullptr;  // the measuring stream is destroyed below
+  for (auto& e : fm) cudaEventDestroy(e);
+  for (auto& e : bm) cudaEventDestroy(e);
+  cudaStreamDestroy(st);
+  cudaFree(x); cudaFree(y); cudaFree(dy); cudaFree(dx); cudaFree(len);
+  if (rc != SKY_OK) return rc;
+  const double T = (double)B * S, H = s->H, F = s->F;
+  const double gemm_fwd = 2.0 * T * (4.0 * H * H + 2.0 * H * F);
+  const double attn_fwd = 4.0 * H * S * T;  // all query rows against all (valid) keys
+  size_t per_param = 0, per_grad = 0;
+  for (int k = 0; k < SKY_NUM_PARAMS; ++k) {
+    per_param += param_elems(s, k) * s->esz;
+    per_grad += param_elems(s, k) * 4;
+  }
+  for (int i = 0; i < s->L; ++i) {
+    auto med = [](std::vector<double>& v) {
+      std::sort(v.begin(), v.end());
+      return v.empty() ? 0.0 : v[v.size() / 2];
+    };
+    sky_layer_cost& o = out[i];
+    std::memset(&o, 0, sizeof(o));
+    o.layer = s->cfg.layer_begin + i;
+    o.fwd_ms = med(ft[i]);
+    o.bwd_ms = med(bt[i]);
+    o.fwd_flops = gemm_fwd + attn_fwd;
+    o.bwd_flops = 2.0 * (gemm_fwd + attn_fwd);
+    o.param_bytes = per_param;
+    o.grad_bytes = per_grad;
+    o.stash_bytes = s->stash_bytes / s->L;
+    o.workspace_bytes = s->ws_bytes_total / s->L;
+  }
+  return sky_slice_sync(s);
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_set_profiling(sky_slice* s, int enable) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s, SKY_ERR_INVALID_ARG, "null handle");
+  s->prof = enable != 0;
+  s->recs.clear();
+  s->event_next = 0;
+  for (int k = 0; k < P_NCAT; ++k) {
+    s->cat_ms[k] = s->cat_flops[k] = s->cat_bytes[k] = 0;
+    s->cat_n[k] = 0;
+  }
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_kernel_stats(sky_slice* s, sky_kernel_stat* out, int32_t n_out,
+                                  int32_t* n_written) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s && out && n_written, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CUDA(cudaDeviceSynchronize());
+  for (const auto& r : s->recs) {
+    float ms = 0;
+    SKY_CUDA(cudaEventElapsedTime(&ms, r.start, r.stop));
+    s->cat_ms[r.cat] += ms;
+    s->cat_flops[r.cat] += r.flops;
+    s->cat_bytes[r.cat] += r.bytes;
+    s->cat_n[r.cat] += 1;
+  }
+  s->recs.clear();
+  s->event_next = 0;
+  int w = 0;
+  for (int k = 0; k < P_NCAT && w < n_out; ++k) {
+    if (s->cat_n[k] == 0) continue;
+    sky_kernel_stat& o = out[w++];
+    std::memset(&o, 0, sizeof(o));
+    std::snprintf(o.name, sizeof(o.name), "%s", kCatNames[k]);
+    o.launches = s->cat_n[k];
+    o.total_ms = s->cat_ms[k];
+    o.flops = s->cat_flops[k];
+    o.bytes = s->cat_bytes[k];
+  }
+  *n_written = w;
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_memory(const sky_slice* s, uint64_t* param_bytes, uint64_t* grad_bytes,
+                            uint64_t* stash_bytes, uint64_t* workspace_bytes) {
+  SKY_CHECK(s, SKY_ERR_INVALID_ARG, "null handle");
+  if (param_bytes) *param_bytes = s->param_bytes;
+  if (grad_bytes) *grad_bytes = s->grad_bytes;
+  if (stash_bytes) *stash_bytes = s->stash_bytes;
+  if (workspace_bytes) *workspace_bytes = s->ws_bytes_total;
+  return SKY_OK;
+}
+
+// ------------------------------------------------------------- sky_ops.h ABI
+size_t sky_gemm_workspace_bytes(sky_gemm_form form, int32_t M, int32_t N, int32_t K,
+                                sky_dtype in_dtype, sky_dtype out_dtype) {
+  if (in_dtype != SKY_DTYPE_BF16 || out_dtype != SKY_DTYPE_FP32 || M <= 0 || N <= 0 || K <= 0)
+    return 0;
+  return gemm::workspace_bytes(form, M, N, K, true);
+}
+
+sky_status sky_gemm(sky_gemm_form form, int32_t M, int32_t N, int32_t K, sky_dtype in_dtype,
+                    const void* A, const void* B, void* C, sky_dtype out_dtype,
+                    sky_epilogue epilogue, const void* bias, const void* aux, void* aux_out,
+                    void* workspace, size_t workspace_bytes, int32_t* d_status, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(A && B && C, SKY_ERR_INVALID_ARG, "null operand");
+  SKY_CHECK(M > 0 && N > 0 && K > 0, SKY_ERR_INVALID_ARG, "sizes must be positive");
+  SKY_CHECK(form >= SKY_GEMM_XWT && form <= SKY_GEMM_XTW, SKY_ERR_INVALID_ARG, "bad form");
+  SKY_CHECK(epilogue >= SKY_EPI_STORE && epilogue <= SKY_EPI_RESIDUAL, SKY_ERR_INVALID_ARG,
+            "bad epilogue");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (in_dtype == SKY_DTYPE_BF16)
+    return gemm::launch_bf16(form, M, N, K, A, B, C, out_dtype == SKY_DTYPE_FP32, epilogue, bias,
+                             aux, aux_out, workspace, workspace_bytes, d_status, st);
+  SKY_CHECK(out_dtype == SKY_DTYPE_FP32, SKY_ERR_UNSUPPORTED, "fp32 input needs fp32 output");
+  return gemm::launch_f32(form, M, N, K, static_cast<const float*>(A),
+                          static_cast<const float*>(B), static_cast<float*>(C), epilogue,
+                          static_cast<const float*>(bias), static_cast<const float*>(aux),
+                          static_cast<float*>(aux_out), st);
+  ABI_GUARD_END
+}
+
+sky_status sky_attention_fwd(const void* qkv, const int32_t* d_len, int32_t B, int32_t S,
+                             int32_t H, int32_t A, sky_dtype dtype, void* ctx, float* lse,
+                             int32_t* d_status, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(qkv && d_len && ctx && lse, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(B > 0 && S > 0 && H > 0 && A > 0 && H % A == 0, SKY_ERR_INVALID_ARG, "bad sizes");
+  return attention_fwd(qkv, d_len, B, S, H, A, dtype, ctx, lse, d_status,
+                       static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+size_t sky_attention_bwd_workspace_bytes(int32_t B, int32_t S, int32_t H, int32_t A) {
+  (void)H;
+  return attention_bwd_ws(B, S, A);
+}
+
+sky_status sky_attention_bwd(const void* qkv, const void* ctx, const void* dctx,
+                             const float* lse, const int32_t* d_len, int32_t B, int32_t S,
+                             int32_t H, int32_t A, sky_dtype dtype, void* dqkv, void* workspace,
+                             size_t workspace_bytes, int32_t* d_status, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(qkv && ctx && dctx && lse && d_len && dqkv && workspace, SKY_ERR_INVALID_ARG,
+            "null argument");
+  SKY_CHECK(B > 0 && S > 0 && H > 0 && A > 0 && H % A == 0, SKY_ERR_INVALID_ARG, "bad sizes");
+  SKY_CHECK(workspace_bytes >= attention_bwd_ws(B, S, A), SKY_ERR_INVALID_ARG,
+            "workspace too small");
+  return attention_bwd(qkv, ctx, dctx, lse, d_len, B, S, H, A, dtype, dqkv,
+                       static_cast<float*>(workspace), d_status, static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+sky_status sky_layernorm_fwd(const float* u, const void* gamma, const void* beta, int32_t T,
+                             int32_t H, float eps, sky_dtype dtype, float* y32, void* y,
+                             float* mean, float* rstd, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(u && gamma && beta && (y32 || y) && mean && rstd, SKY_ERR_INVALID_ARG,
+            "null argument");
+  SKY_CHECK(T > 0 && H > 0, SKY_ERR_INVALID_ARG, "bad sizes");
+  return layernorm_fwd(u, gamma, beta, T, H, eps, dtype, y32, y, mean, rstd,
+                       static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+size_t sky_layernorm_bwd_workspace_bytes(int32_t T, int32_t H) {
+  if (T <= 0 || H <= 0) return 0;
+  return layernorm_bwd_ws(T, H);
+}
+
+sky_status sky_layernorm_bwd(const void* dy, sky_dtype dy_dtype, const float* u,
+                             const void* gamma, const float* mean, const float* rstd, int32_t T,
+                             int32_t H, sky_dtype dtype, float* du32, void* du, float* dgamma,
+                             float* dbeta, float* dbias, void* workspace, size_t workspace_bytes,
+                             void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(dy && u && gamma && mean && rstd && (du32 || du), SKY_ERR_INVALID_ARG,
+            "null argument");
+  SKY_CHECK(T > 0 && H > 0, SKY_ERR_INVALID_ARG, "bad sizes");
+  SKY_CHECK(dy_dtype == SKY_DTYPE_FP32 || dy_dtype == dtype, SKY_ERR_INVALID_ARG,
+            "dy must be fp32 or the slice dtype");
+  return layernorm_bwd(dy, dy_dtype, u, gamma, mean, rstd, T, H, dtype, du32, du, dgamma, dbeta,
+                       dbias, workspace, workspace_bytes, static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+sky_status sky_to_f32(const void* x, int64_t n, sky_dtype dtype, float* out, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(x && out && n >= 0, SKY_ERR_INVALID_ARG, "bad argument");
+  return to_f32(x, n, dtype, out, static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+sky_status sky_bias_gelu_fwd(const void* z, const void* bias, int32_t T, int32_t N,
+                             sky_dtype dtype, void* hpre, void* g, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(z && hpre && g, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(T > 0 && N > 0, SKY_ERR_INVALID_ARG, "bad sizes");
+  return bias_gelu_fwd(z, bias, T, N, dtype, hpre, g, static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+sky_status sky_gelu_bwd(const void* dg, const void* hpre, int32_t T, int32_t N, sky_dtype dtype,
+                        void* dh, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(dg && hpre && dh, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(T > 0 && N > 0, SKY_ERR_INVALID_ARG, "bad sizes");
+  return gelu_bwd(dg, hpre, T, N, dtype, dh, static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+size_t sky_column_sum_workspace_bytes(int32_t T, int32_t N) {
+  if (T <= 0 || N <= 0) return 0;
+  return column_sum_ws(T, N);
+}
+
+sky_status sky_column_sum(const void* x, int32_t T, int32_t N, sky_dtype dtype, float* out,
+                          void* workspace, size_t workspace_bytes, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(x && out, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(T > 0 && N > 0, SKY_ERR_INVALID_ARG, "bad sizes");
+  return column_sum(x, T, N, dtype, out, workspace, workspace_bytes,
+                    static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+}  // extern "C"

@@ -1,0 +1,140 @@
+"""Python view of one encoder slice: a handle on the C ABI of sky_slice.h.
+
+PyTorch supplies device memory and the CUDA stream; every computation runs in
+libsky_slice.so.  A slice owns the layers [layer_begin, layer_end) of a deep
+post-LN BERT encoder (the contiguous layer range a device is assigned,
+Sec. IV-D of the paper) and runs their forward and backward pass.
+"""
+from __future__ import annotations
+
+import ctypes as C
+
+import numpy as np
+
+from . import _lib as L
+from .synth import PARAM_NAMES, from_bf16_bits, to_bf16_bits
+
+
+def _stream_ptr(stream) -> int:
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _ptr(t) -> int:
+    return int(t.data_ptr())
+
+
+class EncoderSlice:
+    """Layers [layer_begin, layer_end) with hidden width H, A heads and FFN width F."""
+
+    def __init__(self, width: int, heads: int, ffn: int, layer_begin: int, layer_end: int,
+                 max_batch: int, max_seq: int, dtype: str = "bf16", ln_eps: float = 1e-12):
+        self.H, self.A, self.F = width, heads, ffn
+        self.layer_begin, self.layer_end = layer_begin, layer_end
+        self.dtype = dtype
+        cfg = L.SkySliceConfig(width, heads, ffn, layer_begin, layer_end, max_batch, max_seq,
+                               L.SKY_DTYPE_BF16 if dtype == "bf16" else L.SKY_DTYPE_FP32,
+                               ln_eps)
+        h = C.c_void_p()
+        L.call("sky_slice_create", C.byref(cfg), C.byref(h))
+        self.h = h
+        self._fwd_keep = None
+
+    # ----------------------------------------------------------- parameters
+    def shapes(self):
+        H, F = self.H, self.F
+        return {"Wqkv": (3 * H, H), "bqkv": (3 * H,), "Wo": (H, H), "bo": (H,),
+                "gamma1": (H,), "beta1": (H,), "W1": (F, H), "b1": (F,), "W2": (H, F),
+                "b2": (H,), "gamma2": (H,), "beta2": (H,)}
+
+    def set_params(self, layer: int, params: dict) -> None:
+        """params: name -> float32 array (bf16-exact values for bf16 slices)."""
+        bufs = []
+        for name in PARAM_NAMES:
+            a = np.ascontiguousarray(params[name], dtype=np.float32)
+            assert a.shape == self.shapes()[name], (name, a.shape)
+            bufs.append(to_bf16_bits(a) if self.dtype == "bf16" else a)
+        arr = (C.c_void_p * 12)(*[b.ctypes.data for b in bufs])
+        L.call("sky_slice_set_params", self.h, layer, arr, 0)
+
+    def _get(self, fn: str, layer: int, fp32: bool) -> dict:
+        out = {}
+        bufs = []
+        for name in PARAM_NAMES:
+            shp = self.shapes()[name]
+            b = np.empty(shp, dtype=np.float32 if fp32 or self.dtype == "fp32" else np.uint16)
+            bufs.append(b)
+        arr = (C.c_void_p * 12)(*[b.ctypes.data for b in bufs])
+        L.call(fn, self.h, layer, arr, 0)
+        for name, b in zip(PARAM_NAMES, bufs):
+            out[name] = from_bf16_bits(b) if b.dtype == np.uint16 else b
+        return out
+
+    def get_params(self, layer: int) -> dict:
+        return self._get("sky_slice_get_params", layer, False)
+
+    def get_grads(self, layer: int) -> dict:
+        """fp32 gradients of the 12 tensors of `layer` from the last backward."""
+        return self._get("sky_slice_get_grads", layer, True)
+
+    # -------------------------------------------------------------- compute
+    def forward(self, x, lens, y=None, stream=None):
+        """x: device [B, S, H] tensor (slice dtype); lens: device int32 [B]."""
+        import torch
+        B, S, H = x.shape
+        assert H == self.H and x.is_contiguous() and lens.dtype == torch.int32
+        if y is None:
+            y = torch.empty_like(x)
+        L.call("sky_slice_forward", self.h, _ptr(x), _ptr(lens), B, S, _ptr(y), _stream_ptr(stream))
+        self._fwd_keep = (x, lens)
+        return y
+
+    def backward(self, dy, dx=None, stream=None):
+        import torch
+        if dx is None:
+            dx = torch.empty_like(dy)
+        L.call("sky_slice_backward", self.h, _ptr(dy), _ptr(dx), _stream_ptr(stream))
+        return dx
+
+    def sync(self) -> None:
+        L.call("sky_slice_sync", self.h)
+
+    def layer_cost(self, B: int, S: int, iters: int = 5) -> list:
+        n = self.layer_end - self.layer_begin
+        out = (L.SkyLayerCost * n)()
+        L.call("sky_slice_layer_cost", self.h, B, S, iters, out, n)
+        return [{f: getattr(o, f) for f, _ in L.SkyLayerCost._fields_ if f != "_pad"} for o in out]
+
+    def set_profiling(self, on: bool) -> None:
+        L.call("sky_slice_set_profiling", self.h, 1 if on else 0)
+
+    def kernel_stats(self) -> dict:
+        out = (L.SkyKernelStat * 16)()
+        n = C.c_int32()
+        L.call("sky_slice_kernel_stats", self.h, out, 16, C.byref(n))
+        return {o.name.decode(): dict(launches=o.launches, total_ms=o.total_ms, flops=o.flops,
+                                      bytes=o.bytes) for o in out[: n.value]}
+
+    def memory(self) -> dict:
+        v = [C.c_uint64() for _ in range(4)]
+        L.call("sky_slice_memory", self.h, *[C.byref(x) for x in v])
+        return dict(zip(("param_bytes", "grad_bytes", "stash_bytes", "workspace_bytes"),
+                        [x.value for x in v]))
+
+    def close(self) -> None:
+        if getattr(self, "h", None):
+            L.lib().sky_slice_destroy(self.h)
+            self.h = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *a):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

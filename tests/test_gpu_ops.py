@@ -1,0 +1,272 @@
+"""Kernel-level parity through the C ABI of sky_ops.h (GPU).
+
+Each kernel runs on seeded inputs whose sizes span several tiles and end in a
+ragged tail; the reference is the plain definition in float64 (the oracle's
+own functions for attention, LayerNorm and GELU).
+"""
+import ctypes as C
+
+import numpy as np
+import pytest
+
+from oracle import encoder_f64 as ORC
+from paper_2202_11836_gb300 import _lib as L
+from paper_2202_11836_gb300.synth import round_bf16
+from parity_util import assert_close, l2rel, maxrel, to_device, to_host
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+def P(t):
+    return C.c_void_p(0 if t is None else int(t.data_ptr()))
+
+
+def stream():
+    return C.c_void_p(int(torch.cuda.current_stream().cuda_stream))
+
+
+def dt_code(dt):
+    return L.SKY_DTYPE_BF16 if dt == "bf16" else L.SKY_DTYPE_FP32
+
+
+def rnd(g, shape, std, dt):
+    a = g.normal(0, std, shape).astype(np.float32)
+    return round_bf16(a) if dt == "bf16" else a
+
+
+GEMM_SHAPES = [(128, 256, 64), (200, 264, 72), (384, 768, 1024), (1000, 520, 136), (8, 8, 8)]
+
+
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+@pytest.mark.parametrize("form", [L.SKY_GEMM_XWT, L.SKY_GEMM_XW, L.SKY_GEMM_XTW])
+@pytest.mark.parametrize("shape", GEMM_SHAPES, ids=lambda s: "x".join(map(str, s)))
+def test_gemm_store(dt, form, shape):
+    M, N, K = shape
+    g = np.random.default_rng(M * 7 + N * 3 + K + form)
+    if form == L.SKY_GEMM_XWT:
+        A, B = rnd(g, (M, K), 1.0, dt), rnd(g, (N, K), 0.05, dt)
+        ref = A.astype(np.float64) @ B.astype(np.float64).T
+    elif form == L.SKY_GEMM_XW:
+        A, B = rnd(g, (M, K), 1.0, dt), rnd(g, (K, N), 0.05, dt)
+        ref = A.astype(np.float64) @ B.astype(np.float64)
+    else:
+        A, B = rnd(g, (K, M), 1.0, dt), rnd(g, (K, N), 0.05, dt)
+        ref = A.astype(np.float64).T @ B.astype(np.float64)
+    for out_dt in (["bf16", "fp32"] if dt == "bf16" else ["fp32"]):
+        a, b = to_device(A, dt), to_device(B, dt)
+        c = torch.zeros((M, N), dtype=torch.bfloat16 if out_dt == "bf16" else torch.float32,
+                        device="cuda")
+        wsb = L.lib().sky_gemm_workspace_bytes(form, M, N, K, dt_code(dt), dt_code(out_dt))
+        ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device="cuda")
+        L.call("sky_gemm", form, M, N, K, dt_code(dt), P(a), P(b), P(c), dt_code(out_dt),
+               L.SKY_EPI_STORE, None, None, None, P(ws), wsb, None, stream())
+        torch.cuda.synchronize()
+        got = to_host(c)
+        if out_dt == "fp32":
+            tol = 1e-5 if dt == "bf16" else 1e-5
+            assert l2rel(got, ref) <= tol and maxrel(got, ref) <= 10 * tol, (out_dt, l2rel(got, ref))
+        else:
+            assert l2rel(got, ref) <= 4e-3 and maxrel(got, ref) <= 8e-3, (l2rel(got, ref), maxrel(got, ref))
+
+
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+@pytest.mark.parametrize("shape", [(256, 512, 128), (200, 264, 72)], ids=lambda s: "x".join(map(str, s)))
+def test_gemm_epilogues(dt, shape):
+    M, N, K = shape
+    g = np.random.default_rng(11)
+    A, W = rnd(g, (M, K), 1.0, dt), rnd(g, (N, K), 0.1, dt)
+    bias = rnd(g, (N,), 0.5, dt)
+    acc = A.astype(np.float64) @ W.astype(np.float64).T
+    a, w, b = to_device(A, dt), to_device(W, dt), to_device(bias, dt)
+    td = torch.bfloat16 if dt == "bf16" else torch.float32
+    tol_l2 = 4e-3 if dt == "bf16" else 1e-5
+    # bias + GELU: C = acc + b, aux_out = GELU(C)
+    c = torch.empty((M, N), dtype=td, device="cuda")
+    gout = torch.empty((M, N), dtype=td, device="cuda")
+    L.call("sky_gemm", L.SKY_GEMM_XWT, M, N, K, dt_code(dt), P(a), P(w), P(c), dt_code(dt),
+           L.SKY_EPI_BIAS_GELU, P(b), None, P(gout), None, 0, None, stream())
+    torch.cuda.synchronize()
+    pre = acc + bias
+    assert l2rel(to_host(c), pre) <= tol_l2
+    assert l2rel(to_host(gout), ORC.gelu(pre)) <= tol_l2
+    # GELU backward: C = acc * GELU'(aux)
+    hp = rnd(g, (M, N), 1.0, dt)
+    aux = to_device(hp, dt)
+    L.call("sky_gemm", L.SKY_GEMM_XWT, M, N, K, dt_code(dt), P(a), P(w), P(c), dt_code(dt),
+           L.SKY_EPI_GELU_BWD, None, P(aux), None, None, 0, None, stream())
+    torch.cuda.synchronize()
+    assert l2rel(to_host(c), acc * ORC.gelu_grad(hp.astype(np.float64))) <= tol_l2
+    # residual (fp32 stream) + bias, into the dtype and into fp32
+    res = g.normal(0, 1, (M, N)).astype(np.float32)
+    r32 = torch.from_numpy(res).cuda()
+    L.call("sky_gemm", L.SKY_GEMM_XWT, M, N, K, dt_code(dt), P(a), P(w), P(c), dt_code(dt),
+           L.SKY_EPI_RESIDUAL, P(b), P(r32), None, None, 0, None, stream())
+    c32 = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    L.call("sky_gemm", L.SKY_GEMM_XWT, M, N, K, dt_code(dt), P(a), P(w), P(c32), 1,
+           L.SKY_EPI_RESIDUAL, P(b), P(r32), None, None, 0, None, stream())
+    torch.cuda.synchronize()
+    assert l2rel(to_host(c), acc + bias + res) <= tol_l2
+    assert l2rel(to_host(c32), acc + bias + res) <= 1e-5
+
+
+def test_gemm_wgrad_split_deterministic():
+    """Split-K weight gradient over a long token dimension: bitwise repeatable."""
+    M, N, K = 768, 768, 8192
+    g = np.random.default_rng(5)
+    A, B = rnd(g, (K, M), 1.0, "bf16"), rnd(g, (K, N), 1e-3, "bf16")
+    a, b = to_device(A, "bf16"), to_device(B, "bf16")
+    wsb = L.lib().sky_gemm_workspace_bytes(L.SKY_GEMM_XTW, M, N, K, 0, 1)
+    assert wsb > 0  # this shape splits the token dimension
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    outs = []
+    for _ in range(2):
+        c = torch.empty((M, N), dtype=torch.float32, device="cuda")
+        L.call("sky_gemm", L.SKY_GEMM_XTW, M, N, K, 0, P(a), P(b), P(c), 1, 0, None, None, None,
+               P(ws), wsb, None, stream())
+        torch.cuda.synchronize()
+        outs.append(c.cpu().numpy())
+    assert np.array_equal(outs[0], outs[1])
+    ref = A.astype(np.float64).T @ B.astype(np.float64)
+    assert l2rel(outs[0], ref) <= 1e-5
+
+
+def attn_case(dt, B, S, A, lens, seed=3):
+    D = 64
+    H = A * D
+    g = np.random.default_rng(seed)
+    qkv = rnd(g, (B * S, 3 * H), 1.0, dt)
+    dctx = rnd(g, (B * S, H), 1.0, dt)
+    return H, qkv, dctx, np.array(lens, dtype=np.int32)
+
+
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+@pytest.mark.parametrize("case", [
+    (2, 100, 2, [100, 1]), (3, 130, 1, [64, 65, 129]), (1, 64, 2, [63]), (2, 256, 4, [256, 200]),
+    (4, 1, 1, [1, 1, 1, 1]),
+], ids=lambda c: f"B{c[0]}S{c[1]}A{c[2]}")
+def test_attention(dt, case):
+    B, S, A, lens = case
+    H, qkv, dctx, lens = attn_case(dt, B, S, A, lens)
+    D = 64
+    q = to_device(qkv, dt)
+    ln = torch.from_numpy(lens).cuda()
+    td = torch.bfloat16 if dt == "bf16" else torch.float32
+    ctx = torch.empty((B * S, H), dtype=td, device="cuda")
+    lse = torch.empty((B, A, S), dtype=torch.float32, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    L.call("sky_attention_fwd", P(q), P(ln), B, S, H, A, dt_code(dt), P(ctx), P(lse), P(st), stream())
+    do = to_device(dctx, dt)
+    dq = torch.empty((B * S, 3 * H), dtype=td, device="cuda")
+    wsb = L.lib().sky_attention_bwd_workspace_bytes(B, S, H, A)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    L.call("sky_attention_bwd", P(q), P(ctx), P(do), P(lse), P(ln), B, S, H, A, dt_code(dt),
+           P(dq), P(ws), wsb, P(st), stream())
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    Q = qkv[:, :H].reshape(B, S, A, D).astype(np.float64)
+    K = qkv[:, H:2 * H].reshape(B, S, A, D).astype(np.float64)
+    V = qkv[:, 2 * H:].reshape(B, S, A, D).astype(np.float64)
+    ctx_o, Pm = ORC.attention_forward(Q, K, V, lens)
+    assert_close("ctx", to_host(ctx), ctx_o.reshape(B * S, H), dt)
+    # the kernel's backward consumes its own (rounded) ctx, as the slice does
+    dQ, dK, dV = ORC.attention_backward(dctx.reshape(B, S, A, D).astype(np.float64), Q, K, V, Pm, lens)
+    got = to_host(dq)
+    assert_close("dQ", got[:, :H], dQ.reshape(B * S, H), dt)
+    assert_close("dK", got[:, H:2 * H], dK.reshape(B * S, H), dt)
+    assert_close("dV", got[:, 2 * H:], dV.reshape(B * S, H), dt)
+    # padded keys get exactly zero dK and dV
+    for b, n in enumerate(lens):
+        assert np.all(got[b * S + n:(b + 1) * S, H:] == 0.0)
+    # log-sum-exp of each row
+    for b, n in enumerate(lens):
+        for a in range(A):
+            s = Q[b, :, a] @ K[b, :n, a].T / 8.0
+            m = s.max(1)
+            ref = m + np.log(np.exp(s - m[:, None]).sum(1))
+            assert np.max(np.abs(lse.cpu().numpy()[b, a] - ref)) <= (2e-2 if dt == "bf16" else 1e-4)
+
+
+def test_attention_bad_length_sets_status():
+    B, S, A = 2, 64, 1
+    H, qkv, _, _ = attn_case("bf16", B, S, A, [1, 1])
+    q = to_device(qkv, "bf16")
+    ln = torch.tensor([0, 65], dtype=torch.int32, device="cuda")
+    ctx = torch.empty((B * S, H), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((B, A, S), dtype=torch.float32, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    L.call("sky_attention_fwd", P(q), P(ln), B, S, H, A, 0, P(ctx), P(lse), P(st), stream())
+    torch.cuda.synchronize()
+    assert int(st.item()) & 1
+    assert torch.isfinite(ctx.float()).all()
+
+
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+@pytest.mark.parametrize("TH", [(300, 768), (257, 1024), (64, 128), (33, 2048)],
+                         ids=lambda t: f"T{t[0]}H{t[1]}")
+def test_layernorm(dt, TH):
+    """LayerNorm of an fp32 residual sum; backward from a dtype or an fp32 dy."""
+    T, H = TH
+    if dt == "fp32" and H > 1024:
+        pytest.skip("fp32 LayerNorm supports H <= 1024")
+    g = np.random.default_rng(T + H)
+    u = g.normal(0.5, 2.0, (T, H)).astype(np.float32)
+    dy = rnd(g, (T, H), 1e-2, dt)
+    gam, bet = (1 + rnd(g, (H,), 0.1, dt)), rnd(g, (H,), 0.1, dt)
+    gam = round_bf16(gam) if dt == "bf16" else gam
+    td = torch.bfloat16 if dt == "bf16" else torch.float32
+    U = torch.from_numpy(u).cuda()
+    G_, B_, DY = (to_device(v, dt) for v in (gam, bet, dy))
+    y = torch.empty((T, H), dtype=td, device="cuda")
+    y32 = torch.empty((T, H), dtype=torch.float32, device="cuda")
+    mean = torch.empty(T, dtype=torch.float32, device="cuda")
+    rstd = torch.empty(T, dtype=torch.float32, device="cuda")
+    eps = 1e-5
+    L.call("sky_layernorm_fwd", P(U), P(G_), P(B_), T, H, C.c_float(eps), dt_code(dt),
+           P(y32), P(y), P(mean), P(rstd), stream())
+    Yo, xhat, rs = ORC.layer_norm(u.astype(np.float64), gam.astype(np.float64),
+                                  bet.astype(np.float64), eps)
+    dUo, dgo, dbo = ORC.layer_norm_backward(dy.astype(np.float64), xhat, rs, gam.astype(np.float64))
+    wsb = L.lib().sky_layernorm_bwd_workspace_bytes(T, H)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    for dy_dt in (dt, "fp32"):
+        dyt = DY if dy_dt == dt else DY.float()
+        du = torch.empty((T, H), dtype=td, device="cuda")
+        du32 = torch.empty((T, H), dtype=torch.float32, device="cuda")
+        dg, db, dbias = (torch.empty(H, dtype=torch.float32, device="cuda") for _ in range(3))
+        L.call("sky_layernorm_bwd", P(dyt), dt_code(dy_dt), P(U), P(G_), P(mean), P(rstd), T, H,
+               dt_code(dt), P(du32), P(du), P(dg), P(db), P(dbias), P(ws), wsb, stream())
+        torch.cuda.synchronize()
+        assert_close("y", to_host(y), Yo, dt)
+        assert l2rel(to_host(y32), Yo) <= 1e-5
+        assert_close("du", to_host(du), dUo, dt)
+        assert l2rel(to_host(du32), dUo) <= 1e-5
+        assert l2rel(dg.cpu().numpy(), dgo) <= 1e-5
+        assert l2rel(db.cpu().numpy(), dbo) <= 1e-5
+        assert l2rel(dbias.cpu().numpy(), dUo.sum(0)) <= 1e-4
+
+
+@pytest.mark.parametrize("dt", ["bf16", "fp32"])
+def test_gelu_and_column_sum(dt):
+    T, N = 333, 1000
+    g = np.random.default_rng(2)
+    z, bias, dgv = rnd(g, (T, N), 2.0, dt), rnd(g, (N,), 0.5, dt), rnd(g, (T, N), 1.0, dt)
+    td = torch.bfloat16 if dt == "bf16" else torch.float32
+    Z, Bv, DG = to_device(z, dt), to_device(bias, dt), to_device(dgv, dt)
+    hpre = torch.empty((T, N), dtype=td, device="cuda")
+    gg = torch.empty((T, N), dtype=td, device="cuda")
+    dh = torch.empty((T, N), dtype=td, device="cuda")
+    L.call("sky_bias_gelu_fwd", P(Z), P(Bv), T, N, dt_code(dt), P(hpre), P(gg), stream())
+    L.call("sky_gelu_bwd", P(DG), P(hpre), T, N, dt_code(dt), P(dh), stream())
+    out = torch.empty(N, dtype=torch.float32, device="cuda")
+    wsb = L.lib().sky_column_sum_workspace_bytes(T, N)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    L.call("sky_column_sum", P(DG), T, N, dt_code(dt), P(out), P(ws), wsb, stream())
+    torch.cuda.synchronize()
+    pre = z.astype(np.float64) + bias
+    assert_close("hpre", to_host(hpre), pre, dt)
+    assert_close("gelu", to_host(gg), ORC.gelu(pre), dt)
+    h_used = to_host(hpre)
+    assert_close("gelu_bwd", to_host(dh), dgv * ORC.gelu_grad(h_used), dt)
+    assert l2rel(out.cpu().numpy(), dgv.astype(np.float64).sum(0)) <= 1e-6

@@ -1,0 +1,168 @@
+"""Slice-level parity: the whole forward + backward of an encoder slice on the
+GPU (through sky_slice.h) against the float64 oracle on the same seeded
+inputs, every output tensor (Y, dX and the 12 gradients of every layer).
+
+Small cases run in full; the full-size workloads are checked on sampled
+sequences: each sequence's forward and input gradient depend on that sequence
+alone, and with the upstream gradient zero on every other sequence the weight
+gradients equal those of the sampled sequences alone, so the oracle runs on
+the sample while the GPU runs the whole batch in the benchmark's launch
+configuration.
+"""
+import numpy as np
+import pytest
+
+from paper_2202_11836_gb300 import synth
+from parity_util import compare_slice, oracle_slice, run_gpu_slice, to_device, to_host
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+
+
+def full_case(w, affine="random"):
+    params = synth.slice_params(w, affine=affine)
+    X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    Y, dX, grads = run_gpu_slice(w, X, lens, dY, params, None)
+    Yo, dXo, go = oracle_slice(w, X, lens, dY, params)
+    return compare_slice(w, Y, dX, grads, Yo, dXo, go)
+
+
+def test_tiny_fp32_slice():
+    """2-layer fp32 slice (H=128, A=2, F=512, S=32, B=4): maxrel <= 1e-4."""
+    full_case(synth.WORKLOADS["tiny-fp32"])
+    full_case(synth.WORKLOADS["tiny-fp32"], affine="bert")
+
+
+@pytest.mark.parametrize("w", [
+    synth.custom("bf16-ragged", layers=2, hidden=256, heads=4, ffn=1024, seq=96, batch=3,
+                 len_lo=1, len_hi=96, dy_std=1e-2),
+    synth.custom("bf16-odd-tail", layers=1, hidden=128, heads=2, ffn=520, seq=77, batch=5,
+                 len_lo=1, len_hi=77, dy_std=1e-2),
+    synth.custom("bf16-s1", layers=1, hidden=128, heads=2, ffn=256, seq=1, batch=8,
+                 len_lo=1, len_hi=1, dy_std=1e-2),
+], ids=lambda w: w.name)
+def test_bf16_small_slices(w):
+    full_case(w)
+
+
+def test_base_width_slice_full():
+    """BERT-base width, 4 layers, S=128, B=32: every sequence checked."""
+    full_case(synth.WORKLOADS["base-s128"], affine="bert")
+
+
+def sampled_case(w, sample):
+    """GPU on the whole batch, oracle on the sampled sequences."""
+    params = synth.slice_params(w, affine="bert")
+    X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    mask = np.zeros(w.batch, bool)
+    mask[list(sample)] = True
+    dY = dY * mask[:, None, None]
+    Y, dX, grads = run_gpu_slice(w, X, lens, dY, params, None)
+    idx = np.array(sample)
+    Yo, dXo, go = oracle_slice(w, X[idx], lens[idx], dY[idx], params)
+    rep = compare_slice(w, Y, dX, grads, Yo, dXo, go, rows=idx)
+    # rows outside the sample receive exactly zero input gradient
+    rest = np.where(~mask)[0]
+    assert np.all(dX[rest] == 0.0)
+    return rep
+
+
+def test_large_width_slice_sampled():
+    """BERT-large width, 8 layers, S=512, B=16 (full size), 2 sequences sampled."""
+    w = synth.WORKLOADS["large-s512"]
+    lens = synth.lengths(w)
+    sampled_case(w, (int(np.argmin(lens)), int(np.argmax(lens))))
+
+
+def test_long_sequence_slice_sampled():
+    """S=2048, B=4, 4 layers (full size): one full-length and one partial sequence."""
+    w = synth.WORKLOADS["large-s2048"]
+    sampled_case(w, (0, 3))
+
+
+def _slice_run(w, lb, le, X, lens, dY, params):
+    from paper_2202_11836_gb300.slice import EncoderSlice
+    with EncoderSlice(w.hidden, w.heads, w.ffn, lb, le, w.batch, w.seq, w.dtype) as s:
+        for l in range(lb, le):
+            s.set_params(l, params[l])
+        x = X if torch.is_tensor(X) else to_device(X, w.dtype)
+        ln = torch.from_numpy(lens).cuda()
+        y = s.forward(x, ln)
+        dx = s.backward(dY if torch.is_tensor(dY) else to_device(dY, w.dtype))
+        s.sync()
+        return y, dx, [s.get_grads(l) for l in range(lb, le)]
+
+
+def test_uneven_slices_compose_bitwise():
+    """Slices [0,1) then [1,4) of the 160-layer base model equal slice [0,4) bit for bit."""
+    w = synth.WORKLOADS["base-s128-b16"]
+    params = {l: synth.layer_params(l, w.hidden, w.ffn, "bf16", affine="random") for l in range(4)}
+    X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    y_full, dx_full, g_full = _slice_run(w, 0, 4, X, lens, dY, params)
+    y1, _, _ = _slice_run(w, 0, 1, X, lens, dY, params)
+    y2, dmid, g2 = _slice_run(w, 1, 4, y1, lens, dY, params)
+    _, dx1, g1 = _slice_run(w, 0, 1, X, lens, dmid, params)
+    assert torch.equal(y2, y_full)
+    assert torch.equal(dx1, dx_full)
+    for a, b in zip(g1 + g2, g_full):
+        for k in a:
+            assert np.array_equal(a[k], b[k]), k
+
+
+def test_uneven_slice_parity():
+    """The 7-layer slice [4, 11) of the 160-layer base-width model vs the oracle."""
+    w0 = synth.WORKLOADS["base-s128-b16"]
+    import dataclasses
+    w = dataclasses.replace(w0, layers=7, layer_begin=4)
+    full_case(w, affine="bert")
+
+
+def test_deterministic_and_status():
+    from paper_2202_11836_gb300 import _lib as L
+    from paper_2202_11836_gb300.slice import EncoderSlice
+    w = synth.custom("det", layers=2, hidden=256, heads=4, ffn=512, seq=64, batch=4, len_lo=1,
+                     len_hi=64)
+    params = synth.slice_params(w, affine="random")
+    X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    a = run_gpu_slice(w, X, lens, dY, params, None)
+    b = run_gpu_slice(w, X, lens, dY, params, None)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+    with EncoderSlice(256, 4, 512, 0, 2, 4, 64) as s:
+        x = to_device(X, "bf16")
+        dy = to_device(dY, "bf16")
+        with pytest.raises(L.SkyError) as e:
+            s.backward(dy)
+        assert e.value.status == L.SKY_ERR_STATE
+        bad = torch.tensor([0, 5, 64, 65], dtype=torch.int32, device="cuda")
+        s.forward(x, bad)
+        with pytest.raises(L.SkyError) as e:
+            s.sync()
+        assert e.value.status == L.SKY_ERR_INVALID_ARG
+        s.sync()  # status word was cleared
+        with pytest.raises(L.SkyError) as e:
+            s.forward(torch.zeros((5, 64, 256), dtype=torch.bfloat16, device="cuda"), bad)
+        assert e.value.status == L.SKY_ERR_INVALID_ARG
+
+
+def test_layer_cost_and_linearity():
+    """Per-layer cost records and slice time linear in the number of layers."""
+    import time
+    from paper_2202_11836_gb300.slice import EncoderSlice
+    w = synth.WORKLOADS["base-s128-b16"]
+    times = []
+    for (lb, le) in synth.UNEVEN_SLICES:
+        with EncoderSlice(w.hidden, w.heads, w.ffn, lb, le, w.batch, w.seq) as s:
+            for l in range(lb, le):
+                s.set_params(l, synth.layer_params(l, w.hidden, w.ffn, "bf16"))
+            rec = s.layer_cost(w.batch, w.seq, iters=3)
+            assert len(rec) == le - lb
+            for r in rec:
+                assert r["fwd_ms"] > 0 and r["bwd_ms"] > 0
+                assert r["param_bytes"] == 2 * (4 * 768 * 768 + 2 * 768 * 3072 + 9 * 768 + 3072)
+            times.append(sum(r["fwd_ms"] + r["bwd_ms"] for r in rec))
+    n = np.array([le - lb for lb, le in synth.UNEVEN_SLICES], float)
+    t = np.array(times)
+    beta, alpha = np.polyfit(n, t, 1)
+    pred = alpha + beta * n
+    r2 = 1 - ((t - pred) ** 2).sum() / ((t - t.mean()) ** 2).sum()
+    assert r2 >= 0.99, (times, r2)
