@@ -43,11 +43,14 @@ typedef enum { SKY_GEMM_XWT = 0, SKY_GEMM_XW = 1, SKY_GEMM_XTW = 2 } sky_gemm_fo
 
 /* Epilogues applied to the fp32 accumulator before the store.
  *   STORE     : C = acc (+ bias[n] if bias != NULL)
- *   BIAS_GELU : C = acc + bias[n] (the GELU input), aux_out = GELU(C)
- *   GELU_BWD  : C = acc * GELU'(aux[m,n])     (aux: the stored GELU input, in_dtype)
- *   RESIDUAL  : C = acc (+ bias[n]) + aux[m,n] (aux: fp32 residual stream)     */
-typedef enum { SKY_EPI_STORE = 0, SKY_EPI_BIAS_GELU = 1, SKY_EPI_GELU_BWD = 2,
-               SKY_EPI_RESIDUAL = 3 } sky_epilogue;
+ *   BIAS_GELU : z = acc + bias[n]; C = GELU(z), aux_out = GELU'(z) -- the
+ *               derivative the backward pass needs, stored as IEEE fp16 for
+ *               bf16 inputs (finer than bf16 on its range [-0.17, 1.13]) and
+ *               as fp32 for fp32 inputs
+ *   GELU_BWD  : C = acc * aux[m,n], aux = GELU'(z) as stored by BIAS_GELU
+ * Residual additions are not fused here: the LayerNorm kernels that follow
+ * every residual branch point read the fp32 residual themselves. */
+typedef enum { SKY_EPI_STORE = 0, SKY_EPI_BIAS_GELU = 1, SKY_EPI_GELU_BWD = 2 } sky_epilogue;
 
 /* Scratch bytes sky_gemm needs for (form, M, N, K) with an fp32 output
  * (deterministic split-K partials); 0 otherwise. */
@@ -58,10 +61,10 @@ size_t sky_gemm_workspace_bytes(sky_gemm_form form, int32_t M, int32_t N, int32_
  * layers).  in_dtype: BF16 runs the tcgen05/TMEM tensor-core kernel (the
  * contiguous dimensions -- K for XWT/XW, M for XTW, and N -- multiples of 8,
  * A, B, C 16-byte aligned, else UNSUPPORTED); FP32 runs the SIMT kernel.
- * out_dtype: the storage type of C (BF16 only with BF16 input).  bias uses
- * in_dtype.  BIAS_GELU and GELU_BWD need out_dtype == in_dtype.  An FP32
- * output with the plain STORE epilogue and no bias may split the K range over
- * CTAs; the partial sums go to `workspace` and are added in a fixed order
+ * out_dtype: the storage type of C (BF16 only with BF16 input); an FP32
+ * output takes the STORE epilogue (with or without bias).  bias uses
+ * in_dtype.  An FP32 output with no bias may split the K range over CTAs; the
+ * partial sums go to `workspace` and are added in a fixed order
  * (deterministic). */
 sky_status sky_gemm(sky_gemm_form form, int32_t M, int32_t N, int32_t K, sky_dtype in_dtype,
                     const void* A, const void* B, void* C, sky_dtype out_dtype,
@@ -88,29 +91,38 @@ sky_status sky_attention_bwd(const void* qkv, const void* ctx, const void* dctx,
                              void* workspace, size_t workspace_bytes, int32_t* d_status,
                              void* stream);
 
-/* LayerNorm forward of the fp32 residual sum u [T, H] (post-LN placement):
+/* Residual + LayerNorm forward (post-LN placement): u = a + r with a the
+ * linear layer's fp32 output and r the fp32 residual stream (r may be NULL);
  * y = gamma * (u - mean) * rstd + beta, rstd = 1/sqrt(var + eps), biased
- * variance.  Writes y32 (fp32) and/or y (dtype), either may be NULL but not
- * both; gamma, beta: [H] (dtype); mean, rstd: fp32 [T].  H % 8 == 0,
- * H <= 2048 (bf16) or 1024 (fp32). */
-sky_status sky_layernorm_fwd(const float* u, const void* gamma, const void* beta, int32_t T,
-                             int32_t H, float eps, sky_dtype dtype, float* y32, void* y,
-                             float* mean, float* rstd, void* stream);
+ * variance.  Writes u to u_out (may alias a, or NULL), y to y32 (fp32) and/or
+ * y (dtype) -- either may be NULL but not both; gamma, beta: [H] (dtype);
+ * mean, rstd: fp32 [T].  H % 8 == 0, H <= 2048 (bf16) or 1024 (fp32). */
+sky_status sky_layernorm_fwd(const float* a, const float* r, const void* gamma,
+                             const void* beta, int32_t T, int32_t H, float eps, sky_dtype dtype,
+                             float* u_out, float* y32, void* y, float* mean, float* rstd,
+                             void* stream);
 
 /* Scratch bytes of sky_layernorm_bwd (per-block column partial sums). */
 size_t sky_layernorm_bwd_workspace_bytes(int32_t T, int32_t H);
 
-/* LayerNorm backward.  dy: [T, H] in dy_dtype (FP32 or the slice dtype);
- * u, mean, rstd as saved by the forward.  With xhat = (u - mean) * rstd and
- * g = dy * gamma writes du = rstd * (g - mean(g) - xhat * mean(g * xhat))
- * to du32 (fp32) and/or du (dtype), and the fp32 column sums
- * dgamma = sum dy*xhat, dbeta = sum dy, dbias = sum du (each [H]; any may be
- * NULL).  The column sums are deterministic (fixed-order partials). */
-sky_status sky_layernorm_bwd(const void* dy, sky_dtype dy_dtype, const float* u,
-                             const void* gamma, const float* mean, const float* rstd, int32_t T,
-                             int32_t H, sky_dtype dtype, float* du32, void* du, float* dgamma,
-                             float* dbeta, float* dbias, void* workspace, size_t workspace_bytes,
-                             void* stream);
+/* LayerNorm backward.  The upstream gradient is dy + dy2 with dy: [T, H] in
+ * dy_dtype (FP32 or the slice dtype) and dy2: fp32 [T, H] or NULL (the two
+ * contributions meeting at a residual branch point); u, mean, rstd as saved
+ * by the forward.  With xhat = (u - mean) * rstd and g = (dy + dy2) * gamma
+ * writes du = rstd * (g - mean(g) - xhat * mean(g * xhat)) to du32 (fp32)
+ * and/or du (dtype), and the fp32 column sums dgamma = sum dy*xhat,
+ * dbeta = sum dy, dbias = sum du (each [H]; any may be NULL), which are
+ * deterministic (fixed-order partials in `workspace`). */
+sky_status sky_layernorm_bwd(const void* dy, sky_dtype dy_dtype, const float* dy2,
+                             const float* u, const void* gamma, const float* mean,
+                             const float* rstd, int32_t T, int32_t H, sky_dtype dtype,
+                             float* du32, void* du, float* dgamma, float* dbeta, float* dbias,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* out = a + b for fp32 a, b [n]; out in out_dtype (the slice's input
+ * gradient is the sum of its two branch terms). */
+sky_status sky_add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dtype, void* out,
+                       void* stream);
 
 /* Widens x [n] (dtype) to fp32: the slice's residual stream is fp32. */
 sky_status sky_to_f32(const void* x, int64_t n, sky_dtype dtype, float* out, void* stream);

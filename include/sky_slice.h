@@ -70,6 +70,11 @@ typedef struct {
   int32_t max_seq;      /* largest S a forward may use */
   sky_dtype dtype;      /* storage type of activations and parameters */
   float ln_eps;         /* LayerNorm epsilon (BERT uses 1e-12) */
+  int32_t io_fp32;      /* 1: x, y, dy, dx are fp32 even in a bf16 slice.  Inside a
+                           slice the residual and gradient streams are fp32, so with
+                           fp32 boundaries a chain of slices [a,b), [b,c) reproduces
+                           slice [a,c) bit for bit; with slice-dtype boundaries
+                           they agree up to one rounding of the boundary tensor. */
 } sky_slice_config;
 
 /* Per-layer cost record (Sec. IV-B: the model benchmark's per-layer FLOPs
@@ -125,7 +130,8 @@ sky_status sky_slice_get_params(sky_slice* s, int32_t layer, void* const* tensor
 sky_status sky_slice_get_grads(sky_slice* s, int32_t layer, void* const* tensors, int on_device);
 
 /* Forward pass of all layers of the slice: y = layer_{l1-1}(...layer_{l0}(x)).
- * x, y: device [B,S,H] in the slice dtype (may not alias); d_len: device
+ * x, y: device [B,S,H] in the boundary dtype (the slice dtype, or fp32 with
+ * io_fp32; may not alias); d_len: device
  * int32[B], each in [1,S] (checked on the device: a bad length is clamped,
  * and reported as INVALID_ARG by the next synchronising call).  x is copied
  * into the stash, so the caller may reuse it once the stream has passed it.
@@ -135,7 +141,7 @@ sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, 
                              int32_t S, void* y, void* stream);
 
 /* Backward pass of the slice for the most recent forward: given dy = dL/dy
- * (device [B,S,H], slice dtype) writes dx = dL/dx and overwrites the fp32
+ * (device [B,S,H], boundary dtype) writes dx = dL/dx and overwrites the fp32
  * gradients of every layer.  Must follow a forward on the same handle (the
  * forward's d_len must still be valid).  Enqueues on `stream`.
  * Errors: STATE (no forward since create), INVALID_ARG (null). */

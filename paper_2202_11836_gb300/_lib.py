@@ -17,7 +17,7 @@ SKY_OK, SKY_ERR_INVALID_ARG, SKY_ERR_OOM, SKY_ERR_CUDA, SKY_ERR_STATE, SKY_ERR_T
     SKY_ERR_UNSUPPORTED = range(7)
 SKY_DTYPE_BF16, SKY_DTYPE_FP32 = 0, 1
 SKY_GEMM_XWT, SKY_GEMM_XW, SKY_GEMM_XTW = 0, 1, 2
-SKY_EPI_STORE, SKY_EPI_BIAS_GELU, SKY_EPI_GELU_BWD, SKY_EPI_RESIDUAL = 0, 1, 2, 3
+SKY_EPI_STORE, SKY_EPI_BIAS_GELU, SKY_EPI_GELU_BWD = 0, 1, 2
 SKY_NUM_PARAMS = 12
 
 
@@ -25,7 +25,7 @@ class SkySliceConfig(C.Structure):
     _fields_ = [("width", C.c_int32), ("heads", C.c_int32), ("ffn", C.c_int32),
                 ("layer_begin", C.c_int32), ("layer_end", C.c_int32),
                 ("max_batch", C.c_int32), ("max_seq", C.c_int32),
-                ("dtype", C.c_int), ("ln_eps", C.c_float)]
+                ("dtype", C.c_int), ("ln_eps", C.c_float), ("io_fp32", C.c_int32)]
 
 
 class SkyLayerCost(C.Structure):
@@ -78,11 +78,12 @@ _SIGNATURES = {
     "sky_attention_bwd_workspace_bytes": (_SZ, [_I32, _I32, _I32, _I32]),
     "sky_attention_bwd": (C.c_int, [_VP, _VP, _VP, _VP, _VP, _I32, _I32, _I32, _I32, C.c_int,
                                     _VP, _VP, _SZ, _VP, _VP]),
-    "sky_layernorm_fwd": (C.c_int, [_VP, _VP, _VP, _I32, _I32, C.c_float, C.c_int, _VP, _VP,
-                                    _VP, _VP, _VP]),
+    "sky_layernorm_fwd": (C.c_int, [_VP, _VP, _VP, _VP, _I32, _I32, C.c_float, C.c_int, _VP,
+                                    _VP, _VP, _VP, _VP, _VP]),
     "sky_layernorm_bwd_workspace_bytes": (_SZ, [_I32, _I32]),
-    "sky_layernorm_bwd": (C.c_int, [_VP, C.c_int, _VP, _VP, _VP, _VP, _I32, _I32, C.c_int, _VP,
-                                    _VP, _VP, _VP, _VP, _VP, _SZ, _VP]),
+    "sky_layernorm_bwd": (C.c_int, [_VP, C.c_int, _VP, _VP, _VP, _VP, _VP, _I32, _I32, C.c_int,
+                                    _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]),
+    "sky_add_f32": (C.c_int, [_VP, _VP, C.c_int64, C.c_int, _VP, _VP]),
     "sky_to_f32": (C.c_int, [_VP, C.c_int64, C.c_int, _VP, _VP]),
     "sky_bias_gelu_fwd": (C.c_int, [_VP, _VP, _I32, _I32, C.c_int, _VP, _VP, _VP]),
     "sky_gelu_bwd": (C.c_int, [_VP, _VP, _I32, _I32, C.c_int, _VP, _VP]),

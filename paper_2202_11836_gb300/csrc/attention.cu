@@ -209,6 +209,37 @@ __global__ void __launch_bounds__(NTHR) attn_fwd_bf16(const bf16* __restrict__ q
 }
 
 // delta[b,a,s] = sum_d dctx[b,s,a,d] * ctx[b,s,a,d]  (equals sum_j P_sj dP_sj)
+// One warp per token row; each lane takes 8 consecutive elements (16 bytes
+// of bf16) per step, and the 8 lanes covering one 64-wide head reduce with
+// shuffles.  Requires D == 64.
+__global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __restrict__ dctx, int S,
+                                int H, int A, int64_t rows, float* __restrict__ delta) {
+  const int64_t row = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  const int l = threadIdx.x & 31;
+  if (row >= rows) return;
+  const int64_t b = row / S, s = row % S;
+  for (int c0 = 0; c0 < H; c0 += 256) {
+    const int col = c0 + l * 8;
+    float acc = 0.f;
+    if (col < H) {
+      const uint4 x = *reinterpret_cast<const uint4*>(ctx + row * H + col);
+      const uint4 y = *reinterpret_cast<const uint4*>(dctx + row * H + col);
+      const __nv_bfloat162* xs = reinterpret_cast<const __nv_bfloat162*>(&x);
+      const __nv_bfloat162* ys = reinterpret_cast<const __nv_bfloat162*>(&y);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 p = __bfloat1622float2(xs[i]), q = __bfloat1622float2(ys[i]);
+        acc += p.x * q.x + p.y * q.y;
+      }
+    }
+    acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+    acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+    acc += __shfl_xor_sync(0xffffffffu, acc, 4);
+    if ((l & 7) == 0 && col < H) delta[(b * A + col / HD) * S + s] = acc;
+  }
+}
+
+// Generic form (fp32 path): one warp per (row, head).
 template <typename T>
 __global__ void attn_delta(const T* __restrict__ ctx, const T* __restrict__ dctx, int S, int H,
                            int A, int D, int64_t rows, float* __restrict__ delta) {
@@ -658,9 +689,9 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
   const int dblocks = ceil_div(rows * A * 32, 256);
   if (dt == SKY_DTYPE_BF16) {
     SKY_CHECK(D == attn::HD, SKY_ERR_UNSUPPORTED, "bf16 attention needs head dim 64 (got %d)", D);
-    attn::attn_delta<__nv_bfloat16><<<dblocks, 256, 0, stream>>>(
+    attn::attn_delta_bf16<<<ceil_div(rows * 32, 256), 256, 0, stream>>>(
         static_cast<const __nv_bfloat16*>(ctx), static_cast<const __nv_bfloat16*>(dctx), S, H, A,
-        D, rows, delta);
+        rows, delta);
     dim3 grid(ceil_div(S, attn::TQ), A, B);
     const auto* q = static_cast<const __nv_bfloat16*>(qkv);
     const auto* o = static_cast<const __nv_bfloat16*>(dctx);

@@ -47,12 +47,33 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
   return __float2bfloat16_rn(v);
 }
 
-// GELU(h) = h * Phi(h) and its derivative Phi(h) + h * phi(h), via CUDA's
-// normcdff / expf (exact-erf form, no tanh approximation).
-__device__ __forceinline__ float gelu_f(float h) { return h * normcdff(h); }
+// GELU(h) = h * Phi(h) and its derivative Phi(h) + h * phi(h), with
+// Phi(h) = (1 + erf(h / sqrt 2)) / 2 from CUDA's erff and phi from expf
+// (exact-erf form, no tanh approximation).
+__device__ __forceinline__ float std_normal_cdf(float h) {
+  return 0.5f * (1.f + erff(h * 0.70710678118654752f));
+}
+__device__ __forceinline__ float gelu_f(float h) { return h * std_normal_cdf(h); }
 __device__ __forceinline__ float gelu_grad_f(float h) {
   const float inv_sqrt_2pi = 0.3989422804014327f;
-  return normcdff(h) + h * inv_sqrt_2pi * expf(-0.5f * h * h);
+  return std_normal_cdf(h) + h * inv_sqrt_2pi * expf(-0.5f * h * h);
+}
+
+// GELU(h) and GELU'(h) together, for the tensor-core epilogues: Phi from the
+// erf approximation of Abramowitz & Stegun, Handbook of Mathematical
+// Functions, formula 7.1.26 (|erf error| <= 1.5e-7 for all x), written for
+// x = |h| / sqrt 2 so that Phi and phi share one exponential exp(-h^2 / 2).
+__device__ __forceinline__ void gelu_and_grad_as(float h, float& g, float& gp) {
+  const float a = fabsf(h) * 0.70710678118654752f;
+  const float t = __fdividef(1.f, 1.f + 0.3275911f * a);
+  const float poly =
+      t * (0.254829592f +
+           t * (-0.284496736f + t * (1.421413741f + t * (-1.453152027f + t * 1.061405429f))));
+  const float E = exp2f(-0.72134752044448170f * h * h);  // exp(-h^2 / 2)
+  const float q = 0.5f * poly * E;                        // = Phi(-|h|)
+  const float Phi = h >= 0.f ? 1.f - q : q;
+  g = h * Phi;
+  gp = Phi + h * 0.3989422804014327f * E;
 }
 
 __device__ __forceinline__ float warp_sum(float v) {

@@ -58,10 +58,12 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(int M, int N, int K, cons
       const int64_t off = static_cast<int64_t>(m) * N + n;
       float v = acc[i][j];
       if (bias) v += bias[n];
-      if (epi == SKY_EPI_GELU_BWD) v *= gelu_grad_f(aux[off]);
-      if (epi == SKY_EPI_RESIDUAL) v += aux[off];
+      if (epi == SKY_EPI_GELU_BWD) v *= aux[off];
+      if (epi == SKY_EPI_BIAS_GELU) {
+        aux_out[off] = gelu_grad_f(v);
+        v = gelu_f(v);
+      }
       C[off] = v;
-      if (epi == SKY_EPI_BIAS_GELU) aux_out[off] = gelu_f(v);
     }
   }
 }
@@ -72,8 +74,9 @@ sky_status launch_f32(sky_gemm_form form, int M, int N, int K, const float* A, c
                       cudaStream_t stream) {
   SKY_CHECK(epi != SKY_EPI_BIAS_GELU || (bias && aux_out), SKY_ERR_INVALID_ARG,
             "BIAS_GELU epilogue needs bias and aux_out");
-  SKY_CHECK((epi != SKY_EPI_GELU_BWD && epi != SKY_EPI_RESIDUAL) || aux, SKY_ERR_INVALID_ARG,
-            "epilogue needs aux");
+  SKY_CHECK(epi == SKY_EPI_STORE || epi == SKY_EPI_BIAS_GELU || epi == SKY_EPI_GELU_BWD,
+            SKY_ERR_INVALID_ARG, "unknown epilogue %d", epi);
+  SKY_CHECK(epi != SKY_EPI_GELU_BWD || aux, SKY_ERR_INVALID_ARG, "GELU' epilogue needs aux");
   int64_t am, ak, bk, bn;
   switch (form) {
     case SKY_GEMM_XWT: am = K; ak = 1; bk = 1; bn = K; break;   // A[M,K], B[N,K]

@@ -9,8 +9,14 @@
 //   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=256,
 //               K=16) into a TMEM accumulator; two accumulators (512 TMEM
 //               columns) let the epilogue of one tile overlap the next,
-//   warps 2..5  epilogue: tcgen05.ld of the accumulator, fused bias / GELU /
-//               GELU' / residual, store to global memory.
+//   warps 2..9  epilogue (two warps per TMEM lane quarter, one per half of
+//               the tile's columns): tcgen05.ld of the accumulator, a
+//               transpose through shared memory so stores coalesce, fused
+//               bias / GELU, store to global memory.  The forward GELU
+//               epilogue also stores GELU'(z) (fp16); the backward epilogue
+//               multiplies by it, loading it for the whole tile before the
+//               accumulator is waited on so its latency hides under the
+//               tile's main loop.
 // K-major operands (x and W in y = x W^T) and MN-major operands (W in
 // dy W, and both operands of dy^T x) are read directly through the
 // descriptors' major-ness bit, so no transpose pass exists.  Weight gradients
@@ -20,6 +26,8 @@
 #include <cudaTypedefs.h>
 
 #include <mutex>
+
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 #include "gemm.h"
@@ -33,33 +41,44 @@ constexpr int A_BYTES = BM * BK * 2;        // 16 KiB
 constexpr int B_BYTES = BN * BK * 2;        // 32 KiB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;           // two fp32 accumulators of 128 x 256
-constexpr int NUM_THREADS = 192;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int NUM_EPI_WARPS = 8;            // two per TMEM lane quarter
+constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
+constexpr int EPI_OFF = STAGES * STAGE_BYTES;           // per epilogue warp: 32 x 32 fp32 staging
+constexpr int EPI_BYTES = NUM_EPI_WARPS * 32 * 32 * 4;
+constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
+constexpr int SMEM_BYTES = BAR_OFF + 256 /*barriers*/ + 1024 /*alignment slack*/;
 constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
+constexpr uint32_t kSleepNs = 20000;         // suspend hint of the epilogue's accumulator wait
 
 struct Params {
   int M, N, K;
   int m_tiles, n_tiles, splits, kb_per_split, k_blocks;
-  int epi;
-  int out_f32;
   void* C;                        // bf16 [M,N], fp32 [M,N], or fp32 [splits][M][N]
   const __nv_bfloat16* bias;      // [N] or null
-  const __nv_bfloat16* aux;       // [M,N] GELU input (GELU_BWD) or null
-  const float* aux32;             // [M,N] fp32 residual (RESIDUAL) or null
-  __nv_bfloat16* aux_out;         // [M,N] or null
+  const __half* aux;              // [M,N] GELU'(z) (GELU_BWD) or null
+  __half* aux_out;                // [M,N] GELU'(z) (BIAS_GELU) or null
   int32_t* status;
   uint64_t timeout_ns;
   int skip_loads;                 // fault injection: producer never issues TMA
 };
 
-template <bool A_MN, bool B_MN>
+// 8-byte read-only load that does not allocate in L1 (streamed once).
+__device__ __forceinline__ uint2 ld_nc_u2(const void* p) {
+  uint2 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0, %1}, [%2];"
+               : "=r"(v.x), "=r"(v.y)
+               : "l"(p));
+  return v;
+}
+
+template <bool A_MN, bool B_MN, int EPI, bool OUT_F32>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA,
                    const __grid_constant__ CUtensorMap tmB, const Params p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + BAR_OFF);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
@@ -74,7 +93,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(&tfull[a], 1);
-      ptx::mbar_init(&tempty[a], 128);
+      ptx::mbar_init(&tempty[a], 32 * NUM_EPI_WARPS);
     }
     ptx::mbar_init(done, 1);
     ptx::fence_mbar_init();
@@ -181,97 +200,108 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // -------------------------------------------------------------- epilogue
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    // Warp w owns TMEM lanes [32q, 32q+32) (q = w % 4: rows m0+32q..) and the
+    // column half hf of the tile.  Per 32-column chunk: tcgen05.ld (thread =
+    // row) -> XOR-swizzled smem tile -> read back so that 8 lanes cover one
+    // row's 32 columns, then the fused epilogue and coalesced stores.
+    constexpr int HALF = BN / 2, CHUNKS = HALF / 32;
+    const int q = warp & 3, hf = (warp - 2) >> 2;
+    float* stage = reinterpret_cast<float*>(smem + EPI_OFF) + (warp - 2) * 32 * 32;
+    const int c4 = lane & 7;          // this lane's 4-column group in a chunk
+    const int rsub = lane >> 3;       // row within each group of 4 rows
     int acc = 0;
     uint32_t aphase = 0;
     for (int u = blockIdx.x; u < units; u += gridDim.x) {
       const int split = u / tiles, rem = u % tiles;
-      const int m0 = (rem / p.n_tiles) * BM, n0 = (rem % p.n_tiles) * BN;
-      if (!ptx::mbar_wait(&tfull[acc], aphase, lim, p.status)) break;
+      const int m0 = (rem / p.n_tiles) * BM, n0 = (rem % p.n_tiles) * BN + hf * HALF;
+      // GELU' input of this warp's whole sub-tile, fetched before the wait
+      uint2 pre[EPI == SKY_EPI_GELU_BWD ? CHUNKS : 1][8];
+      if constexpr (EPI == SKY_EPI_GELU_BWD) {
+#pragma unroll
+        for (int cc = 0; cc < CHUNKS; ++cc) {
+          const int col = n0 + cc * 32 + 4 * c4;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int row = m0 + q * 32 + 4 * i + rsub;
+            pre[cc][i] = (col < p.N && row < p.M)
+                                            ? ld_nc_u2(p.aux + static_cast<int64_t>(row) * p.N + col)
+                             : make_uint2(0u, 0u);
+          }
+        }
+      }
+      if (!ptx::mbar_wait(&tfull[acc], aphase, lim, p.status, kSleepNs)) break;
       ptx::tc_fence_after();
-      const int row = m0 + q * 32 + lane;
-      const bool row_ok = row < p.M;
-      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
-#pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN + hf * HALF;
+      float* outf = OUT_F32 ? static_cast<float*>(p.C) +
+                                  static_cast<int64_t>(split) * p.M * static_cast<int64_t>(p.N)
+                            : nullptr;
+#pragma unroll
+      for (int cc = 0; cc < CHUNKS; ++cc) {
+        const int c = cc * 32;
         uint32_t r[32];
         __syncwarp();
         ptx::tmem_ld_32x32b_x32(taddr + c, r);
         ptx::tmem_ld_wait();
-        const int n = n0 + c;
-        if (!row_ok || n >= p.N) continue;
-        const bool full_chunk = n + 32 <= p.N;
-        float v[32];
+        if (n0 + c >= p.N) continue;  // warp-uniform
+        // stage: row `lane`, 16-byte chunk j at position j ^ (lane & 7)
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-        const int64_t off = static_cast<int64_t>(row) * p.N + n;
-        const int nv = full_chunk ? 32 : p.N - n;
-        if (p.bias) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (j < nv) v[j] += __bfloat162float(p.bias[n + j]);
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<float4*>(stage + lane * 32 + ((j ^ (lane & 7)) << 2)) =
+              make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                          __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+        __syncwarp();
+        const int col = n0 + c + 4 * c4;
+        const bool col_ok = col < p.N;
+        float b4[4] = {0.f, 0.f, 0.f, 0.f};
+        if (p.bias && col_ok) {
+          const uint2 raw = *reinterpret_cast<const uint2*>(p.bias + col);
+          const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&raw);
+          const float2 f0 = __bfloat1622float2(h[0]), f1 = __bfloat1622float2(h[1]);
+          b4[0] = f0.x; b4[1] = f0.y; b4[2] = f1.x; b4[3] = f1.y;
         }
-        if (p.epi == SKY_EPI_GELU_BWD) {
-          __nv_bfloat16 a[32];
-          if (full_chunk) {
+        // all 8 rows x 4 columns first (independent, branch-free), then the
+        // bounds-checked stores
+        float v[8][4];
 #pragma unroll
-            for (int j = 0; j < 32; j += 8)
-              *reinterpret_cast<uint4*>(&a[j]) = *reinterpret_cast<const uint4*>(p.aux + off + j);
-          } else {
+        for (int i = 0; i < 8; ++i) {
+          const int rl = 4 * i + rsub;
+          const float4 t4 = *reinterpret_cast<const float4*>(stage + rl * 32 + ((c4 ^ (rl & 7)) << 2));
+          v[i][0] = t4.x + b4[0]; v[i][1] = t4.y + b4[1]; v[i][2] = t4.z + b4[2]; v[i][3] = t4.w + b4[3];
+        }
+        if constexpr (EPI == SKY_EPI_GELU_BWD) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) a[j] = j < nv ? p.aux[off + j] : __float2bfloat16(0.f);
+          for (int i = 0; i < 8; ++i) {
+            const __half2* h = reinterpret_cast<const __half2*>(&pre[cc][i]);
+            const float2 f0 = __half22float2(h[0]), f1 = __half22float2(h[1]);
+            v[i][0] *= f0.x; v[i][1] *= f0.y; v[i][2] *= f1.x; v[i][3] *= f1.y;
           }
+        }
+        uint2 gq[EPI == SKY_EPI_BIAS_GELU ? 8 : 1];
+        if constexpr (EPI == SKY_EPI_BIAS_GELU) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] *= gelu_grad_f(__bfloat162float(a[j]));
-        } else if (p.epi == SKY_EPI_RESIDUAL) {
-          if (full_chunk) {
+          for (int i = 0; i < 8; ++i) {
+            float gp[4];
 #pragma unroll
-            for (int j = 0; j < 32; j += 4) {
-              const float4 q = *reinterpret_cast<const float4*>(p.aux32 + off + j);
-              v[j] += q.x; v[j + 1] += q.y; v[j + 2] += q.z; v[j + 3] += q.w;
+            for (int j = 0; j < 4; ++j) gelu_and_grad_as(v[i][j], v[i][j], gp[j]);
+            const __half2 h0 = __floats2half2_rn(gp[0], gp[1]), h1 = __floats2half2_rn(gp[2], gp[3]);
+            gq[i] = make_uint2(*reinterpret_cast<const uint32_t*>(&h0),
+                               *reinterpret_cast<const uint32_t*>(&h1));
+          }
+        }
+        if (col_ok) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int row = m0 + q * 32 + 4 * i + rsub;
+            if (row >= p.M) continue;
+            const int64_t off = static_cast<int64_t>(row) * p.N + col;
+            if constexpr (OUT_F32) {
+              *reinterpret_cast<float4*>(outf + off) = make_float4(v[i][0], v[i][1], v[i][2], v[i][3]);
+            } else {
+              *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.C) + off) =
+                  make_uint2(ptx::pack_bf16(v[i][0], v[i][1]), ptx::pack_bf16(v[i][2], v[i][3]));
+              if constexpr (EPI == SKY_EPI_BIAS_GELU)
+                *reinterpret_cast<uint2*>(p.aux_out + off) = gq[i];
             }
-          } else {
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-              if (j < nv) v[j] += p.aux32[off + j];
-          }
-        }
-        if (p.out_f32) {
-          float* out = static_cast<float*>(p.C) +
-                       static_cast<int64_t>(split) * p.M * static_cast<int64_t>(p.N) + off;
-          if (full_chunk) {
-#pragma unroll
-            for (int j = 0; j < 32; j += 4)
-              *reinterpret_cast<float4*>(out + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-          } else {
-            for (int j = 0; j < nv; ++j) out[j] = v[j];
-          }
-          continue;
-        }
-        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.C) + off;
-        uint32_t packed[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) packed[j] = ptx::pack_bf16(v[2 * j], v[2 * j + 1]);
-        if (full_chunk) {
-#pragma unroll
-          for (int j = 0; j < 16; j += 4)
-            *reinterpret_cast<uint4*>(out + 2 * j) =
-                make_uint4(packed[j], packed[j + 1], packed[j + 2], packed[j + 3]);
-        } else {
-          for (int j = 0; j < nv; ++j) out[j] = __float2bfloat16_rn(v[j]);
-        }
-        if (p.epi == SKY_EPI_BIAS_GELU) {
-          __nv_bfloat16* g = p.aux_out + off;
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            packed[j] = ptx::pack_bf16(gelu_f(v[2 * j]), gelu_f(v[2 * j + 1]));
-          if (full_chunk) {
-#pragma unroll
-            for (int j = 0; j < 16; j += 4)
-              *reinterpret_cast<uint4*>(g + 2 * j) =
-                  make_uint4(packed[j], packed[j + 1], packed[j + 2], packed[j + 3]);
-          } else {
-            for (int j = 0; j < nv; ++j) g[j] = __float2bfloat16_rn(gelu_f(v[j]));
           }
         }
       }
@@ -340,12 +370,31 @@ bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, in
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+template <bool A_MN, bool B_MN, int EPI, bool OUT_F32>
+cudaError_t launch_variant(dim3 grid, const CUtensorMap& ta, const CUtensorMap& tb,
+                           const Params& p, cudaStream_t stream) {
+  static cudaError_t attr = cudaFuncSetAttribute(gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 SMEM_BYTES);
+  if (attr != cudaSuccess) return attr;
+  gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
+  return cudaGetLastError();
+}
+
+// One instantiation per (operand majorness, epilogue, output type) keeps
+// every kernel's code to the epilogue it runs.
 template <bool A_MN, bool B_MN>
-cudaError_t set_smem_attr() {
-  static cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<A_MN, B_MN>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              SMEM_BYTES);
-  return e;
+cudaError_t launch_form(dim3 grid, const CUtensorMap& ta, const CUtensorMap& tb, const Params& p,
+                        int epi, bool out_f32, cudaStream_t stream) {
+  if (out_f32) return launch_variant<A_MN, B_MN, SKY_EPI_STORE, true>(grid, ta, tb, p, stream);
+  switch (epi) {
+    case SKY_EPI_BIAS_GELU:
+      return launch_variant<A_MN, B_MN, SKY_EPI_BIAS_GELU, false>(grid, ta, tb, p, stream);
+    case SKY_EPI_GELU_BWD:
+      return launch_variant<A_MN, B_MN, SKY_EPI_GELU_BWD, false>(grid, ta, tb, p, stream);
+    default:
+      return launch_variant<A_MN, B_MN, SKY_EPI_STORE, false>(grid, ta, tb, p, stream);
+  }
 }
 
 uint64_t g_timeout_ns = 2000000000ull;  // 2 s per wait
@@ -396,12 +445,13 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
             SKY_ERR_UNSUPPORTED, "bf16 GEMM operands must be 16-byte aligned");
   SKY_CHECK(reinterpret_cast<uintptr_t>(C) % 16 == 0, SKY_ERR_UNSUPPORTED,
             "GEMM output must be 16-byte aligned");
-  SKY_CHECK(!out_f32 || epi == SKY_EPI_STORE || epi == SKY_EPI_RESIDUAL, SKY_ERR_UNSUPPORTED,
-            "fp32-output GEMM supports the STORE and RESIDUAL epilogues");
+  SKY_CHECK(epi == SKY_EPI_STORE || epi == SKY_EPI_BIAS_GELU || epi == SKY_EPI_GELU_BWD,
+            SKY_ERR_INVALID_ARG, "unknown epilogue %d", epi);
+  SKY_CHECK(!out_f32 || epi == SKY_EPI_STORE, SKY_ERR_UNSUPPORTED,
+            "fp32-output GEMM supports the STORE epilogue");
   SKY_CHECK(epi != SKY_EPI_BIAS_GELU || (bias && aux_out), SKY_ERR_INVALID_ARG,
             "BIAS_GELU epilogue needs bias and aux_out");
-  SKY_CHECK(epi != SKY_EPI_GELU_BWD && epi != SKY_EPI_RESIDUAL || aux, SKY_ERR_INVALID_ARG,
-            "epilogue needs aux");
+  SKY_CHECK(epi != SKY_EPI_GELU_BWD || aux, SKY_ERR_INVALID_ARG, "GELU' epilogue needs aux");
   const int sms = sm_count();
   SKY_CHECK(sms > 0, SKY_ERR_CUDA, "no CUDA device");
 
@@ -425,16 +475,13 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   }
   p.kb_per_split = ceil_div(p.k_blocks, p.splits);
   p.splits = ceil_div(p.k_blocks, p.kb_per_split);
-  p.epi = epi;
-  p.out_f32 = out_f32 ? 1 : 0;
   const size_t need = p.splits > 1 ? static_cast<size_t>(p.splits) * M * N * sizeof(float) : 0;
   SKY_CHECK(ws_bytes >= need && (need == 0 || ws), SKY_ERR_INVALID_ARG,
             "GEMM workspace too small (%zu < %zu)", ws_bytes, need);
   p.C = p.splits > 1 ? ws : C;
   p.bias = static_cast<const __nv_bfloat16*>(bias);
-  p.aux = epi == SKY_EPI_GELU_BWD ? static_cast<const __nv_bfloat16*>(aux) : nullptr;
-  p.aux32 = epi == SKY_EPI_RESIDUAL ? static_cast<const float*>(aux) : nullptr;
-  p.aux_out = static_cast<__nv_bfloat16*>(aux_out);
+  p.aux = epi == SKY_EPI_GELU_BWD ? static_cast<const __half*>(aux) : nullptr;
+  p.aux_out = static_cast<__half*>(aux_out);
   p.status = status;
   p.timeout_ns = g_timeout_ns;
   p.skip_loads = g_skip_loads;
@@ -442,18 +489,13 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   const int units = p.m_tiles * p.n_tiles * p.splits;
   const int grid = units < sms ? units : sms;
   cudaError_t e;
-  if (form == SKY_GEMM_XWT) {
-    SKY_CUDA((set_smem_attr<false, false>()));
-    gemm_tc_kernel<false, false><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
-  } else if (form == SKY_GEMM_XW) {
-    SKY_CUDA((set_smem_attr<false, true>()));
-    gemm_tc_kernel<false, true><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
-  } else {
-    SKY_CUDA((set_smem_attr<true, true>()));
-    gemm_tc_kernel<true, true><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
-  }
+  if (form == SKY_GEMM_XWT)
+    e = launch_form<false, false>(grid, ta, tb, p, epi, out_f32, stream);
+  else if (form == SKY_GEMM_XW)
+    e = launch_form<false, true>(grid, ta, tb, p, epi, out_f32, stream);
+  else
+    e = launch_form<true, true>(grid, ta, tb, p, epi, out_f32, stream);
   count_launches(1);
-  e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "gemm_tc_kernel launch");
   if (p.splits > 1) {
     const int64_t n = static_cast<int64_t>(M) * N;

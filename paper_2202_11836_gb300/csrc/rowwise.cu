@@ -41,24 +41,18 @@ __device__ __forceinline__ void store8(__nv_bfloat16* p, const float (&v)[8]) {
 constexpr int LN_WARPS = 8;
 constexpr int V = 8;  // elements per lane per chunk; chunk c of a lane starts at (c*32+lane)*8
 
-// y = gamma * (u - mean) * rstd + beta on the fp32 residual sum u.
+// u = a + r (the linear layer's output plus the fp32 residual stream), then
+// y = gamma * (u - mean) * rstd + beta.  u is written back (u_out may alias a)
+// for the backward pass; y goes to y32 (fp32) and/or yT (slice dtype).
 template <typename T, int NV>
 __global__ void __launch_bounds__(LN_WARPS * 32) ln_fwd_kernel(
-    const float* __restrict__ u, const T* __restrict__ gamma, const T* __restrict__ beta,
-    int rows, int H, float eps, float* __restrict__ y32, T* __restrict__ yT,
-    float* __restrict__ mean_out, float* __restrict__ rstd_out) {
+    const float* a, const float* __restrict__ r, const T* __restrict__ gamma,
+    const T* __restrict__ beta, int rows, int H, float eps, float* u_out,
+    float* __restrict__ y32, T* __restrict__ yT, float* __restrict__ mean_out,
+    float* __restrict__ rstd_out) {
   const int lane = threadIdx.x & 31;
   const int warp = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
   const int nwarps = gridDim.x * LN_WARPS;
-  float gm[NV][V], bt[NV][V];
-#pragma unroll
-  for (int c = 0; c < NV; ++c) {
-    const int col = (c * 32 + lane) * V;
-    if (col < H) {
-      load8(gamma + col, gm[c]);
-      load8(beta + col, bt[c]);
-    }
-  }
   const float invH = 1.f / H;
   for (int row = warp; row < rows; row += nwarps) {
     float x[NV][V];
@@ -67,7 +61,14 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_fwd_kernel(
     for (int c = 0; c < NV; ++c) {
       const int col = (c * 32 + lane) * V;
       if (col < H) {
-        load8(u + (int64_t)row * H + col, x[c]);
+        const int64_t off = (int64_t)row * H + col;
+        load8(a + off, x[c]);
+        if (r) {
+          float rv[V];
+          load8(r + off, rv);
+#pragma unroll
+          for (int i = 0; i < V; ++i) x[c][i] += rv[i];
+        }
 #pragma unroll
         for (int i = 0; i < V; ++i) s += x[c][i];
       }
@@ -90,11 +91,15 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_fwd_kernel(
     for (int c = 0; c < NV; ++c) {
       const int col = (c * 32 + lane) * V;
       if (col < H) {
-        float o[V];
+        const int64_t off = (int64_t)row * H + col;
+        float gm[V], bt[V], o[V];
+        load8(gamma + col, gm);
+        load8(beta + col, bt);
 #pragma unroll
-        for (int i = 0; i < V; ++i) o[i] = gm[c][i] * ((x[c][i] - mu) * rs) + bt[c][i];
-        if (y32) store8(y32 + (int64_t)row * H + col, o);
-        if (yT) store8(yT + (int64_t)row * H + col, o);
+        for (int i = 0; i < V; ++i) o[i] = gm[i] * ((x[c][i] - mu) * rs) + bt[i];
+        if (u_out) store8(u_out + off, x[c]);
+        if (y32) store8(y32 + off, o);
+        if (yT) store8(yT + off, o);
       }
     }
     if (lane == 0) {
@@ -104,47 +109,26 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_fwd_kernel(
   }
 }
 
-// Writes this CTA's column sums of `acc` (one per warp, added in warp order)
-// to part[k][blockIdx.x][:].
-template <int NV>
-__device__ __forceinline__ void ln_flush_partial(const float (&acc)[NV][V], int k, float* red,
-                                                 float* __restrict__ part, int H) {
-  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-#pragma unroll
-  for (int c = 0; c < NV; ++c) {
-    const int col = (c * 32 + lane) * V;
-    if (col < H) {
-#pragma unroll
-      for (int i = 0; i < V; ++i) red[wib * H + col + i] = acc[c][i];
-    }
-  }
-  __syncthreads();
-  for (int col = threadIdx.x; col < H; col += blockDim.x) {
-    float s = 0.f;
-    for (int w = 0; w < LN_WARPS; ++w) s += red[w * H + col];
-    part[((int64_t)k * gridDim.x + blockIdx.x) * H + col] = s;
-  }
-  __syncthreads();
-}
-
-// du = rstd * (g - mean(g) - xhat * mean(g * xhat)), g = dy * gamma, and the
-// per-CTA column partials of dy * xhat, dy and du.
+// du = rstd * (g - mean(g) - xhat * mean(g * xhat)), g = dy * gamma with
+// dy = dy + dy2 (the two gradient contributions of a residual branch point,
+// dy2 optional), and the per-CTA column partials of dy * xhat, dy and du.
+// Each warp keeps its running
+// column sums in its own shared-memory rows (red[w][k][:]), which keeps the
+// register count low enough for two or more CTAs per SM; at the end the CTA's
+// warps are added in order into part[k][blockIdx.x][:].
 template <typename TDY, typename T, int NV>
 __global__ void __launch_bounds__(LN_WARPS * 32) ln_bwd_kernel(
-    const TDY* __restrict__ dy, const float* __restrict__ u, const T* __restrict__ gamma,
+    const TDY* __restrict__ dy, const float* __restrict__ dy2, const float* __restrict__ u,
+    const T* __restrict__ gamma,
     const float* __restrict__ mean, const float* __restrict__ rstd, int rows, int H,
     float* __restrict__ du32, T* __restrict__ duT, float* __restrict__ part) {
-  extern __shared__ float red[];  // [LN_WARPS][H]
+  extern __shared__ float red[];  // [LN_WARPS][3][H]
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const int warp = blockIdx.x * LN_WARPS + wib;
   const int nwarps = gridDim.x * LN_WARPS;
-  float gm[NV][V];
-  float pg[NV][V] = {}, pb[NV][V] = {}, pu[NV][V] = {};
-#pragma unroll
-  for (int c = 0; c < NV; ++c) {
-    const int col = (c * 32 + lane) * V;
-    if (col < H) load8(gamma + col, gm[c]);
-  }
+  float* mine = red + (size_t)wib * 3 * H;
+  for (int i = lane * 4; i < 3 * H; i += 128) *reinterpret_cast<float4*>(mine + i) = make_float4(0.f, 0.f, 0.f, 0.f);
+  __syncwarp();
   const float invH = 1.f / H;
   for (int row = warp; row < rows; row += nwarps) {
     const float mu = mean[row], rs = rstd[row];
@@ -157,10 +141,24 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_bwd_kernel(
         const int64_t off = (int64_t)row * H + col;
         load8(u + off, xh[c]);
         load8(dy + off, dyv[c]);
+        if (dy2) {
+          float d2[V];
+          load8(dy2 + off, d2);
+#pragma unroll
+          for (int i = 0; i < V; ++i) dyv[c][i] += d2[i];
+        }
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < NV; ++c) {
+      const int col = (c * 32 + lane) * V;
+      if (col < H) {
+        float gm[V];
+        load8(gamma + col, gm);
 #pragma unroll
         for (int i = 0; i < V; ++i) {
           xh[c][i] = (xh[c][i] - mu) * rs;
-          const float g = dyv[c][i] * gm[c][i];
+          const float g = dyv[c][i] * gm[i];
           s1 += g;
           s2 += g * xh[c][i];
         }
@@ -171,23 +169,50 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_bwd_kernel(
     for (int c = 0; c < NV; ++c) {
       const int col = (c * 32 + lane) * V;
       if (col < H) {
-        float o[V];
+        float gm[V], o[V], pg[V], pb[V], pu[V];
+        load8(gamma + col, gm);
+        load8(mine + col, pg);
+        load8(mine + H + col, pb);
+        load8(mine + 2 * H + col, pu);
 #pragma unroll
         for (int i = 0; i < V; ++i) {
-          o[i] = rs * (dyv[c][i] * gm[c][i] - mg - xh[c][i] * mgx);
-          pg[c][i] += dyv[c][i] * xh[c][i];
-          pb[c][i] += dyv[c][i];
-          pu[c][i] += o[i];
+          o[i] = rs * (dyv[c][i] * gm[i] - mg - xh[c][i] * mgx);
+          pg[i] += dyv[c][i] * xh[c][i];
+          pb[i] += dyv[c][i];
+          pu[i] += o[i];
         }
+        store8(mine + col, pg);
+        store8(mine + H + col, pb);
+        store8(mine + 2 * H + col, pu);
         if (du32) store8(du32 + (int64_t)row * H + col, o);
         if (duT) store8(duT + (int64_t)row * H + col, o);
       }
     }
   }
-  // CTA column partials: [3][gridDim.x][H], summed over the CTA's warps in order
-  ln_flush_partial<NV>(pg, 0, red, part, H);
-  ln_flush_partial<NV>(pb, 1, red, part, H);
-  ln_flush_partial<NV>(pu, 2, red, part, H);
+  __syncthreads();
+  for (int k = 0; k < 3; ++k) {
+    for (int col = threadIdx.x; col < H; col += blockDim.x) {
+      float s = 0.f;
+      for (int w = 0; w < LN_WARPS; ++w) s += red[((size_t)w * 3 + k) * H + col];
+      part[((int64_t)k * gridDim.x + blockIdx.x) * H + col] = s;
+    }
+  }
+}
+
+// out = a + b (fp32 inputs) in fp32 or bf16.
+template <typename T>
+__global__ void add_kernel(const float* __restrict__ a, const float* __restrict__ b, int64_t n,
+                           T* __restrict__ out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = from_f32<T>(a[i] + b[i]);
+}
+
+__global__ void to_bf16_kernel(const float* __restrict__ x, int64_t n,
+                               __nv_bfloat16* __restrict__ out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = __float2bfloat16_rn(x[i]);
 }
 
 template <typename T>
@@ -197,27 +222,73 @@ __global__ void to_f32_kernel(const T* __restrict__ x, int64_t n, float* __restr
     out[i] = to_f32(x[i]);
 }
 
-// out_k[n] = sum_b part[k][b][n] for the non-null outputs (fixed order).
-__global__ void reduce_partials(const float* __restrict__ part, int nblk, int N, float* out0,
-                                float* out1, float* out2) {
-  const int n = blockIdx.x * blockDim.x + threadIdx.x;
+// out_k[n] = sum_b part[k][b][n] for the non-null outputs, in a fixed order:
+// CTA (cx, k) owns 32 columns; its 8 warps each add every 8th partial row
+// (coalesced 128-byte reads), then the 8 warp sums are added in order.
+__global__ void __launch_bounds__(256) reduce_partials(const float* __restrict__ part, int nblk,
+                                                       int N, float* out0, float* out1,
+                                                       float* out2) {
+  __shared__ float red[8][33];
   const int k = blockIdx.y;
   float* out = k == 0 ? out0 : (k == 1 ? out1 : out2);
-  if (n >= N || out == nullptr) return;
-  const float* p = part + (int64_t)k * nblk * N + n;
+  if (out == nullptr) return;  // uniform over the CTA
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int n = blockIdx.x * 32 + lane;
   float s = 0.f;
-  for (int b = 0; b < nblk; ++b) s += p[(int64_t)b * N];
-  out[n] = s;
+  if (n < N) {
+    const float* p = part + (int64_t)k * nblk * N + n;
+    for (int b = w; b < nblk; b += 8) s += p[(int64_t)b * N];
+  }
+  red[w][lane] = s;
+  __syncthreads();
+  if (w == 0 && n < N) {
+    float t = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) t += red[j][lane];
+    out[n] = t;
+  }
 }
 
-// Column partial sums of x[T, N]: part[y][n] over rows y, y + gridDim.y, ...
+// Column partial sums of x[T, N] (N % 8 == 0): CTA (cx, g) owns columns
+// [256 cx, 256 cx + 256); warp w of the CTA adds rows 8 g + w, + 8 G, ...
+// with 16-byte loads (a warp reads 512 contiguous bytes of bf16 per row), the
+// CTA's 8 warps are added in order and part[g][n] is written.
 template <typename T>
-__global__ void colsum_partial(const T* __restrict__ x, int rows, int N, float* __restrict__ part) {
-  const int n = blockIdx.x * blockDim.x + threadIdx.x;
-  if (n >= N) return;
-  float s = 0.f;
-  for (int r = blockIdx.y; r < rows; r += gridDim.y) s += to_f32(x[(int64_t)r * N + n]);
-  part[(int64_t)blockIdx.y * N + n] = s;
+__global__ void __launch_bounds__(256) colsum_partial(const T* __restrict__ x, int rows, int N,
+                                                      float* __restrict__ part) {
+  __shared__ float red[8][256];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int col = blockIdx.x * 256 + lane * 8;
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (col < N) {
+    const int step = gridDim.y * 8;
+    int r = blockIdx.y * 8 + w;
+    for (; r + 3 * step < rows; r += 4 * step) {
+      float v[4][8];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) load8(x + (int64_t)(r + k * step) * N + col, v[k]);
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] += v[k][i];
+    }
+    for (; r < rows; r += step) {
+      float v[8];
+      load8(x + (int64_t)r * N + col, v);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] += v[i];
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) red[w][lane * 8 + i] = acc[i];
+  __syncthreads();
+  const int c = blockIdx.x * 256 + threadIdx.x;
+  if (c < N) {
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) s += red[k][threadIdx.x];
+    part[(int64_t)blockIdx.y * N + c] = s;
+  }
 }
 
 template <typename T>
@@ -244,24 +315,31 @@ int ln_blocks(int rows) {
   const int cap = 4 * (sm_count() > 0 ? sm_count() : 148);
   return want < cap ? want : cap;
 }
+// Backward CTAs also write column partials, so fewer, longer-lived CTAs.
+int ln_bwd_blocks(int rows) {
+  const int want = ceil_div(rows, LN_WARPS);
+  const int cap = 2 * (sm_count() > 0 ? sm_count() : 148);
+  return want < cap ? want : cap;
+}
 
 template <typename T, int NV>
-void ln_fwd_launch(const float* u, const void* gm, const void* bt, int rows, int H, float eps,
-                   float* y32, void* y, float* mean, float* rstd, cudaStream_t st) {
+void ln_fwd_launch(const float* a, const float* r, const void* gm, const void* bt, int rows, int H,
+                   float eps, float* u_out, float* y32, void* y, float* mean, float* rstd,
+                   cudaStream_t st) {
   ln_fwd_kernel<T, NV><<<ln_blocks(rows), LN_WARPS * 32, 0, st>>>(
-      u, static_cast<const T*>(gm), static_cast<const T*>(bt), rows, H, eps, y32,
+      a, r, static_cast<const T*>(gm), static_cast<const T*>(bt), rows, H, eps, u_out, y32,
       static_cast<T*>(y), mean, rstd);
 }
 template <typename TDY, typename T, int NV>
-void ln_bwd_launch(const void* dy, const float* u, const void* gm, const float* mean,
-                   const float* rstd, int rows, int H, float* du32, void* du, float* part,
-                   int nblk, cudaStream_t st) {
-  const size_t smem = (size_t)LN_WARPS * H * sizeof(float);
+void ln_bwd_launch(const void* dy, const float* dy2, const float* u, const void* gm,
+                   const float* mean, const float* rstd, int rows, int H, float* du32, void* du,
+                   float* part, int nblk, cudaStream_t st) {
+  const size_t smem = (size_t)LN_WARPS * 3 * H * sizeof(float);
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(ln_bwd_kernel<TDY, T, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
   ln_bwd_kernel<TDY, T, NV><<<nblk, LN_WARPS * 32, smem, st>>>(
-      static_cast<const TDY*>(dy), u, static_cast<const T*>(gm), mean, rstd, rows, H, du32,
+      static_cast<const TDY*>(dy), dy2, u, static_cast<const T*>(gm), mean, rstd, rows, H, du32,
       static_cast<T*>(du), part);
 }
 
@@ -285,21 +363,21 @@ int lane_vectors(int H) { return ceil_div(H, 32 * rw::V); }
     default: CALL(8); break;       \
   }
 
-sky_status layernorm_fwd(const float* u, const void* gamma, const void* beta, int rows, int H,
-                         float eps, sky_dtype dt, float* y32, void* y, float* mean, float* rstd,
-                         cudaStream_t st) {
+sky_status layernorm_fwd(const float* a, const float* r, const void* gamma, const void* beta,
+                         int rows, int H, float eps, sky_dtype dt, float* u_out, float* y32,
+                         void* y, float* mean, float* rstd, cudaStream_t st) {
   SKY_CHECK(H % rw::V == 0 && lane_vectors(H) <= kMaxNV && (dt == SKY_DTYPE_BF16 || H <= 1024),
             SKY_ERR_UNSUPPORTED, "LayerNorm width %d unsupported", H);
   SKY_CHECK(y32 || y, SKY_ERR_INVALID_ARG, "LayerNorm forward needs an output");
   const int nv = lane_vectors(H);
   if (dt == SKY_DTYPE_BF16) {
-#define LNF(NV) rw::ln_fwd_launch<__nv_bfloat16, NV>(u, gamma, beta, rows, H, eps, y32, y, mean, rstd, st)
+#define LNF(NV) rw::ln_fwd_launch<__nv_bfloat16, NV>(a, r, gamma, beta, rows, H, eps, u_out, y32, y, mean, rstd, st)
     SKY_NV_DISPATCH(nv, LNF)
 #undef LNF
   } else {
     // fp32 slices: the dtype output is itself fp32, so one store suffices
     float* only = y32 ? y32 : static_cast<float*>(y);
-#define LNF(NV) rw::ln_fwd_launch<float, NV>(u, gamma, beta, rows, H, eps, only, nullptr, mean, rstd, st)
+#define LNF(NV) rw::ln_fwd_launch<float, NV>(a, r, gamma, beta, rows, H, eps, u_out, only, nullptr, mean, rstd, st)
     SKY_NV_DISPATCH(nv, LNF)
 #undef LNF
     if (y32 && y && y != y32)
@@ -311,44 +389,66 @@ sky_status layernorm_fwd(const float* u, const void* gamma, const void* beta, in
 }
 
 size_t layernorm_bwd_ws(int rows, int H) {
-  return (size_t)3 * rw::ln_blocks(rows) * H * sizeof(float);
+  return (size_t)3 * rw::ln_bwd_blocks(rows) * H * sizeof(float);
 }
 
-sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* u, const void* gamma,
-                         const float* mean, const float* rstd, int rows, int H, sky_dtype dt,
-                         float* du32, void* du, float* dgamma, float* dbeta, float* dbias,
-                         void* ws, size_t ws_bytes, cudaStream_t st) {
+sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, const float* u,
+                         const void* gamma, const float* mean, const float* rstd, int rows, int H,
+                         sky_dtype dt, float* du32, void* du, float* dgamma, float* dbeta,
+                         float* dbias, void* ws, size_t ws_bytes, cudaStream_t st) {
   SKY_CHECK(H % rw::V == 0 && lane_vectors(H) <= kMaxNV && (dt == SKY_DTYPE_BF16 || H <= 1024),
             SKY_ERR_UNSUPPORTED, "LayerNorm width %d unsupported", H);
   SKY_CHECK(du32 || du, SKY_ERR_INVALID_ARG, "LayerNorm backward needs an output");
-  const int nblk = rw::ln_blocks(rows);
+  const int nblk = rw::ln_bwd_blocks(rows);
   SKY_CHECK(ws && ws_bytes >= (size_t)3 * nblk * H * sizeof(float), SKY_ERR_INVALID_ARG,
             "LayerNorm backward workspace too small");
   float* part = static_cast<float*>(ws);
   const int nv = lane_vectors(H);
   if (dt == SKY_DTYPE_BF16) {
     if (dy_dt == SKY_DTYPE_BF16) {
-#define LNB(NV) rw::ln_bwd_launch<__nv_bfloat16, __nv_bfloat16, NV>(dy, u, gamma, mean, rstd, rows, H, du32, du, part, nblk, st)
+#define LNB(NV) rw::ln_bwd_launch<__nv_bfloat16, __nv_bfloat16, NV>(dy, dy2, u, gamma, mean, rstd, rows, H, du32, du, part, nblk, st)
       SKY_NV_DISPATCH(nv, LNB)
 #undef LNB
     } else {
-#define LNB(NV) rw::ln_bwd_launch<float, __nv_bfloat16, NV>(dy, u, gamma, mean, rstd, rows, H, du32, du, part, nblk, st)
+#define LNB(NV) rw::ln_bwd_launch<float, __nv_bfloat16, NV>(dy, dy2, u, gamma, mean, rstd, rows, H, du32, du, part, nblk, st)
       SKY_NV_DISPATCH(nv, LNB)
 #undef LNB
     }
   } else {
     float* only = du32 ? du32 : static_cast<float*>(du);
-#define LNB(NV) rw::ln_bwd_launch<float, float, NV>(dy, u, gamma, mean, rstd, rows, H, only, nullptr, part, nblk, st)
+#define LNB(NV) rw::ln_bwd_launch<float, float, NV>(dy, dy2, u, gamma, mean, rstd, rows, H, only, nullptr, part, nblk, st)
     SKY_NV_DISPATCH(nv, LNB)
 #undef LNB
     if (du32 && du && du != du32)
       SKY_CUDA(cudaMemcpyAsync(du, du32, (size_t)rows * H * 4, cudaMemcpyDeviceToDevice, st));
   }
-  dim3 grid(ceil_div(H, 256), 3);
+  dim3 grid(ceil_div(H, 32), 3);
   rw::reduce_partials<<<grid, 256, 0, st>>>(part, nblk, H, dgamma, dbeta, dbias);
   count_launches(2);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward launch");
+}
+
+sky_status add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dt, void* out,
+                   cudaStream_t st) {
+  if (n <= 0) return SKY_OK;
+  const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
+  if (out_dt == SKY_DTYPE_BF16)
+    rw::add_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(a, b, n, static_cast<__nv_bfloat16*>(out));
+  else
+    rw::add_kernel<float><<<blocks, 256, 0, st>>>(a, b, n, static_cast<float*>(out));
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "add launch");
+}
+
+sky_status f32_to_bf16(const float* x, int64_t n, void* out, cudaStream_t st) {
+  if (n <= 0) return SKY_OK;
+  const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
+  rw::to_bf16_kernel<<<blocks, 256, 0, st>>>(x, n, static_cast<__nv_bfloat16*>(out));
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "narrow launch");
 }
 
 sky_status to_f32(const void* x, int64_t n, sky_dtype dt, float* out, cudaStream_t st) {
@@ -367,10 +467,11 @@ sky_status to_f32(const void* x, int64_t n, sky_dtype dt, float* out, cudaStream
 namespace {
 int colsum_row_groups(int rows, int N) {
   const int cb = ceil_div(N, 256);
-  int g = 4 * (sm_count() > 0 ? sm_count() : 148) / cb;
-  if (g < 1) g = 1;
-  if (g > rows) g = rows;
-  return g;
+  int g = 2 * (sm_count() > 0 ? sm_count() : 148) / cb;
+  const int max_g = ceil_div(rows, 8);
+  if (g > max_g) g = max_g;
+  if (g > 65535) g = 65535;
+  return g < 1 ? 1 : g;
 }
 }  // namespace
 
@@ -380,6 +481,7 @@ size_t column_sum_ws(int rows, int N) {
 
 sky_status column_sum(const void* x, int rows, int N, sky_dtype dt, float* out, void* ws,
                       size_t ws_bytes, cudaStream_t st) {
+  SKY_CHECK(N % 8 == 0, SKY_ERR_UNSUPPORTED, "column sum needs N %% 8 == 0 (got %d)", N);
   const int groups = colsum_row_groups(rows, N);
   SKY_CHECK(ws && ws_bytes >= (size_t)groups * N * sizeof(float), SKY_ERR_INVALID_ARG,
             "column-sum workspace too small");
@@ -390,8 +492,8 @@ sky_status column_sum(const void* x, int rows, int N, sky_dtype dt, float* out, 
         static_cast<const __nv_bfloat16*>(x), rows, N, part);
   else
     rw::colsum_partial<float><<<grid, 256, 0, st>>>(static_cast<const float*>(x), rows, N, part);
-  rw::reduce_partials<<<dim3(ceil_div(N, 256), 1), 256, 0, st>>>(part, groups, N, out, nullptr,
-                                                                 nullptr);
+  rw::reduce_partials<<<dim3(ceil_div(N, 32), 1), 256, 0, st>>>(part, groups, N, out, nullptr,
+                                                                nullptr);
   count_launches(2);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "column sum launch");

@@ -13,14 +13,17 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
                          const int32_t* lens, int B, int S, int H, int A, sky_dtype dt, void* dqkv,
                          float* delta, int32_t* status, cudaStream_t st);
 
-sky_status layernorm_fwd(const float* u, const void* gamma, const void* beta, int rows, int H,
-                         float eps, sky_dtype dt, float* y32, void* y, float* mean, float* rstd,
-                         cudaStream_t st);
+sky_status layernorm_fwd(const float* a, const float* r, const void* gamma, const void* beta,
+                         int rows, int H, float eps, sky_dtype dt, float* u_out, float* y32,
+                         void* y, float* mean, float* rstd, cudaStream_t st);
 size_t layernorm_bwd_ws(int rows, int H);
-sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* u, const void* gamma,
-                         const float* mean, const float* rstd, int rows, int H, sky_dtype dt,
-                         float* du32, void* du, float* dgamma, float* dbeta, float* dbias,
-                         void* ws, size_t ws_bytes, cudaStream_t st);
+sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, const float* u,
+                         const void* gamma, const float* mean, const float* rstd, int rows, int H,
+                         sky_dtype dt, float* du32, void* du, float* dgamma, float* dbeta,
+                         float* dbias, void* ws, size_t ws_bytes, cudaStream_t st);
+sky_status add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dt, void* out,
+                   cudaStream_t st);
+sky_status f32_to_bf16(const float* x, int64_t n, void* out, cudaStream_t st);
 sky_status to_f32(const void* x, int64_t n, sky_dtype dt, float* out, cudaStream_t st);
 size_t column_sum_ws(int rows, int N);
 sky_status column_sum(const void* x, int rows, int N, sky_dtype dt, float* out, void* ws,

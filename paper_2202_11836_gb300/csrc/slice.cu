@@ -77,7 +77,7 @@ static const char* kCatNames[P_NCAT] = {"gemm_fwd", "gemm_dgrad", "gemm_wgrad", 
 struct LayerBufs {
   void* p[SKY_NUM_PARAMS];
   float* g[SKY_NUM_PARAMS];
-  void *Xb, *QKV, *ctx, *X1b, *Hpre, *G;
+  void *Xb, *QKV, *ctx, *X1b, *Gp, *G;  // Gp = GELU'(Z) (fp16 in bf16 slices)
   float *X32, *U1, *X1_32, *U2;
   float *lse, *mean1, *rstd1, *mean2, *rstd2;
 };
@@ -93,7 +93,10 @@ struct sky_slice {
   void* arena = nullptr;
   uint64_t param_bytes = 0, grad_bytes = 0, stash_bytes = 0, ws_bytes_total = 0;
   std::vector<sky::LayerBufs> layers;
-  float *g32a, *g32b, *dU2_32, *dX1_32, *dU1_32;  // fp32 gradient stream
+  // fp32 gradient stream.  Between layers it travels as two terms that the
+  // next LayerNorm backward adds: dP[k] (dQKV Wqkv) and dR[k] (dU1, the
+  // residual branch); k alternates per layer.
+  float *dP[2], *dR[2], *dU2_32, *dP1;
   void *dU2b, *dU1b, *dH, *dctx, *dqkv;           // dtype copies / branch gradients
   float* delta;
   void* ws;
@@ -211,31 +214,33 @@ sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
     Timed t(s, st, P_ATTN_FWD, 4.0 * H * S * (double)T, e * T * 4.0 * H);
     SKY_TRY(attention_fwd(Lb.QKV, s->d_len, B, S, H, A, dt, Lb.ctx, Lb.lse, s->d_status, st));
   }
-  // a3 + residual: U1 = ctx Wo^T + bo + X  (fp32)
+  // a3: U1 = ctx Wo^T + bo  (fp32; the residual is added by the LayerNorm)
   SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, H, Lb.ctx, Lb.p[2], Lb.U1, true,
-                   SKY_EPI_RESIDUAL, Lb.p[3], Lb.X32, nullptr));
-  // a4: X1 = LN(U1)
+                   SKY_EPI_STORE, Lb.p[3], nullptr, nullptr));
+  // a4: U1 += X; X1 = LN(U1)
   {
-    Timed t(s, st, P_LN_FWD, 0, 4.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
-    SKY_TRY(layernorm_fwd(Lb.U1, Lb.p[4], Lb.p[5], T, H, s->cfg.ln_eps, dt,
+    Timed t(s, st, P_LN_FWD, 0, 12.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_fwd(Lb.U1, Lb.X32, Lb.p[4], Lb.p[5], T, H, s->cfg.ln_eps, dt, Lb.U1,
                           dt == SKY_DTYPE_BF16 ? Lb.X1_32 : nullptr, Lb.X1b, Lb.mean1, Lb.rstd1,
                           st));
   }
-  // a5 + a6: Hpre = X1 W1^T + b1, G = GELU(Hpre) (fused epilogue)
-  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, F, H, Lb.X1b, Lb.p[6], Lb.Hpre, false,
-                   SKY_EPI_BIAS_GELU, Lb.p[7], nullptr, Lb.G));
-  // a7 + residual: U2 = G W2^T + b2 + X1  (fp32)
+  // a5 + a6: Z = X1 W1^T + b1; G = GELU(Z) and GELU'(Z) for the backward (fused epilogue)
+  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, F, H, Lb.X1b, Lb.p[6], Lb.G, false,
+                   SKY_EPI_BIAS_GELU, Lb.p[7], nullptr, Lb.Gp));
+  // a7: U2 = G W2^T + b2  (fp32)
   SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, F, Lb.G, Lb.p[8], Lb.U2, true,
-                   SKY_EPI_RESIDUAL, Lb.p[9], Lb.X1_32, nullptr));
-  // a8: Y = LN(U2) -> next layer's input (fp32 + dtype copy) or the caller's y
+                   SKY_EPI_STORE, Lb.p[9], nullptr, nullptr));
+  // a8: U2 += X1; Y = LN(U2) -> next layer's input (fp32 + dtype copy) or the caller's y
   {
-    Timed t(s, st, P_LN_FWD, 0, 4.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
+    Timed t(s, st, P_LN_FWD, 0, 12.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
     if (y_out) {
-      SKY_TRY(layernorm_fwd(Lb.U2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, nullptr, y_out,
+      const bool f32 = dt == SKY_DTYPE_BF16 && s->cfg.io_fp32;
+      SKY_TRY(layernorm_fwd(Lb.U2, Lb.X1_32, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, Lb.U2,
+                            f32 ? static_cast<float*>(y_out) : nullptr, f32 ? nullptr : y_out,
                             Lb.mean2, Lb.rstd2, st));
     } else {
       LayerBufs& Nx = s->layers[i + 1];
-      SKY_TRY(layernorm_fwd(Lb.U2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt,
+      SKY_TRY(layernorm_fwd(Lb.U2, Lb.X1_32, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, Lb.U2,
                             dt == SKY_DTYPE_BF16 ? Nx.X32 : nullptr, Nx.Xb, Lb.mean2, Lb.rstd2,
                             st));
     }
@@ -244,49 +249,51 @@ sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
 }
 
 // ----------------------------------------------------------------- backward
-// One layer, steps a9..a16.  dY: dtype (top layer, from the caller) or fp32;
-// dX: fp32 stream buffer, or the caller's dx (dtype) for the first layer.
-sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, void* dX,
-                          bool dx_f32, cudaStream_t st) {
+// One layer, steps a9..a16.  The upstream gradient is dY + dY2: dY in dy_dt
+// (the caller's dy for the top layer) and dY2 fp32 or null.  Outputs go to
+// dP[k] and dR[k]; for the slice's first layer they are added into dx.
+sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, const float* dY2,
+                          int k, void* dx, cudaStream_t st) {
   LayerBufs& Lb = s->layers[i];
   const int B = s->B, S = s->S, H = s->H, A = s->A, F = s->F;
   const int T = B * S;
   const sky_dtype dt = s->cfg.dtype;
   const bool bf = dt == SKY_DTYPE_BF16;
   const double e = (double)s->esz;
-  const double dye = dy_dt == SKY_DTYPE_BF16 ? 2.0 : 4.0;
+  const double dye = (dy_dt == SKY_DTYPE_BF16 ? 2.0 : 4.0) + (dY2 ? 4.0 : 0.0);
+  void* dU1b = bf ? s->dU1b : s->dR[k];
   // a9: LN2 backward -> dU2 (fp32 + dtype), dgamma2, dbeta2, db2
   {
     Timed t(s, st, P_LN_BWD, 0, (dye + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
-    SKY_TRY(layernorm_bwd(dY, dy_dt, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
+    SKY_TRY(layernorm_bwd(dY, dy_dt, dY2, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
                           bf ? s->dU2_32 : nullptr, s->dU2b, Lb.g[10], Lb.g[11], Lb.g[9], s->ws,
                           s->ws_bytes, st));
   }
-  // a10 + a11: dHpre = (dU2 W2) * GELU'(Hpre);  dW2 = dU2^T G
+  // a10 + a11: dZ = (dU2 W2) * GELU'(Z);  dW2 = dU2^T G
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
-                   SKY_EPI_GELU_BWD, nullptr, Lb.Hpre, nullptr));
+                   SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr));
   SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
   {
     Timed t(s, st, P_COLSUM, 0, e * T * F);
     SKY_TRY(column_sum(s->dH, T, F, dt, Lb.g[7], s->ws, s->ws_bytes, st));
   }
-  // a12: dX1 = dHpre W1 + dU2 (fp32);  dW1 = dHpre^T X1
-  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dX1_32, true,
-                   SKY_EPI_RESIDUAL, nullptr, s->dU2_32, nullptr));
+  // a12: P1 = dZ W1 (fp32; dX1 = P1 + dU2 is formed by the LN1 backward);  dW1 = dZ^T X1
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dP1, true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
   SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, F, H, T, s->dH, Lb.X1b, Lb.g[6], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
-  // a13: LN1 backward -> dU1 (fp32 + dtype), dgamma1, dbeta1, dbo
+  // a13: LN1 backward of dX1 = P1 + dU2 -> dU1 (fp32 + dtype), dgamma1, dbeta1, dbo
   {
-    Timed t(s, st, P_LN_BWD, 0, (4.0 + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
-    SKY_TRY(layernorm_bwd(s->dX1_32, SKY_DTYPE_FP32, Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H,
-                          dt, bf ? s->dU1_32 : nullptr, s->dU1b, Lb.g[4], Lb.g[5], Lb.g[3], s->ws,
-                          s->ws_bytes, st));
+    Timed t(s, st, P_LN_BWD, 0, (4.0 + 4.0 + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? s->dU2_32 : static_cast<float*>(s->dU2b),
+                          Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H, dt, bf ? s->dR[k] : nullptr,
+                          dU1b, Lb.g[4], Lb.g[5], Lb.g[3], s->ws, s->ws_bytes, st));
   }
   // a14: dctx = dU1 Wo;  dWo = dU1^T ctx
-  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, H, s->dU1b, Lb.p[2], s->dctx, false,
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, H, dU1b, Lb.p[2], s->dctx, false,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
-  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, H, T, s->dU1b, Lb.ctx, Lb.g[2], true,
+  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, H, T, dU1b, Lb.ctx, Lb.g[2], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
   // a15: attention backward -> dQKV
   {
@@ -298,9 +305,15 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, st, P_COLSUM, 0, e * T * 3.0 * H);
     SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], s->ws, s->ws_bytes, st));
   }
-  // a16: dX = dQKV Wqkv + dU1;  dWqkv = dQKV^T X
-  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, 3 * H, s->dqkv, Lb.p[0], dX, dx_f32,
-                   SKY_EPI_RESIDUAL, nullptr, bf ? s->dU1_32 : s->dU1b, nullptr));
+  // a16: dX = dQKV Wqkv + dU1 (the sum is formed by the next LayerNorm backward,
+  // or here for the slice's first layer);  dWqkv = dQKV^T X
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, 3 * H, s->dqkv, Lb.p[0], s->dP[k], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  if (dx) {
+    Timed t(s, st, P_COPY, 0, (8.0 + ((bf && !s->cfg.io_fp32) ? 2.0 : 4.0)) * T * H);
+    SKY_TRY(add_f32(s->dP[k], s->dR[k], (int64_t)T * H,
+                    s->cfg.io_fp32 ? SKY_DTYPE_FP32 : dt, dx, st));
+  }
   SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, 3 * H, H, T, s->dqkv, Lb.Xb, Lb.g[0], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
   return SKY_OK;
@@ -311,9 +324,14 @@ sky_status forward_all(sky_slice* s, const void* x, void* y, cudaStream_t st,
   const int64_t n = (int64_t)s->B * s->S * s->H;
   {
     Timed t(s, st, P_COPY, 0, (2.0 * s->esz + (s->esz == 2 ? 6.0 : 0.0)) * n);
-    SKY_CUDA(cudaMemcpyAsync(s->layers[0].Xb, x, n * s->esz, cudaMemcpyDeviceToDevice, st));
-    if (s->cfg.dtype == SKY_DTYPE_BF16)
-      SKY_TRY(to_f32(x, n, s->cfg.dtype, s->layers[0].X32, st));
+    LayerBufs& L0 = s->layers[0];
+    if (s->cfg.dtype == SKY_DTYPE_BF16 && s->cfg.io_fp32) {
+      SKY_CUDA(cudaMemcpyAsync(L0.X32, x, n * 4, cudaMemcpyDeviceToDevice, st));
+      SKY_TRY(f32_to_bf16(L0.X32, n, L0.Xb, st));
+    } else {
+      SKY_CUDA(cudaMemcpyAsync(L0.Xb, x, n * s->esz, cudaMemcpyDeviceToDevice, st));
+      if (s->cfg.dtype == SKY_DTYPE_BF16) SKY_TRY(to_f32(x, n, s->cfg.dtype, L0.X32, st));
+    }
   }
   for (int i = 0; i < s->L; ++i) {
     if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i], st));
@@ -326,14 +344,15 @@ sky_status forward_all(sky_slice* s, const void* x, void* y, cudaStream_t st,
 sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
                         std::vector<cudaEvent_t>* marks) {
   const void* cur = dy;
-  sky_dtype cur_dt = s->cfg.dtype;
+  const float* cur2 = nullptr;
+  sky_dtype cur_dt = s->cfg.io_fp32 ? SKY_DTYPE_FP32 : s->cfg.dtype;
   for (int i = s->L - 1; i >= 0; --i) {
-    const bool last = i == 0;
-    void* out = last ? dx : ((s->L - 1 - i) % 2 == 0 ? (void*)s->g32a : (void*)s->g32b);
+    const int k = (s->L - 1 - i) & 1;
     if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i], st));
-    SKY_TRY(backward_layer(s, i, cur, cur_dt, out, !last, st));
+    SKY_TRY(backward_layer(s, i, cur, cur_dt, cur2, k, i == 0 ? dx : nullptr, st));
     if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
-    cur = out;
+    cur = s->dP[k];
+    cur2 = s->dR[k];
     cur_dt = SKY_DTYPE_FP32;
   }
   return SKY_OK;
@@ -417,7 +436,7 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   const size_t t32 = align_up((size_t)T * s->H * 4);
   const bool bf = c.dtype == SKY_DTYPE_BF16;
   const size_t lse = align_up((size_t)c.max_batch * s->A * c.max_seq * 4);
-  // Xb ctx X1b | QKV | Hpre G | U1 U2 (+ X32 X1_32 for bf16) | lse | 4 stats
+  // Xb ctx X1b | QKV | Gp G | U1 U2 (+ X32 X1_32 for bf16) | lse | 4 stats
   const size_t stash = 3 * th + align_up((size_t)T * 3 * s->H * s->esz) +
                        2 * align_up((size_t)T * s->F * s->esz) + (bf ? 4 : 2) * t32 + lse +
                        4 * align_up((size_t)T * 4);
@@ -425,8 +444,8 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   s->grad_bytes = gb * s->L;
   s->stash_bytes = stash * s->L;
   s->ws_bytes = align_up(workspace_need(s, T));
-  // g32a g32b dU2_32 dX1_32 dU1_32 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | status
-  const size_t wk = 5 * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
+  // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | status
+  const size_t wk = 6 * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
                     align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes + 256;
   s->ws_bytes_total = wk;
   *total = s->param_bytes + s->grad_bytes + s->stash_bytes + wk;
@@ -447,6 +466,7 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   SKY_CHECK(c.dtype == SKY_DTYPE_BF16 || c.dtype == SKY_DTYPE_FP32, SKY_ERR_INVALID_ARG,
             "unknown dtype");
   SKY_CHECK(c.ln_eps >= 0.f, SKY_ERR_INVALID_ARG, "ln_eps must be >= 0");
+  SKY_CHECK(c.io_fp32 == 0 || c.io_fp32 == 1, SKY_ERR_INVALID_ARG, "io_fp32 must be 0 or 1");
   const int D = c.width / c.heads;
   if (c.dtype == SKY_DTYPE_BF16) {
     SKY_CHECK(D == 64, SKY_ERR_UNSUPPORTED, "bf16 slices need head dim 64 (got %d)", D);
@@ -507,7 +527,7 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
     for (int k = 0; k < SKY_NUM_PARAMS; ++k) Lb.g[k] = static_cast<float*>(take(param_elems(s, k) * 4));
     Lb.Xb = take(th); Lb.ctx = take(th); Lb.X1b = take(th);
     Lb.QKV = take((size_t)T * 3 * s->H * s->esz);
-    Lb.Hpre = take((size_t)T * s->F * s->esz);
+    Lb.Gp = take((size_t)T * s->F * s->esz);
     Lb.G = take((size_t)T * s->F * s->esz);
     Lb.U1 = static_cast<float*>(take(t32));
     Lb.U2 = static_cast<float*>(take(t32));
@@ -519,13 +539,14 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
     Lb.mean2 = static_cast<float*>(take((size_t)T * 4));
     Lb.rstd2 = static_cast<float*>(take((size_t)T * 4));
   }
-  s->g32a = static_cast<float*>(take(t32));
-  s->g32b = static_cast<float*>(take(t32));
+  for (int k = 0; k < 2; ++k) {
+    s->dP[k] = static_cast<float*>(take(t32));
+    s->dR[k] = static_cast<float*>(take(t32));
+  }
   s->dU2_32 = static_cast<float*>(take(t32));
-  s->dX1_32 = static_cast<float*>(take(t32));
-  s->dU1_32 = static_cast<float*>(take(t32));
+  s->dP1 = static_cast<float*>(take(t32));
   s->dU2b = bf ? take(th) : s->dU2_32;
-  s->dU1b = bf ? take(th) : s->dU1_32;
+  s->dU1b = bf ? take(th) : nullptr;  // fp32 slices use dR[k] directly
   s->dctx = take(th);
   s->dH = take((size_t)T * s->F * s->esz);
   s->dqkv = take((size_t)T * 3 * s->H * s->esz);
@@ -648,7 +669,8 @@ sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, int32_t iter
   SKY_CHECK(n_out == s->L, SKY_ERR_INVALID_ARG, "n_out must be %d", s->L);
   SKY_CHECK(iters >= 1 && B >= 1 && S >= 1 && B <= s->cfg.max_batch && S <= s->cfg.max_seq,
             SKY_ERR_INVALID_ARG, "bad B/S/iters");
-  const size_t xb = (size_t)B * S * s->H * s->esz;
+  const bool io32 = s->cfg.io_fp32 && s->cfg.dtype == SKY_DTYPE_BF16;
+  const size_t xb = (size_t)B * S * s->H * (io32 ? 4 : s->esz);
   void *x = nullptr, *y = nullptr, *dy = nullptr, *dx = nullptr;
   int32_t* len = nullptr;
   SKY_CUDA(cudaMalloc(&x, xb));
@@ -659,7 +681,7 @@ sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, int32_t iter
   cudaStream_t st;
   SKY_CUDA(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
   const int64_t n = (int64_t)B * S * s->H;
-  const int bf = s->cfg.dtype == SKY_DTYPE_BF16;
+  const int bf = s->cfg.dtype == SKY_DTYPE_BF16 && !io32;
   fill_pattern<<<256, 256, 0, st>>>(x, n, bf, 1.0f, 1u);
   fill_pattern<<<256, 256, 0, st>>>(dy, n, bf, 1e-3f, 2u);
   fill_int<<<ceil_div(B, 256), 256, 0, st>>>(len, B, S);
@@ -795,7 +817,7 @@ sky_status sky_gemm(sky_gemm_form form, int32_t M, int32_t N, int32_t K, sky_dty
   SKY_CHECK(A && B && C, SKY_ERR_INVALID_ARG, "null operand");
   SKY_CHECK(M > 0 && N > 0 && K > 0, SKY_ERR_INVALID_ARG, "sizes must be positive");
   SKY_CHECK(form >= SKY_GEMM_XWT && form <= SKY_GEMM_XTW, SKY_ERR_INVALID_ARG, "bad form");
-  SKY_CHECK(epilogue >= SKY_EPI_STORE && epilogue <= SKY_EPI_RESIDUAL, SKY_ERR_INVALID_ARG,
+  SKY_CHECK(epilogue >= SKY_EPI_STORE && epilogue <= SKY_EPI_GELU_BWD, SKY_ERR_INVALID_ARG,
             "bad epilogue");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (in_dtype == SKY_DTYPE_BF16)
@@ -840,14 +862,15 @@ sky_status sky_attention_bwd(const void* qkv, const void* ctx, const void* dctx,
   ABI_GUARD_END
 }
 
-sky_status sky_layernorm_fwd(const float* u, const void* gamma, const void* beta, int32_t T,
-                             int32_t H, float eps, sky_dtype dtype, float* y32, void* y,
-                             float* mean, float* rstd, void* stream) {
+sky_status sky_layernorm_fwd(const float* a, const float* r, const void* gamma,
+                             const void* beta, int32_t T, int32_t H, float eps, sky_dtype dtype,
+                             float* u_out, float* y32, void* y, float* mean, float* rstd,
+                             void* stream) {
   ABI_GUARD_BEGIN
-  SKY_CHECK(u && gamma && beta && (y32 || y) && mean && rstd, SKY_ERR_INVALID_ARG,
+  SKY_CHECK(a && gamma && beta && (y32 || y) && mean && rstd, SKY_ERR_INVALID_ARG,
             "null argument");
   SKY_CHECK(T > 0 && H > 0, SKY_ERR_INVALID_ARG, "bad sizes");
-  return layernorm_fwd(u, gamma, beta, T, H, eps, dtype, y32, y, mean, rstd,
+  return layernorm_fwd(a, r, gamma, beta, T, H, eps, dtype, u_out, y32, y, mean, rstd,
                        static_cast<cudaStream_t>(stream));
   ABI_GUARD_END
 }
@@ -857,19 +880,27 @@ size_t sky_layernorm_bwd_workspace_bytes(int32_t T, int32_t H) {
   return layernorm_bwd_ws(T, H);
 }
 
-sky_status sky_layernorm_bwd(const void* dy, sky_dtype dy_dtype, const float* u,
-                             const void* gamma, const float* mean, const float* rstd, int32_t T,
-                             int32_t H, sky_dtype dtype, float* du32, void* du, float* dgamma,
-                             float* dbeta, float* dbias, void* workspace, size_t workspace_bytes,
-                             void* stream) {
+sky_status sky_layernorm_bwd(const void* dy, sky_dtype dy_dtype, const float* dy2,
+                             const float* u, const void* gamma, const float* mean,
+                             const float* rstd, int32_t T, int32_t H, sky_dtype dtype,
+                             float* du32, void* du, float* dgamma, float* dbeta, float* dbias,
+                             void* workspace, size_t workspace_bytes, void* stream) {
   ABI_GUARD_BEGIN
   SKY_CHECK(dy && u && gamma && mean && rstd && (du32 || du), SKY_ERR_INVALID_ARG,
             "null argument");
   SKY_CHECK(T > 0 && H > 0, SKY_ERR_INVALID_ARG, "bad sizes");
   SKY_CHECK(dy_dtype == SKY_DTYPE_FP32 || dy_dtype == dtype, SKY_ERR_INVALID_ARG,
             "dy must be fp32 or the slice dtype");
-  return layernorm_bwd(dy, dy_dtype, u, gamma, mean, rstd, T, H, dtype, du32, du, dgamma, dbeta,
-                       dbias, workspace, workspace_bytes, static_cast<cudaStream_t>(stream));
+  return layernorm_bwd(dy, dy_dtype, dy2, u, gamma, mean, rstd, T, H, dtype, du32, du, dgamma,
+                       dbeta, dbias, workspace, workspace_bytes, static_cast<cudaStream_t>(stream));
+  ABI_GUARD_END
+}
+
+sky_status sky_add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dtype, void* out,
+                       void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(a && b && out && n >= 0, SKY_ERR_INVALID_ARG, "bad argument");
+  return add_f32(a, b, n, out_dtype, out, static_cast<cudaStream_t>(stream));
   ABI_GUARD_END
 }
 

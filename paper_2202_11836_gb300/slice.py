@@ -29,13 +29,15 @@ class EncoderSlice:
     """Layers [layer_begin, layer_end) with hidden width H, A heads and FFN width F."""
 
     def __init__(self, width: int, heads: int, ffn: int, layer_begin: int, layer_end: int,
-                 max_batch: int, max_seq: int, dtype: str = "bf16", ln_eps: float = 1e-12):
+                 max_batch: int, max_seq: int, dtype: str = "bf16", ln_eps: float = 1e-12,
+                 io_fp32: bool = False):
         self.H, self.A, self.F = width, heads, ffn
         self.layer_begin, self.layer_end = layer_begin, layer_end
         self.dtype = dtype
+        self.io_fp32 = io_fp32
         cfg = L.SkySliceConfig(width, heads, ffn, layer_begin, layer_end, max_batch, max_seq,
                                L.SKY_DTYPE_BF16 if dtype == "bf16" else L.SKY_DTYPE_FP32,
-                               ln_eps)
+                               ln_eps, 1 if io_fp32 else 0)
         h = C.c_void_p()
         L.call("sky_slice_create", C.byref(cfg), C.byref(h))
         self.h = h
