@@ -143,6 +143,27 @@ size_t sky_column_sum_workspace_bytes(int32_t T, int32_t N);
 sky_status sky_column_sum(const void* x, int32_t T, int32_t N, sky_dtype dtype, float* out,
                           void* workspace, size_t workspace_bytes, void* stream);
 
+/* sky_column_sum without any device allocation, for callers that cannot
+ * allocate: code that takes all device memory from a fixed pool it does not
+ * own (a framework's caching allocator, a pre-sized arena) must not call
+ * cudaMalloc around it, and code that must not allocate inside its step loop
+ * cannot supply a fresh workspace per call.  (The paper has no counterpart;
+ * this is a library-usability variant of the bias-gradient reduction.)
+ * Same arguments and result as sky_column_sum minus the workspace: the
+ * partial sums live in a 1 MiB device array inside the library, which every
+ * device that loads the library holds until the process exits.
+ *   - The first call on a device looks up that array's device address
+ *     (cudaGetSymbolAddress) with the device current; make that first call
+ *     before capturing the stream into a CUDA graph.
+ *   - All calls share the array and it keeps the previous call's contents;
+ *     nothing in it needs to start at zero, but calls that may overlap on
+ *     the GPU (different streams, or different host threads, same device)
+ *     race on it and must be serialised by the caller.
+ *   - Sizes whose partials exceed 1 MiB are rejected with INVALID_ARG (on a
+ *     152-SM GB300 that is N > 262144, for any T); use sky_column_sum then. */
+sky_status sky_column_sum_noalloc(const void* x, int32_t T, int32_t N, sky_dtype dtype,
+                                  float* out, void* stream);
+
 /* Number of streaming multiprocessors of the current device (0 on error). */
 int32_t sky_device_sm_count(void);
 

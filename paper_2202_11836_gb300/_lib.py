@@ -89,6 +89,7 @@ _SIGNATURES = {
     "sky_gelu_bwd": (C.c_int, [_VP, _VP, _I32, _I32, C.c_int, _VP, _VP]),
     "sky_column_sum_workspace_bytes": (_SZ, [_I32, _I32]),
     "sky_column_sum": (C.c_int, [_VP, _I32, _I32, C.c_int, _VP, _VP, _SZ, _VP]),
+    "sky_column_sum_noalloc": (C.c_int, [_VP, _I32, _I32, C.c_int, _VP, _VP]),
     "sky_device_sm_count": (_I32, []),
 }
 
