@@ -164,6 +164,15 @@ sky_status sky_column_sum(const void* x, int32_t T, int32_t N, sky_dtype dtype, 
 sky_status sky_column_sum_noalloc(const void* x, int32_t T, int32_t N, sky_dtype dtype,
                                   float* out, void* stream);
 
+/* Test hook of the tensor-core GEMM's failure path (not for production use).
+ * limit_ns caps every mbarrier wait of GEMM launches made after the call
+ * (0 restores the default, 2 s).  skip_loads != 0 makes the TMA producer
+ * arrive on its barriers without issuing the copies, so the consumers' waits
+ * run out: the kernel then sets the timeout bit (2) of the status word it was
+ * given, frees its tensor memory and exits, and the context stays usable.
+ * Process-wide setting; pass (0, 0) to restore normal operation. */
+void sky_debug_gemm_fault(uint64_t limit_ns, int32_t skip_loads);
+
 /* Number of streaming multiprocessors of the current device (0 on error). */
 int32_t sky_device_sm_count(void);
 

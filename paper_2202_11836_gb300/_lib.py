@@ -90,6 +90,7 @@ _SIGNATURES = {
     "sky_column_sum_workspace_bytes": (_SZ, [_I32, _I32]),
     "sky_column_sum": (C.c_int, [_VP, _I32, _I32, C.c_int, _VP, _VP, _SZ, _VP]),
     "sky_column_sum_noalloc": (C.c_int, [_VP, _I32, _I32, C.c_int, _VP, _VP]),
+    "sky_debug_gemm_fault": (None, [C.c_uint64, C.c_int32]),
     "sky_device_sm_count": (_I32, []),
 }
 

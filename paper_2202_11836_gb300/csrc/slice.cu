@@ -422,6 +422,10 @@ const char* sky_last_error(void) { return g_last_error.c_str(); }
 
 int32_t sky_device_sm_count(void) { return sm_count(); }
 
+void sky_debug_gemm_fault(uint64_t limit_ns, int32_t skip_loads) {
+  gemm::set_debug(limit_ns, skip_loads);
+}
+
 // Sizes of the arena carved at create, computed on the host only.
 static sky_status plan_slice(sky_slice* s, size_t* total) {
   const sky_slice_config& c = s->cfg;
