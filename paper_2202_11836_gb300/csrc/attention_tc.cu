@@ -43,6 +43,10 @@ constexpr int TMEM_COLS = 128;  // S: columns [0, 64), O: [64, 128)
 constexpr int NTHR = 192;       // warp 0 TMA, warp 1 MMA, warps 2..5 softmax
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr float LN2 = 0.6931471805599453f;
+// Suspend-time hint (ns) of every mbarrier wait: a waiting thread sleeps
+// until the phase completes instead of spinning on issue slots that the
+// softmax warps (the critical path) share with the producer and MMA threads.
+constexpr uint32_t kWaitHint = 10000;
 
 struct FwdParams {
   int S, H, A;
@@ -114,7 +118,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
       for (int j = 0; j < n_kt && ok; ++j) {
         const int st = j & 1;
         const uint32_t ph = (j >> 1) & 1;
-        if (!ptx::mbar_wait(&kv_empty[st], ph ^ 1u, lim, p.status)) { ok = false; break; }
+        if (!ptx::mbar_wait(&kv_empty[st], ph ^ 1u, lim, p.status, kWaitHint)) { ok = false; break; }
         ptx::mbar_arrive_expect_tx(&kv_full[st], 2 * KV_BYTES);
         ptx::tma_load_2d(smem + K_OFF + st * KV_BYTES, &tmKV, &kv_full[st], H + a * HD,
                          row0 + j * BKV);
@@ -123,9 +127,9 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
         ++issued;
       }
       // drain: bounded waits for the copies still in flight
-      ptx::mbar_wait(q_full, 0, lim, p.status);
+      ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint);
       for (int j = issued - 1; j >= 0 && j >= issued - STAGES; --j)
-        ptx::mbar_wait(&kv_full[j & 1], (j >> 1) & 1, lim, p.status);
+        ptx::mbar_wait(&kv_full[j & 1], (j >> 1) & 1, lim, p.status, kWaitHint);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------- MMA issue
@@ -133,11 +137,11 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
       constexpr uint32_t idS = ptx::idesc_bf16_f32(BQ, BKV, false, false);
       constexpr uint32_t idO = ptx::idesc_bf16_f32(BQ, HD, false, true);
       const uint32_t sq = ptx::smem_u32(smem + Q_OFF), sp = ptx::smem_u32(smem + P_OFF);
-      bool ok = ptx::mbar_wait(q_full, 0, lim, p.status);
+      bool ok = ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint);
       for (int j = 0; j < n_kt && ok; ++j) {
         const int st = j & 1;
         const uint32_t ph = (j >> 1) & 1;
-        if (!ptx::mbar_wait(&kv_full[st], ph, lim, p.status)) break;
+        if (!ptx::mbar_wait(&kv_full[st], ph, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
         const uint32_t sk = ptx::smem_u32(smem + K_OFF + st * KV_BYTES);
         const uint32_t sv = ptx::smem_u32(smem + V_OFF + st * KV_BYTES);
@@ -146,7 +150,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
           ptx::tc_mma_f16(tS, ptx::smem_desc_sw128(sq + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(sk + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
         ptx::tc_commit(s_full);
-        if (!ptx::mbar_wait(p_full, j & 1, lim, p.status)) break;
+        if (!ptx::mbar_wait(p_full, j & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < BKV / 16; ++kk)
@@ -157,7 +161,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
         ptx::tc_commit(&kv_empty[st]);
       }
       ptx::tc_commit(done);
-      ptx::mbar_wait(done, 0, lim, p.status);
+      ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
     }
   } else {
     // --------------------------------------------------- softmax / epilogue
@@ -171,7 +175,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
     // every lane waits (bounded); the outcome is made warp-uniform so the
     // warp-collective tcgen05 loads and votes below never see a split warp
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
-      const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, 2000);
+      const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, kWaitHint);
       return __all_sync(0xffffffffu, mine);
     };
     for (int j = 0; j < n_kt; ++j) {
@@ -227,7 +231,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
         ptx::tmem_ld_wait();
         float pv[32];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) pv[i] = exp2f(fmaf(__uint_as_float(v[i]), sl2, nm));
+        for (int i = 0; i < 32; ++i) pv[i] = ptx::ex2_ftz(fmaf(__uint_as_float(v[i]), sl2, nm));
         if (!full_tile) {
 #pragma unroll
           for (int i = 0; i < 32; ++i)
@@ -368,7 +372,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
       int issued = 0;
       for (int j = 0; j < n_kt; ++j) {
         const int st = j & 1;
-        if (!ptx::mbar_wait(&kv_empty[st], ((j >> 1) & 1) ^ 1u, lim, p.status)) break;
+        if (!ptx::mbar_wait(&kv_empty[st], ((j >> 1) & 1) ^ 1u, lim, p.status, kWaitHint)) break;
         ptx::mbar_arrive_expect_tx(&kv_full[st], 2 * KV_BYTES);
         ptx::tma_load_2d(smem + DQ_K_OFF + st * KV_BYTES, &tmKV, &kv_full[st], H + a * HD,
                          row0 + j * BKV);
@@ -376,9 +380,9 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
                          row0 + j * BKV);
         ++issued;
       }
-      ptx::mbar_wait(qd_full, 0, lim, p.status);
+      ptx::mbar_wait(qd_full, 0, lim, p.status, kWaitHint);
       for (int j = issued - 1; j >= 0 && j >= issued - STAGES; --j)
-        ptx::mbar_wait(&kv_full[j & 1], (j >> 1) & 1, lim, p.status);
+        ptx::mbar_wait(&kv_full[j & 1], (j >> 1) & 1, lim, p.status, kWaitHint);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -386,10 +390,10 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
       constexpr uint32_t idQ = ptx::idesc_bf16_f32(BQ, HD, false, true);
       const uint32_t sq = ptx::smem_u32(smem + DQ_Q_OFF), so = ptx::smem_u32(smem + DQ_DO_OFF);
       const uint32_t sds = ptx::smem_u32(smem + DQ_DS_OFF);
-      bool ok = ptx::mbar_wait(qd_full, 0, lim, p.status);
+      bool ok = ptx::mbar_wait(qd_full, 0, lim, p.status, kWaitHint);
       for (int j = 0; j < n_kt && ok; ++j) {
         const int st = j & 1;
-        if (!ptx::mbar_wait(&kv_full[st], (j >> 1) & 1, lim, p.status)) break;
+        if (!ptx::mbar_wait(&kv_full[st], (j >> 1) & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
         const uint32_t sk = ptx::smem_u32(smem + DQ_K_OFF + st * KV_BYTES);
         const uint32_t sv = ptx::smem_u32(smem + DQ_V_OFF + st * KV_BYTES);
@@ -402,7 +406,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
           ptx::tc_mma_f16(tdP, ptx::smem_desc_sw128(so + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(sv + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
         ptx::tc_commit(s_full);
-        if (!ptx::mbar_wait(ds_full, j & 1, lim, p.status)) break;
+        if (!ptx::mbar_wait(ds_full, j & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < BKV / 16; ++kk)
@@ -413,7 +417,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
         ptx::tc_commit(&kv_empty[st]);
       }
       ptx::tc_commit(done);
-      ptx::mbar_wait(done, 0, lim, p.status);
+      ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
     }
   } else {
     const int q4 = warp & 3;
@@ -427,7 +431,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
     uint8_t* drow = smem + DQ_DS_OFF + r * 128;
     bool ok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
-      const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, 2000);
+      const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, kWaitHint);
       return __all_sync(0xffffffffu, mine);
     };
     for (int j = 0; j < n_kt; ++j) {
@@ -445,7 +449,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
         float ds[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float pr = exp2f(fmaf(__uint_as_float(sv[i]), sl2, nlse2));
+          const float pr = ptx::ex2_ftz(fmaf(__uint_as_float(sv[i]), sl2, nlse2));
           ds[i] = pr * (__uint_as_float(dv[i]) - dl);
         }
         if (!full_tile) {
@@ -594,7 +598,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
     for (int i = 0; i < n_qt; ++i) {
       const int st = i & 1;
       bool ok = true;
-      if (lane == 0) ok = ptx::mbar_wait(&q_empty[st], ((i >> 1) & 1) ^ 1u, lim, p.status);
+      if (lane == 0) ok = ptx::mbar_wait(&q_empty[st], ((i >> 1) & 1) ^ 1u, lim, p.status, kWaitHint);
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
       float* l2 = ldst + st * 2 * BQ2;
       for (int t = lane; t < BQ2; t += 32) {
@@ -614,9 +618,9 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
       ++issued;
     }
     if (lane == 0) {
-      ptx::mbar_wait(kv_full, 0, lim, p.status);
+      ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint);
       for (int i = issued - 1; i >= 0 && i >= issued - STAGES; --i)
-        ptx::mbar_wait(&q_full[i & 1], (i >> 1) & 1, lim, p.status);
+        ptx::mbar_wait(&q_full[i & 1], (i >> 1) & 1, lim, p.status, kWaitHint);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -624,10 +628,10 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
       constexpr uint32_t idG = ptx::idesc_bf16_f32(BK2, HD, false, true);
       const uint32_t sk = ptx::smem_u32(smem + KV_K_OFF), sv = ptx::smem_u32(smem + KV_V_OFF);
       const uint32_t sp = ptx::smem_u32(smem + KV_P_OFF), sds = ptx::smem_u32(smem + KV_DS_OFF);
-      bool ok = ptx::mbar_wait(kv_full, 0, lim, p.status);
+      bool ok = ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint);
       for (int i = 0; i < n_qt && ok; ++i) {
         const int st = i & 1;
-        if (!ptx::mbar_wait(&q_full[st], (i >> 1) & 1, lim, p.status)) break;
+        if (!ptx::mbar_wait(&q_full[st], (i >> 1) & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
         const uint32_t sq = ptx::smem_u32(smem + KV_Q_OFF + st * QO2_BYTES);
         const uint32_t so = ptx::smem_u32(smem + KV_O_OFF + st * QO2_BYTES);
@@ -640,7 +644,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
           ptx::tc_mma_f16(tdPT, ptx::smem_desc_sw128(sv + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(so + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
         ptx::tc_commit(s_full);
-        if (!ptx::mbar_wait(pds_full, i & 1, lim, p.status)) break;
+        if (!ptx::mbar_wait(pds_full, i & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < BQ2 / 16; ++kk) {
@@ -655,7 +659,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
         ptx::tc_commit(&q_empty[st]);
       }
       ptx::tc_commit(done);
-      ptx::mbar_wait(done, 0, lim, p.status);
+      ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
     }
   } else {
     const int q4 = warp & 3;
@@ -668,7 +672,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
     uint8_t* drow = smem + KV_DS_OFF + r * 128;
     bool ok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
-      const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, 2000);
+      const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, kWaitHint);
       return __all_sync(0xffffffffu, mine);
     };
     for (int i = 0; i < n_qt; ++i) {
@@ -688,7 +692,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
 #pragma unroll
         for (int t = 0; t < 32; ++t) {
           const int qq = c * 32 + t;
-          pt[t] = kvalid ? exp2f(fmaf(__uint_as_float(sv[t]), sl2, -l2[qq])) : 0.f;
+          pt[t] = kvalid ? ptx::ex2_ftz(fmaf(__uint_as_float(sv[t]), sl2, -l2[qq])) : 0.f;
           ds[t] = pt[t] * (__uint_as_float(dv[t]) - l2[BQ2 + qq]);
         }
 #pragma unroll
