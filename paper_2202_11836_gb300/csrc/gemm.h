@@ -8,10 +8,14 @@ namespace sky {
 namespace gemm {
 
 // bf16 inputs on tcgen05; C is bf16 unless out_f32.
+// colsum (optional, bf16 output, no split): also writes out[n] = sum_m C[m, n]
+// (before rounding), with fixed-order partials in `ws` (m_tiles*4 x N fp32).
 sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
-                       cudaStream_t stream);
+                       cudaStream_t stream, float* colsum = nullptr);
+// out[n] = sum over r of part[r][n] in order r = 0, 1, ... (rowwise.cu).
+cudaError_t reduce_rows_f32(const float* part, int rows, int N, float* out, cudaStream_t stream);
 size_t workspace_bytes(sky_gemm_form form, int M, int N, int K, bool out_f32);
 int choose_splits(int tiles, int k_blocks, int sms);
 // Debug controls: per-wait timeout (0 = default 2 s) and the fault-injection

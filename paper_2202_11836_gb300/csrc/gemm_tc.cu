@@ -57,6 +57,7 @@ struct Params {
   const __nv_bfloat16* bias;      // [N] or null
   const __half* aux;              // [M,N] GELU'(z) (GELU_BWD) or null
   __half* aux_out;                // [M,N] GELU'(z) (BIAS_GELU) or null
+  float* colpart;                 // [m_tiles * 4][N] per-warp column sums of C, or null
   int32_t* status;
   uint64_t timeout_ns;
   int skip_loads;                 // fault injection: producer never issues TMA
@@ -288,6 +289,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                *reinterpret_cast<const uint32_t*>(&h1));
           }
         }
+        if (p.colpart) {
+          // column sums of this warp's 32 rows (the bias gradient), fixed order
+          float cs[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (m0 + q * 32 + 4 * i + rsub < p.M) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j) cs[j] += v[i][j];
+            }
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            cs[j] += __shfl_xor_sync(0xffffffffu, cs[j], 8);
+            cs[j] += __shfl_xor_sync(0xffffffffu, cs[j], 16);
+          }
+          if (rsub == 0 && col_ok)
+            *reinterpret_cast<float4*>(p.colpart + (static_cast<int64_t>(m0 / 32 + q)) * p.N + col) =
+                make_float4(cs[0], cs[1], cs[2], cs[3]);
+        }
         if (col_ok) {
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
@@ -433,7 +452,7 @@ size_t workspace_bytes(sky_gemm_form form, int M, int N, int K, bool out_f32) {
 sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
-                       cudaStream_t stream) {
+                       cudaStream_t stream, float* colsum) {
   // TMA row pitches and the 16-byte epilogue stores need the contiguous
   // dimensions to be multiples of 8 elements; the token dimension is free.
   const bool dims_ok = N % 8 == 0 && (form == SKY_GEMM_XTW ? M % 8 == 0 : K % 8 == 0);
@@ -479,6 +498,15 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   SKY_CHECK(ws_bytes >= need && (need == 0 || ws), SKY_ERR_INVALID_ARG,
             "GEMM workspace too small (%zu < %zu)", ws_bytes, need);
   p.C = p.splits > 1 ? ws : C;
+  // optional fused column sum of C (bf16 outputs only): per-warp partials in
+  // the workspace, added in a fixed order after the kernel
+  const int colpart_rows = p.m_tiles * 4;
+  if (colsum) {
+    SKY_CHECK(!out_f32 && p.splits == 1, SKY_ERR_UNSUPPORTED, "fused column sum needs a bf16 output");
+    SKY_CHECK(ws && ws_bytes >= static_cast<size_t>(colpart_rows) * N * sizeof(float),
+              SKY_ERR_INVALID_ARG, "GEMM column-sum workspace too small");
+    p.colpart = static_cast<float*>(ws);
+  }
   p.bias = static_cast<const __nv_bfloat16*>(bias);
   p.aux = epi == SKY_EPI_GELU_BWD ? static_cast<const __half*>(aux) : nullptr;
   p.aux_out = static_cast<__half*>(aux_out);
@@ -497,6 +525,10 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
     e = launch_form<true, true>(grid, ta, tb, p, epi, out_f32, stream);
   count_launches(1);
   if (e != cudaSuccess) return cuda_fail(e, "gemm_tc_kernel launch");
+  if (colsum) {
+    e = reduce_rows_f32(p.colpart, colpart_rows, N, colsum, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "column-sum reduce launch");
+  }
   if (p.splits > 1) {
     const int64_t n = static_cast<int64_t>(M) * N;
     const int blocks = static_cast<int>(std::min<int64_t>(ceil_div(n / 4 + 1, 256), sms * 8));

@@ -9,6 +9,8 @@
 // Column sums never use floating-point atomics: each CTA writes per-column
 // partials, and a second pass adds them in a fixed order.
 #include "common.cuh"
+#include "ptx.cuh"
+#include "gemm.h"
 #include "rowwise.h"
 
 namespace sky {
@@ -222,6 +224,157 @@ __global__ void to_f32_kernel(const T* __restrict__ x, int64_t n, float* __restr
     out[i] = to_f32(x[i]);
 }
 
+// LayerNorm backward, streamed through shared memory (bf16 slices, H = 1024
+// or less, H % 256 == 0).  One persistent CTA per SM owns a contiguous block
+// of rows.  A producer thread keeps RING rows of (u, dy, dy2) in flight with
+// 1-D bulk copies into a shared-memory ring; 8 consumer warps take rows
+// round-robin, each lane holding 32 columns (four 8-wide chunks), compute
+//   du = rstd * (g - mean(g) - xhat * mean(g * xhat)),  g = (dy + dy2) * gamma
+// and keep the column sums of dy*xhat, dy and du in registers.  At the end
+// the 8 warps' sums are added in order into part[k][blockIdx.x][:].
+constexpr int SB_WARPS = 8, SB_RING = 16, SB_NV = 4;  // 32 columns per lane: H <= 1024
+constexpr int SB_ROW_BYTES = 3 * 1024 * 4;            // u, dy, dy2 (fp32 capacity)
+
+// part[k][blockIdx.x][:] = sum over the consumer warps (in order) of acc.
+__device__ __forceinline__ void sb_flush(const float (&acc)[SB_NV][8], int k, float* red,
+                                         float* __restrict__ part, int H) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp < SB_WARPS) {
+#pragma unroll
+    for (int c = 0; c < SB_NV; ++c) {
+      const int col = (c * 32 + lane) * 8;
+      if (col < H) store8(red + warp * H + col, acc[c]);
+    }
+  }
+  __syncthreads();
+  for (int col = threadIdx.x; col < H; col += blockDim.x) {
+    float s = 0.f;
+    for (int w = 0; w < SB_WARPS; ++w) s += red[w * H + col];
+    part[(static_cast<int64_t>(k) * gridDim.x + blockIdx.x) * H + col] = s;
+  }
+  __syncthreads();
+}
+
+template <typename TDY>
+__global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
+    const TDY* __restrict__ dy, const float* __restrict__ dy2, const float* __restrict__ u,
+    const __nv_bfloat16* __restrict__ gamma, const float* __restrict__ mean,
+    const float* __restrict__ rstd, int rows, int H, float* __restrict__ du32,
+    __nv_bfloat16* __restrict__ duT, float* __restrict__ part, int32_t* status) {
+  extern __shared__ uint8_t sm_raw[];
+  uint8_t* sm = sm_raw + ((128 - (ptx::smem_u32(sm_raw) & 127)) & 127);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sm + SB_RING * SB_ROW_BYTES);
+  uint64_t* empty = full + SB_RING;
+  float* sgm = reinterpret_cast<float*>(empty + SB_RING);  // gamma as fp32 [H]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int per = (rows + gridDim.x - 1) / gridDim.x;
+  const int r0 = blockIdx.x * per, r1 = min(rows, r0 + per);
+  const int n = r1 > r0 ? r1 - r0 : 0;
+  const uint32_t ubytes = H * 4, dbytes = H * sizeof(TDY);
+  const uint64_t lim = 2000000000ull;
+  for (int c = threadIdx.x; c < H; c += blockDim.x) sgm[c] = __bfloat162float(gamma[c]);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < SB_RING; ++s) {
+      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&empty[s], 32);
+    }
+    ptx::fence_mbar_init();
+    ptx::fence_proxy_async_smem();
+  }
+  __syncthreads();
+  float pg[SB_NV][8] = {}, pb[SB_NV][8] = {}, pu[SB_NV][8] = {};  // column sums (consumers)
+  if (warp == SB_WARPS) {
+    // producer
+    if (lane == 0) {
+      for (int i = 0; i < n; ++i) {
+        const int s = i % SB_RING;
+        if (!ptx::mbar_wait(&empty[s], ((i / SB_RING) & 1) ^ 1u, lim, status, 5000)) break;
+        uint8_t* slot = sm + s * SB_ROW_BYTES;
+        const int64_t row = r0 + i;
+        ptx::mbar_arrive_expect_tx(&full[s], ubytes + dbytes + (dy2 ? ubytes : 0));
+        ptx::bulk_load(slot, u + row * H, ubytes, &full[s]);
+        ptx::bulk_load(slot + 4096, dy + row * H, dbytes, &full[s]);
+        if (dy2) ptx::bulk_load(slot + 8192, dy2 + row * H, ubytes, &full[s]);
+      }
+    }
+    // wait (bounded) for the last copies before the CTA may exit
+    if (lane == 0)
+      for (int i = n - 1; i >= 0 && i >= n - SB_RING; --i)
+        ptx::mbar_wait(&full[i % SB_RING], (i / SB_RING) & 1, lim, status, 5000);
+  } else {
+    const float invH = 1.f / H;
+    for (int i = warp; i < n; i += SB_WARPS) {
+      const int s = i % SB_RING;
+      const int64_t row = r0 + i;
+      const float mu = mean[row], rs = rstd[row];
+      const bool ok = ptx::mbar_wait(&full[s], (i / SB_RING) & 1, lim, status, 5000);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      const uint8_t* slot = sm + s * SB_ROW_BYTES;
+      const float* su = reinterpret_cast<const float*>(slot);
+      const TDY* sdy = reinterpret_cast<const TDY*>(slot + 4096);
+      const float* sd2 = reinterpret_cast<const float*>(slot + 8192);
+      // x-hat and dy (+ dy2) of 8 columns, read from the slot
+      auto fetch = [&](int col, float (&xh)[8], float (&d)[8]) {
+        load8(su + col, xh);
+        load8(sdy + col, d);
+        if (dy2) {
+          float e[8];
+          load8(sd2 + col, e);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) d[k] += e[k];
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) xh[k] = (xh[k] - mu) * rs;
+      };
+      float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+      for (int c = 0; c < SB_NV; ++c) {
+        const int col = (c * 32 + lane) * 8;
+        if (col < H) {
+          float xh[8], d[8], gm[8];
+          fetch(col, xh, d);
+          load8(sgm + col, gm);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const float g = d[k] * gm[k];
+            s1 += g;
+            s2 += g * xh[k];
+          }
+        }
+      }
+      const float mg = warp_sum(s1) * invH, mgx = warp_sum(s2) * invH;
+      // second pass re-reads the slot instead of holding the row in registers
+#pragma unroll
+      for (int c = 0; c < SB_NV; ++c) {
+        const int col = (c * 32 + lane) * 8;
+        if (col < H) {
+          float xh[8], d[8], gm[8], o[8];
+          fetch(col, xh, d);
+          load8(sgm + col, gm);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            o[k] = rs * (d[k] * gm[k] - mg - xh[k] * mgx);
+            pg[c][k] += d[k] * xh[k];
+            pb[c][k] += d[k];
+            pu[c][k] += o[k];
+          }
+          if (du32) store8(du32 + row * H + col, o);
+          if (duT) store8(duT + row * H + col, o);
+        }
+      }
+      __syncwarp();
+      ptx::mbar_arrive(&empty[s]);  // slot s may be refilled
+    }
+  }
+  // every row's copy has landed and been consumed: the ring is free for the
+  // CTA's fixed-order reduction of the 8 warps' column sums
+  __syncthreads();
+  float* red = reinterpret_cast<float*>(sm);  // [SB_WARPS][H]
+  sb_flush(pg, 0, red, part, H);
+  sb_flush(pb, 1, red, part, H);
+  sb_flush(pu, 2, red, part, H);
+}
+
 // out_k[n] = sum_b part[k][b][n] for the non-null outputs, in a fixed order:
 // CTA (cx, k) owns 32 columns; its 8 warps each add every 8th partial row
 // (coalesced 128-byte reads), then the 8 warp sums are added in order.
@@ -315,6 +468,7 @@ int ln_blocks(int rows) {
   const int cap = 4 * (sm_count() > 0 ? sm_count() : 148);
   return want < cap ? want : cap;
 }
+int stream_blocks() { return sm_count() > 0 ? sm_count() : 148; }
 // Backward CTAs also write column partials, so fewer, longer-lived CTAs.
 int ln_bwd_blocks(int rows) {
   const int want = ceil_div(rows, LN_WARPS);
@@ -404,6 +558,34 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
             "LayerNorm backward workspace too small");
   float* part = static_cast<float*>(ws);
   const int nv = lane_vectors(H);
+  if (dt == SKY_DTYPE_BF16 && H <= 1024 && H % 256 == 0 && rw::stream_blocks() <= nblk) {
+    // streamed variant: one CTA per SM, rows staged through shared memory
+    const int sb = rw::stream_blocks();
+    const size_t smem = (size_t)rw::SB_RING * rw::SB_ROW_BYTES + 2 * rw::SB_RING * 8 + (size_t)H * 4 + 128;
+    // the attribute is set once, for the largest H this variant takes
+    const size_t smem_max = (size_t)rw::SB_RING * rw::SB_ROW_BYTES + 2 * rw::SB_RING * 8 + 1024 * 4 + 128;
+    const int threads = 32 * (rw::SB_WARPS + 1);
+    if (dy_dt == SKY_DTYPE_BF16) {
+      static cudaError_t a = cudaFuncSetAttribute(rw::ln_bwd_stream_kernel<__nv_bfloat16>,
+                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
+      if (a != cudaSuccess) return cuda_fail(a, "LayerNorm backward smem attribute");
+      rw::ln_bwd_stream_kernel<__nv_bfloat16><<<sb, threads, smem, st>>>(
+          static_cast<const __nv_bfloat16*>(dy), dy2, u, static_cast<const __nv_bfloat16*>(gamma),
+          mean, rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, nullptr);
+    } else {
+      static cudaError_t a = cudaFuncSetAttribute(rw::ln_bwd_stream_kernel<float>,
+                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
+      if (a != cudaSuccess) return cuda_fail(a, "LayerNorm backward smem attribute");
+      rw::ln_bwd_stream_kernel<float><<<sb, threads, smem, st>>>(
+          static_cast<const float*>(dy), dy2, u, static_cast<const __nv_bfloat16*>(gamma), mean,
+          rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, nullptr);
+    }
+    dim3 grid(ceil_div(H, 32), 3);
+    rw::reduce_partials<<<grid, 256, 0, st>>>(part, sb, H, dgamma, dbeta, dbias);
+    count_launches(2);
+    const cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward launch");
+  }
   if (dt == SKY_DTYPE_BF16) {
     if (dy_dt == SKY_DTYPE_BF16) {
 #define LNB(NV) rw::ln_bwd_launch<__nv_bfloat16, __nv_bfloat16, NV>(dy, dy2, u, gamma, mean, rstd, rows, H, du32, du, part, nblk, st)
@@ -428,6 +610,15 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward launch");
 }
+
+namespace gemm {
+cudaError_t reduce_rows_f32(const float* part, int rows, int N, float* out, cudaStream_t stream) {
+  rw::reduce_partials<<<dim3(ceil_div(N, 32), 1), 256, 0, stream>>>(part, rows, N, out, nullptr,
+                                                                  nullptr);
+  count_launches(1);
+  return cudaGetLastError();
+}
+}  // namespace gemm
 
 sky_status add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dt, void* out,
                    cudaStream_t st) {

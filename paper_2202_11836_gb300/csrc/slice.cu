@@ -146,6 +146,7 @@ size_t workspace_need(const sky_slice* s, int64_t T) {
       need = std::max(need, gemm::workspace_bytes(SKY_GEMM_XTW, (int)sh[0], (int)sh[1], (int)T, true));
   }
   need = std::max(need, layernorm_bwd_ws((int)T, H));
+  need = std::max(need, (size_t)ceil_div(T, 128) * 4 * F * sizeof(float));  // fused db1 partials
   need = std::max(need, column_sum_ws((int)T, F));
   need = std::max(need, column_sum_ws((int)T, 3 * H));
   return need;
@@ -181,11 +182,11 @@ struct Timed {
 
 sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, int M, int N,
                     int K, const void* A, const void* Bm, void* C, bool out_f32, int epi,
-                    const void* bias, const void* aux, void* aux_out) {
+                    const void* bias, const void* aux, void* aux_out, float* colsum = nullptr) {
   Timed t(s, st, cat, 2.0 * M * N * K, 0);
   if (s->cfg.dtype == SKY_DTYPE_BF16)
     return gemm::launch_bf16(form, M, N, K, A, Bm, C, out_f32, epi, bias, aux, aux_out, s->ws,
-                             s->ws_bytes, s->d_status, st);
+                             s->ws_bytes, s->d_status, st, colsum);
   return gemm::launch_f32(form, M, N, K, static_cast<const float*>(A),
                           static_cast<const float*>(Bm), static_cast<float*>(C), epi,
                           static_cast<const float*>(bias), static_cast<const float*>(aux),
@@ -270,14 +271,15 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
                           s->ws_bytes, st));
   }
   // a10 + a11: dZ = (dU2 W2) * GELU'(Z);  dW2 = dU2^T G
+  //          db1 = sum_rows dZ (fused into the bf16 epilogue; a column-sum pass for fp32)
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
-                   SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr));
-  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
-  {
+                   SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr, bf ? Lb.g[7] : nullptr));
+  if (!bf) {
     Timed t(s, st, P_COLSUM, 0, e * T * F);
     SKY_TRY(column_sum(s->dH, T, F, dt, Lb.g[7], s->ws, s->ws_bytes, st));
   }
+  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
   // a12: P1 = dZ W1 (fp32; dX1 = P1 + dU2 is formed by the LN1 backward);  dW1 = dZ^T X1
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dP1, true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
