@@ -1,8 +1,8 @@
-// Masked scaled dot-product attention (Eq. 1) forward on the 5th-generation
-// tensor cores, bf16, head dim D = 64.
+// Masked scaled dot-product attention (Eq. 1) forward and backward on the
+// 5th-generation tensor cores, bf16, head dim D = 64.
 //
-// One CTA owns 128 query rows of one (sequence b, head a).  Per 64-key tile j
-// (only tiles below len[b] are visited):
+// Forward: one CTA owns 128 query rows of one (sequence b, head a).  Per
+// 64-key tile j (only tiles below len[b] are visited):
 //   S_j = Q K_j^T                  tcgen05.mma M=128 N=64 K=64 -> TMEM
 //   softmax (4 warps, thread = query row = TMEM lane): row max over the
 //     valid keys, P_j = exp2(S_j log2(e)/sqrt(D) - m) written as bf16 to
@@ -10,13 +10,18 @@
 //   O += P_j V_j                   tcgen05.mma M=128 N=64 K=64 -> TMEM
 // Q, K and V come straight out of the packed QKV activations by TMA (one
 // tensor map, per-head column offsets).  Because a thread owns a whole query
-// row, the row max and row sum need no shuffles.  When a row's running max
-// rises, that row of O is rescaled in TMEM (tcgen05.ld / st) before the next
-// P V product is issued; the final O is divided by the row sum and the
-// log-sum-exp is kept for the backward pass.  Everything in one CTA is
-// sequential; three CTAs per SM (64 KB shared memory, 128 TMEM columns each)
-// overlap one CTA's softmax with another's MMAs.  All mbarrier waits are
-// time-bounded.
+// row, the row max and row sum need no shuffles.
+//
+// The steps are pipelined inside the CTA: S has two TMEM buffers and P two
+// shared-memory buffers, so the MMA warp computes S_{j+1} (issued one tile
+// ahead) and P_{j-1} V_{j-1} while the softmax warps work on tile j, and K/V
+// tiles stream through a 3-stage TMA ring.  The exponent offset m of a row
+// is only raised when the tile's max exceeds it by more than 2^8 (a factor
+// 256 in P): then O and the row sum are rescaled in TMEM once the pending
+// P V product has landed.  Otherwise P may exceed 1 by at most that factor,
+// which bf16 and the fp32 sums carry with the same relative precision; the
+// final O / l and the log-sum-exp do not depend on m.  All mbarrier waits
+// are time-bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -32,21 +37,28 @@ constexpr int BQ = 128, BKV = 64, HD = 64;
 constexpr int Q_BYTES = BQ * HD * 2;    // 16 KiB
 constexpr int KV_BYTES = BKV * HD * 2;  // 8 KiB per K or V tile
 constexpr int P_BYTES = BQ * BKV * 2;   // 16 KiB
-constexpr int STAGES = 2;
-constexpr int Q_OFF = 0;
-constexpr int K_OFF = Q_OFF + Q_BYTES;
-constexpr int V_OFF = K_OFF + STAGES * KV_BYTES;
-constexpr int P_OFF = V_OFF + STAGES * KV_BYTES;
-constexpr int BAR_OFF = P_OFF + P_BYTES;
-constexpr int SMEM_BYTES = BAR_OFF + 128 + 1024;
-constexpr int TMEM_COLS = 128;  // S: columns [0, 64), O: [64, 128)
-constexpr int NTHR = 192;       // warp 0 TMA, warp 1 MMA, warps 2..5 softmax
+constexpr int STAGES = 2;               // backward operand rings
+constexpr int NTHR = 192;               // warp 0 TMA, warp 1 MMA, warps 2..5 softmax
+// The backward kernels run eight softmax warps: warps w and w + 4 share TMEM
+// lane quarter w % 4 and take the low / high 32 columns of each 64-wide tile.
+constexpr int NTHR_B = 320;             // warp 0 TMA, warp 1 MMA, warps 2..9 softmax
+constexpr int NSM_B = 256;              // softmax threads in the backward kernels
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr float LN2 = 0.6931471805599453f;
 // Suspend-time hint (ns) of every mbarrier wait: a waiting thread sleeps
 // until the phase completes instead of spinning on issue slots that the
 // softmax warps (the critical path) share with the producer and MMA threads.
 constexpr uint32_t kWaitHint = 10000;
+
+// forward shared-memory layout (offsets from a 1024-byte aligned base)
+constexpr int F_STAGES = 3;
+constexpr int F_Q_OFF = 0;
+constexpr int F_KV_OFF = F_Q_OFF + Q_BYTES;                  // [F_STAGES] x {K, V}
+constexpr int F_P_OFF = F_KV_OFF + F_STAGES * 2 * KV_BYTES;  // [2] P tiles
+constexpr int F_BAR_OFF = F_P_OFF + 2 * P_BYTES;
+constexpr int F_SMEM = F_BAR_OFF + 256 + 1024;
+constexpr int F_TMEM_COLS = 256;  // S_0: [0, 64), S_1: [64, 128), O: [128, 192)
+constexpr float kRescaleLog2 = 8.f;
 
 struct FwdParams {
   int S, H, A;
@@ -63,13 +75,13 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
-  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + BAR_OFF);
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + F_BAR_OFF);
   uint64_t* kv_full = q_full + 1;
-  uint64_t* kv_empty = kv_full + STAGES;
-  uint64_t* s_full = kv_empty + STAGES;
-  uint64_t* p_full = s_full + 1;
-  uint64_t* pv_done = p_full + 1;
-  uint64_t* done = pv_done + 1;
+  uint64_t* kv_empty = kv_full + F_STAGES;
+  uint64_t* s_full = kv_empty + F_STAGES;  // [2]
+  uint64_t* p_full = s_full + 2;           // [2]
+  uint64_t* pv_done = p_full + 2;          // [2]
+  uint64_t* done = pv_done + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
 
   const int qt = blockIdx.x, a = blockIdx.y, b = blockIdx.z;
@@ -87,78 +99,108 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
 
   if (threadIdx.x == 0) {
     ptx::mbar_init(q_full, 1);
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < F_STAGES; ++s) {
       ptx::mbar_init(&kv_full[s], 1);
       ptx::mbar_init(&kv_empty[s], 1);
     }
-    ptx::mbar_init(s_full, 1);
-    ptx::mbar_init(p_full, 128);
-    ptx::mbar_init(pv_done, 1);
+    for (int s = 0; s < 2; ++s) {
+      ptx::mbar_init(&s_full[s], 1);
+      ptx::mbar_init(&p_full[s], 128);
+      ptx::mbar_init(&pv_done[s], 1);
+    }
     ptx::mbar_init(done, 1);
     ptx::fence_mbar_init();
     ptx::fence_proxy_async_smem();
   }
   if (warp == 1) {
-    ptx::tmem_alloc(tmem_slot, TMEM_COLS);
+    ptx::tmem_alloc(tmem_slot, F_TMEM_COLS);
     ptx::tmem_relinquish();
   }
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS = tmem, tO = tmem + 64;
+  const uint32_t tS = tmem, tO = tmem + 128;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       ptx::mbar_arrive_expect_tx(q_full, Q_BYTES);
-      ptx::tma_load_2d(smem + Q_OFF, &tmQ, q_full, a * HD, row0 + q0);
-      bool ok = true;
+      ptx::tma_load_2d(smem + F_Q_OFF, &tmQ, q_full, a * HD, row0 + q0);
       int issued = 0;
-      for (int j = 0; j < n_kt && ok; ++j) {
-        const int st = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        if (!ptx::mbar_wait(&kv_empty[st], ph ^ 1u, lim, p.status, kWaitHint)) { ok = false; break; }
+      for (int j = 0; j < n_kt; ++j) {
+        const int st = j % F_STAGES;
+        const uint32_t ph = (j / F_STAGES) & 1;
+        if (!ptx::mbar_wait(&kv_empty[st], ph ^ 1u, lim, p.status, kWaitHint)) break;
+        uint8_t* kv = smem + F_KV_OFF + st * 2 * KV_BYTES;
         ptx::mbar_arrive_expect_tx(&kv_full[st], 2 * KV_BYTES);
-        ptx::tma_load_2d(smem + K_OFF + st * KV_BYTES, &tmKV, &kv_full[st], H + a * HD,
-                         row0 + j * BKV);
-        ptx::tma_load_2d(smem + V_OFF + st * KV_BYTES, &tmKV, &kv_full[st], 2 * H + a * HD,
-                         row0 + j * BKV);
+        ptx::tma_load_2d(kv, &tmKV, &kv_full[st], H + a * HD, row0 + j * BKV);
+        ptx::tma_load_2d(kv + KV_BYTES, &tmKV, &kv_full[st], 2 * H + a * HD, row0 + j * BKV);
         ++issued;
       }
       // drain: bounded waits for the copies still in flight
       ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint);
-      for (int j = issued - 1; j >= 0 && j >= issued - STAGES; --j)
-        ptx::mbar_wait(&kv_full[j & 1], (j >> 1) & 1, lim, p.status, kWaitHint);
+      for (int j = issued - 1; j >= 0 && j >= issued - F_STAGES; --j)
+        ptx::mbar_wait(&kv_full[j % F_STAGES], (j / F_STAGES) & 1, lim, p.status, kWaitHint);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------- MMA issue
     if (lane == 0) {
       constexpr uint32_t idS = ptx::idesc_bf16_f32(BQ, BKV, false, false);
       constexpr uint32_t idO = ptx::idesc_bf16_f32(BQ, HD, false, true);
-      const uint32_t sq = ptx::smem_u32(smem + Q_OFF), sp = ptx::smem_u32(smem + P_OFF);
-      bool ok = ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint);
-      for (int j = 0; j < n_kt && ok; ++j) {
-        const int st = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        if (!ptx::mbar_wait(&kv_full[st], ph, lim, p.status, kWaitHint)) break;
-        ptx::tc_fence_after();
-        const uint32_t sk = ptx::smem_u32(smem + K_OFF + st * KV_BYTES);
-        const uint32_t sv = ptx::smem_u32(smem + V_OFF + st * KV_BYTES);
+      const uint32_t sq = ptx::smem_u32(smem + F_Q_OFF);
+      const uint32_t skv = ptx::smem_u32(smem + F_KV_OFF);
+      const uint32_t sp = ptx::smem_u32(smem + F_P_OFF);
+      // S_j = Q K_j^T into S buffer j & 1 (K_j already landed)
+      auto mma_s = [&](int j) {
+        const uint32_t sk = skv + (j % F_STAGES) * 2 * KV_BYTES;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
-          ptx::tc_mma_f16(tS, ptx::smem_desc_sw128(sq + kk * 32, 16, 1024),
+          ptx::tc_mma_f16(tS + (j & 1) * BKV, ptx::smem_desc_sw128(sq + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(sk + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
-        ptx::tc_commit(s_full);
-        if (!ptx::mbar_wait(p_full, j & 1, lim, p.status, kWaitHint)) break;
+        ptx::tc_commit(&s_full[j & 1]);
+      };
+      auto wait_k = [&](int j) {
+        return ptx::mbar_wait(&kv_full[j % F_STAGES], (j / F_STAGES) & 1, lim, p.status, kWaitHint);
+      };
+      bool ok = ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint) && wait_k(0);
+      if (ok) {
         ptx::tc_fence_after();
+        mma_s(0);
+      }
+      // S_{s_next} is due next; it goes in while the MMA thread waits for P,
+      // as soon as its K tile has landed
+      int s_next = 1;
+      bool s_done = n_kt <= 1;
+      for (int j = 0; j < n_kt && ok; ++j) {
+        auto s_ready = [&] {
+          return ptx::mbar_try_wait(&kv_full[s_next % F_STAGES], (s_next / F_STAGES) & 1);
+        };
+        auto s_issue = [&] {
+          ptx::tc_fence_after();
+          mma_s(s_next);
+        };
+        if (!ptx::mbar_wait_with(&p_full[j & 1], (j >> 1) & 1, lim, p.status, kWaitHint, s_done, s_ready,
+                                 s_issue))
+          break;
+        ptx::tc_fence_after();
+        const uint32_t sv = skv + (j % F_STAGES) * 2 * KV_BYTES + KV_BYTES;
+        const uint32_t spj = sp + (j & 1) * P_BYTES;
 #pragma unroll
         for (int kk = 0; kk < BKV / 16; ++kk)
-          ptx::tc_mma_f16(tO, ptx::smem_desc_sw128(sp + kk * 32, 16, 1024),
+          ptx::tc_mma_f16(tO, ptx::smem_desc_sw128(spj + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(sv + kk * 2048, 8192, 1024), idO,
                           (j > 0 || kk > 0) ? 1u : 0u);
-        ptx::tc_commit(pv_done);
-        ptx::tc_commit(&kv_empty[st]);
+        ptx::tc_commit(&pv_done[j & 1]);
+        ptx::tc_commit(&kv_empty[j % F_STAGES]);
+        if (!s_done) {  // S_{j+1} is needed before P_{j+1} can exist
+          if (!wait_k(s_next)) break;
+          s_issue();
+        }
+        // the softmax warps have read S_j (they arrived on p_full[j & 1]
+        // after their TMEM loads), so its buffer takes S_{j+2}
+        s_next = j + 2;
+        s_done = s_next >= n_kt;
       }
       ptx::tc_commit(done);
       ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
@@ -169,7 +211,6 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
     const int r = q4 * 32 + lane;  // query row within the tile == TMEM lane
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
     const float sl2 = LOG2E * 0.125f;  // log2(e) / sqrt(64)
-    uint8_t* prow = smem + P_OFF + r * 128;
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     // every lane waits (bounded); the outcome is made warp-uniform so the
@@ -179,85 +220,74 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
       return __all_sync(0xffffffffu, mine);
     };
     for (int j = 0; j < n_kt; ++j) {
-      if (!wait_all(s_full, j & 1)) { ok = false; break; }
+      if (!wait_all(&s_full[j & 1], (j >> 1) & 1)) { ok = false; break; }
       ptx::tc_fence_after();
+      uint32_t v[BKV];
+      {
+        uint32_t (&v0)[32] = *reinterpret_cast<uint32_t(*)[32]>(&v[0]);
+        uint32_t (&v1)[32] = *reinterpret_cast<uint32_t(*)[32]>(&v[32]);
+        ptx::tmem_ld_32x32b_x32(tS + (j & 1) * BKV + lane_base, v0);
+        ptx::tmem_ld_32x32b_x32(tS + (j & 1) * BKV + lane_base + 32, v1);
+      }
+      ptx::tmem_ld_wait();
       const int kbase = j * BKV;
-      const bool full_tile = kbase + BKV <= len;  // CTA-uniform: only the last tile is masked
-      // pass 1: row max of the raw scores (scaling by log2(e)/sqrt(D) > 0 commutes with max)
-      float mx = -INFINITY;
+      if (kbase + BKV > len) {  // CTA-uniform: only the last tile holds masked keys
 #pragma unroll
-      for (int c = 0; c < BKV / 32; ++c) {
-        uint32_t v[32];
-        ptx::tmem_ld_32x32b_x32(tS + lane_base + c * 32, v);
-        ptx::tmem_ld_wait();
-        if (full_tile) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) mx = fmaxf(mx, __uint_as_float(v[i]));
-        } else {
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (kbase + c * 32 + i < len) mx = fmaxf(mx, __uint_as_float(v[i]));
-        }
+        for (int i = 0; i < BKV; ++i)
+          if (kbase + i >= len) v[i] = 0xff800000u;  // -inf: excluded from the max, P = 0
       }
-      mx *= sl2;
-      const float m_new = fmaxf(m, mx);
-      if (j > 0) {
-        // P_{j-1} V_{j-1} must be done: the P buffer is reused and O may be rescaled
-        if (!wait_all(pv_done, (j - 1) & 1)) { ok = false; break; }
+      // row max of the raw scores (scaling by log2(e)/sqrt(D) > 0 commutes with max)
+      float mx8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mx8[i] = __uint_as_float(v[i]);
+#pragma unroll
+      for (int i = 8; i < BKV; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(v[i]));
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7]))) * sl2;
+      if (j == 0) {
+        m = mx;
+      } else if (__any_sync(0xffffffffu, mx > m + kRescaleLog2)) {
+        // O must hold P_{j-1} V_{j-1} before it is rescaled
+        if (!wait_all(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1)) { ok = false; break; }
         ptx::tc_fence_after();
-        const bool need = m_new > m;
-        if (__any_sync(0xffffffffu, need)) {
-          const float alpha = need ? exp2f(m - m_new) : 1.f;
+        const float m_new = fmaxf(m, mx);
+        const float alpha = exp2f(m - m_new);
 #pragma unroll
-          for (int c = 0; c < HD / 32; ++c) {
-            uint32_t o[32];
-            ptx::tmem_ld_32x32b_x32(tO + lane_base + c * 32, o);
-            ptx::tmem_ld_wait();
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t o[32];
+          ptx::tmem_ld_32x32b_x32(tO + lane_base + c * 32, o);
+          ptx::tmem_ld_wait();
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-            ptx::tmem_st_32x32b_x32(tO + lane_base + c * 32, o);
-          }
-          ptx::tmem_st_wait();
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+          ptx::tmem_st_32x32b_x32(tO + lane_base + c * 32, o);
         }
-        l *= exp2f(m - m_new);
+        ptx::tmem_st_wait();
+        l *= alpha;
+        m = m_new;
       }
-      m = m_new;
-      // pass 2: P = exp2(s * sl2 - m) as bf16, row r of the swizzled K-major tile
+      // P buffer j & 1 was last read by P_{j-2} V_{j-2}
+      if (j >= 2 && !wait_all(&pv_done[j & 1], ((j - 2) >> 1) & 1)) { ok = false; break; }
+      // P = exp2(s * sl2 - m) as bf16, row r of the swizzled K-major tile
+      uint8_t* prow = smem + F_P_OFF + (j & 1) * P_BYTES + r * 128;
       const float nm = -m;
+      float ls = 0.f;
 #pragma unroll
-      for (int c = 0; c < BKV / 32; ++c) {
-        uint32_t v[32];
-        ptx::tmem_ld_32x32b_x32(tS + lane_base + c * 32, v);
-        ptx::tmem_ld_wait();
-        float pv[32];
+      for (int u = 0; u < BKV / 8; ++u) {  // 16-byte unit u holds keys 8u .. 8u+7
+        float e[8];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) pv[i] = ptx::ex2_ftz(fmaf(__uint_as_float(v[i]), sl2, nm));
-        if (!full_tile) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (kbase + c * 32 + i >= len) pv[i] = 0.f;
-        }
-        uint32_t pk[16];
-        float ls = 0.f;
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          ls += pv[i] + pv[i + 1];
-          pk[i >> 1] = ptx::pack_bf16(pv[i], pv[i + 1]);
-        }
-        l += ls;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int unit = c * 4 + u;  // 16-byte unit (8 keys) within the 128-byte row
-          *reinterpret_cast<uint4*>(prow + ((unit ^ (r & 7)) << 4)) =
-              make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-        }
+        for (int t = 0; t < 8; ++t) e[t] = ptx::ex2_ftz(fmaf(__uint_as_float(v[8 * u + t]), sl2, nm));
+        ls += ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
+        *reinterpret_cast<uint4*>(prow + ((u ^ (r & 7)) << 4)) =
+            make_uint4(ptx::pack_bf16(e[0], e[1]), ptx::pack_bf16(e[2], e[3]),
+                       ptx::pack_bf16(e[4], e[5]), ptx::pack_bf16(e[6], e[7]));
       }
+      l += ls;
       ptx::fence_proxy_async_smem();
       ptx::tc_fence_before();
-      ptx::mbar_arrive(p_full);
+      ptx::mbar_arrive(&p_full[j & 1]);
     }
     // epilogue: O / l -> ctx (bf16), log-sum-exp
-    if (ok && wait_all(pv_done, (n_kt - 1) & 1)) {
+    if (ok && wait_all(&pv_done[(n_kt - 1) & 1], ((n_kt - 1) >> 1) & 1)) {
       ptx::tc_fence_after();
       const float inv = 1.f / l;
       const int q = q0 + r;
@@ -286,7 +316,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
   __syncthreads();
   if (warp == 1) {
     ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem, TMEM_COLS);
+    ptx::tmem_dealloc(tmem, F_TMEM_COLS);
   }
 }
 
@@ -295,16 +325,20 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
 //   S = Q K_j^T, dP = dO V_j^T (TMEM); thread = query row:
 //   P = exp2(S log2(e)/sqrt(D) - lse2), dS = P (dP - delta) -> smem (bf16)
 //   dQ += dS K_j (TMEM); finally dQ / sqrt(D) -> dQKV[:, Q block].
+// Pipelining: the softmax warps release S / dP as soon as they hold them in
+// registers (s_free), so S_{j+1} and dP_{j+1} run on the tensor cores while
+// dS_j is formed; K / V tiles stream through a 3-stage TMA ring.
+constexpr int DQ_STAGES = 3;
 constexpr int DQ_QD_BYTES = 2 * Q_BYTES;  // Q and dO tiles (128 x 64 each)
 constexpr int DQ_Q_OFF = 0, DQ_DO_OFF = Q_BYTES;
-constexpr int DQ_K_OFF = DQ_QD_BYTES;
-constexpr int DQ_V_OFF = DQ_K_OFF + STAGES * KV_BYTES;
-constexpr int DQ_DS_OFF = DQ_V_OFF + STAGES * KV_BYTES;
+constexpr int DQ_KV_OFF = DQ_QD_BYTES;                           // [DQ_STAGES] x {K, V}
+constexpr int DQ_DS_OFF = DQ_KV_OFF + DQ_STAGES * 2 * KV_BYTES;  // dS tile
 constexpr int DQ_BAR_OFF = DQ_DS_OFF + P_BYTES;
-constexpr int DQ_SMEM = DQ_BAR_OFF + 128 + 1024;
+constexpr int DQ_SMEM = DQ_BAR_OFF + 256 + 1024;
 
 struct BwdParams {
   int S, H, A;
+  int lse_bulk;  // lse / delta rows may be bulk-copied: S % 4 == 0, 16-byte aligned bases
   const int32_t* lens;
   const float* lse;
   const float* delta;
@@ -313,7 +347,7 @@ struct BwdParams {
   uint64_t timeout_ns;
 };
 
-__global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant__ CUtensorMap tmQ,
+__global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorMap tmQ,
                                                           const __grid_constant__ CUtensorMap tmKV,
                                                           const __grid_constant__ CUtensorMap tmO,
                                                           const BwdParams p) {
@@ -322,9 +356,10 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
   uint64_t* qd_full = reinterpret_cast<uint64_t*>(smem + DQ_BAR_OFF);
   uint64_t* kv_full = qd_full + 1;
-  uint64_t* kv_empty = kv_full + STAGES;
-  uint64_t* s_full = kv_empty + STAGES;
-  uint64_t* ds_full = s_full + 1;
+  uint64_t* kv_empty = kv_full + DQ_STAGES;
+  uint64_t* s_full = kv_empty + DQ_STAGES;
+  uint64_t* s_free = s_full + 1;
+  uint64_t* ds_full = s_free + 1;
   uint64_t* dq_done = ds_full + 1;
   uint64_t* done = dq_done + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
@@ -343,12 +378,13 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
 
   if (threadIdx.x == 0) {
     ptx::mbar_init(qd_full, 1);
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < DQ_STAGES; ++s) {
       ptx::mbar_init(&kv_full[s], 1);
       ptx::mbar_init(&kv_empty[s], 1);
     }
     ptx::mbar_init(s_full, 1);
-    ptx::mbar_init(ds_full, 128);
+    ptx::mbar_init(s_free, NSM_B);
+    ptx::mbar_init(ds_full, NSM_B);
     ptx::mbar_init(dq_done, 1);
     ptx::mbar_init(done, 1);
     ptx::fence_mbar_init();
@@ -366,37 +402,37 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
 
   if (warp == 0) {
     if (lane == 0) {
+      ptx::prefetch_tensormap(&tmQ);
+      ptx::prefetch_tensormap(&tmO);
+      ptx::prefetch_tensormap(&tmKV);
       ptx::mbar_arrive_expect_tx(qd_full, DQ_QD_BYTES);
       ptx::tma_load_2d(smem + DQ_Q_OFF, &tmQ, qd_full, a * HD, row0 + q0);
       ptx::tma_load_2d(smem + DQ_DO_OFF, &tmO, qd_full, a * HD, row0 + q0);
       int issued = 0;
       for (int j = 0; j < n_kt; ++j) {
-        const int st = j & 1;
-        if (!ptx::mbar_wait(&kv_empty[st], ((j >> 1) & 1) ^ 1u, lim, p.status, kWaitHint)) break;
+        const int st = j % DQ_STAGES;
+        if (!ptx::mbar_wait(&kv_empty[st], ((j / DQ_STAGES) & 1) ^ 1u, lim, p.status, kWaitHint))
+          break;
+        uint8_t* kv = smem + DQ_KV_OFF + st * 2 * KV_BYTES;
         ptx::mbar_arrive_expect_tx(&kv_full[st], 2 * KV_BYTES);
-        ptx::tma_load_2d(smem + DQ_K_OFF + st * KV_BYTES, &tmKV, &kv_full[st], H + a * HD,
-                         row0 + j * BKV);
-        ptx::tma_load_2d(smem + DQ_V_OFF + st * KV_BYTES, &tmKV, &kv_full[st], 2 * H + a * HD,
-                         row0 + j * BKV);
+        ptx::tma_load_2d(kv, &tmKV, &kv_full[st], H + a * HD, row0 + j * BKV);
+        ptx::tma_load_2d(kv + KV_BYTES, &tmKV, &kv_full[st], 2 * H + a * HD, row0 + j * BKV);
         ++issued;
       }
       ptx::mbar_wait(qd_full, 0, lim, p.status, kWaitHint);
-      for (int j = issued - 1; j >= 0 && j >= issued - STAGES; --j)
-        ptx::mbar_wait(&kv_full[j & 1], (j >> 1) & 1, lim, p.status, kWaitHint);
+      for (int j = issued - 1; j >= 0 && j >= issued - DQ_STAGES; --j)
+        ptx::mbar_wait(&kv_full[j % DQ_STAGES], (j / DQ_STAGES) & 1, lim, p.status, kWaitHint);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idS = ptx::idesc_bf16_f32(BQ, BKV, false, false);
       constexpr uint32_t idQ = ptx::idesc_bf16_f32(BQ, HD, false, true);
       const uint32_t sq = ptx::smem_u32(smem + DQ_Q_OFF), so = ptx::smem_u32(smem + DQ_DO_OFF);
+      const uint32_t skv = ptx::smem_u32(smem + DQ_KV_OFF);
       const uint32_t sds = ptx::smem_u32(smem + DQ_DS_OFF);
-      bool ok = ptx::mbar_wait(qd_full, 0, lim, p.status, kWaitHint);
-      for (int j = 0; j < n_kt && ok; ++j) {
-        const int st = j & 1;
-        if (!ptx::mbar_wait(&kv_full[st], (j >> 1) & 1, lim, p.status, kWaitHint)) break;
-        ptx::tc_fence_after();
-        const uint32_t sk = ptx::smem_u32(smem + DQ_K_OFF + st * KV_BYTES);
-        const uint32_t sv = ptx::smem_u32(smem + DQ_V_OFF + st * KV_BYTES);
+      // S_j = Q K_j^T and dP_j = dO V_j^T (operands already landed)
+      auto mma_sdp = [&](int j) {
+        const uint32_t sk = skv + (j % DQ_STAGES) * 2 * KV_BYTES, sv = sk + KV_BYTES;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
           ptx::tc_mma_f16(tS, ptx::smem_desc_sw128(sq + kk * 32, 16, 1024),
@@ -406,21 +442,55 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
           ptx::tc_mma_f16(tdP, ptx::smem_desc_sw128(so + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(sv + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
         ptx::tc_commit(s_full);
-        if (!ptx::mbar_wait(ds_full, j & 1, lim, p.status, kWaitHint)) break;
+      };
+      bool ok = ptx::mbar_wait(qd_full, 0, lim, p.status, kWaitHint) &&
+                ptx::mbar_wait(&kv_full[0], 0, lim, p.status, kWaitHint);
+      if (ok) {
         ptx::tc_fence_after();
+        mma_sdp(0);
+      }
+      for (int j = 0; j < n_kt && ok; ++j) {
+        // While dS_j is being formed, issue S_{j+1} / dP_{j+1} as soon as the
+        // softmax warps hold S_j / dP_j in registers (s_free) and K_{j+1} /
+        // V_{j+1} have landed; the dQ product of tile j is never held up by
+        // that tile's loads.
+        const int jn = j + 1;
+        bool next_done = jn >= n_kt;
+        auto next_ready = [&] {
+          return ptx::mbar_try_wait(s_free, j & 1) &&
+                 ptx::mbar_try_wait(&kv_full[jn % DQ_STAGES], (jn / DQ_STAGES) & 1);
+        };
+        auto next_issue = [&] {
+          ptx::tc_fence_after();
+          mma_sdp(jn);
+        };
+        if (!ptx::mbar_wait_with(ds_full, j & 1, lim, p.status, kWaitHint, next_done, next_ready,
+                                 next_issue))
+          break;
+        ptx::tc_fence_after();
+        const uint32_t sk = skv + (j % DQ_STAGES) * 2 * KV_BYTES;
+        const uint32_t sdj = sds;
 #pragma unroll
         for (int kk = 0; kk < BKV / 16; ++kk)
-          ptx::tc_mma_f16(tdQ, ptx::smem_desc_sw128(sds + kk * 32, 16, 1024),
+          ptx::tc_mma_f16(tdQ, ptx::smem_desc_sw128(sdj + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(sk + kk * 2048, 8192, 1024), idQ,
                           (j > 0 || kk > 0) ? 1u : 0u);
         ptx::tc_commit(dq_done);
-        ptx::tc_commit(&kv_empty[st]);
+        ptx::tc_commit(&kv_empty[j % DQ_STAGES]);
+        if (!next_done) {
+          if (!ptx::mbar_wait(s_free, j & 1, lim, p.status, kWaitHint) ||
+              !ptx::mbar_wait(&kv_full[jn % DQ_STAGES], (jn / DQ_STAGES) & 1, lim, p.status,
+                              kWaitHint))
+            break;
+          next_issue();
+        }
       }
       ptx::tc_commit(done);
       ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
     }
   } else {
     const int q4 = warp & 3;
+    const int hf = (warp - 2) >> 2;  // column half: keys [32 hf, 32 hf + 32) of a tile
     const int r = q4 * 32 + lane;
     const int q = q0 + r;
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
@@ -436,59 +506,59 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
     };
     for (int j = 0; j < n_kt; ++j) {
       if (!wait_all(s_full, j & 1)) { ok = false; break; }
-      if (j > 0 && !wait_all(dq_done, (j - 1) & 1)) { ok = false; break; }
       ptx::tc_fence_after();
-      const int kbase = j * BKV;
-      const bool full_tile = kbase + BKV <= len;
+      uint32_t sv[32], dv[32];
+      ptx::tmem_ld_32x32b_x32(tS + lane_base + hf * 32, sv);
+      ptx::tmem_ld_32x32b_x32(tdP + lane_base + hf * 32, dv);
+      ptx::tmem_ld_wait();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(s_free);
+      const int kbase = j * BKV + hf * 32;
+      uint32_t pk[16];
 #pragma unroll
-      for (int c = 0; c < BKV / 32; ++c) {
-        uint32_t sv[32], dv[32];
-        ptx::tmem_ld_32x32b_x32(tS + lane_base + c * 32, sv);
-        ptx::tmem_ld_32x32b_x32(tdP + lane_base + c * 32, dv);
-        ptx::tmem_ld_wait();
-        float ds[32];
+      for (int i = 0; i < 32; i += 2) {
+        float ds2[2];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float pr = ptx::ex2_ftz(fmaf(__uint_as_float(sv[i]), sl2, nlse2));
-          ds[i] = pr * (__uint_as_float(dv[i]) - dl);
+        for (int t = 0; t < 2; ++t) {
+          const float pr = ptx::ex2_ftz(fmaf(__uint_as_float(sv[i + t]), sl2, nlse2));
+          ds2[t] = pr * (__uint_as_float(dv[i + t]) - dl);
         }
-        if (!full_tile) {
+        pk[i >> 1] = ptx::pack_bf16(ds2[0], ds2[1]);
+      }
+      if (kbase + 32 > len) {  // warp-uniform: only the last tile holds masked keys
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (kbase + c * 32 + i >= len) ds[i] = 0.f;
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int unit = c * 4 + u;
-          *reinterpret_cast<uint4*>(drow + ((unit ^ (r & 7)) << 4)) =
-              make_uint4(ptx::pack_bf16(ds[8 * u], ds[8 * u + 1]),
-                         ptx::pack_bf16(ds[8 * u + 2], ds[8 * u + 3]),
-                         ptx::pack_bf16(ds[8 * u + 4], ds[8 * u + 5]),
-                         ptx::pack_bf16(ds[8 * u + 6], ds[8 * u + 7]));
+        for (int i = 0; i < 32; i += 2) {
+          const uint32_t lo = kbase + i < len ? 0x0000ffffu : 0u;
+          const uint32_t hi = kbase + i + 1 < len ? 0xffff0000u : 0u;
+          pk[i >> 1] &= lo | hi;
         }
       }
+      // the dS buffer was last read by the dQ product of tile j - 1
+      if (j >= 1 && !wait_all(dq_done, (j - 1) & 1)) { ok = false; break; }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        *reinterpret_cast<uint4*>(drow + (((hf * 4 + u) ^ (r & 7)) << 4)) =
+            make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
       ptx::fence_proxy_async_smem();
       ptx::tc_fence_before();
       ptx::mbar_arrive(ds_full);
     }
+    // epilogue: each half writes 32 of the 64 dQ columns
     if (ok && wait_all(dq_done, (n_kt - 1) & 1)) {
       ptx::tc_fence_after();
-      __nv_bfloat16* out = p.dqkv + (static_cast<int64_t>(row0) + q) * (3 * H) + a * HD;
+      __nv_bfloat16* out = p.dqkv + (static_cast<int64_t>(row0) + q) * (3 * H) + a * HD + hf * 32;
+      uint32_t o[32];
+      ptx::tmem_ld_32x32b_x32(tdQ + lane_base + hf * 32, o);
+      ptx::tmem_ld_wait();
+      if (q < S) {
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t o[32];
-        ptx::tmem_ld_32x32b_x32(tdQ + lane_base + c * 32, o);
-        ptx::tmem_ld_wait();
-        if (q < S) {
+        for (int u = 0; u < 4; ++u) {
+          uint32_t w[4];
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            uint32_t w[4];
-#pragma unroll
-            for (int t = 0; t < 4; ++t)
-              w[t] = ptx::pack_bf16(__uint_as_float(o[8 * u + 2 * t]) * 0.125f,
-                                    __uint_as_float(o[8 * u + 2 * t + 1]) * 0.125f);
-            *reinterpret_cast<uint4*>(out + c * 32 + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-          }
+          for (int t = 0; t < 4; ++t)
+            w[t] = ptx::pack_bf16(__uint_as_float(o[8 * u + 2 * t]) * 0.125f,
+                                  __uint_as_float(o[8 * u + 2 * t + 1]) * 0.125f);
+          *reinterpret_cast<uint4*>(out + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
         }
       }
     }
@@ -508,7 +578,9 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dq_tc(const __grid_constant_
 //   P^T = exp2(S^T log2(e)/sqrt(D) - lse2_q), dS^T = P^T (dP^T - delta_q) -> smem
 //   dV += P^T dO_i, dK += dS^T Q_i (TMEM); finally dK / sqrt(D), dV -> dQKV.
 // The Q_i / dO_i tiles serve both as K-major operands (S^T, dP^T) and as
-// MN-major operands (dK, dV).
+// MN-major operands (dK, dV).  As in the dQ kernel, S^T / dP^T are released
+// (s_free) as soon as the softmax warps hold them in registers, so the next
+// tile's S^T, dP^T products overlap the forming of P^T and dS^T.
 constexpr int BK2 = 128, BQ2 = 64;
 constexpr int KV2_BYTES = BK2 * HD * 2;    // 16 KiB (K or V of 128 keys)
 constexpr int QO2_BYTES = BQ2 * HD * 2;    // 8 KiB  (Q or dO of 64 queries)
@@ -518,11 +590,11 @@ constexpr int KV_Q_OFF = 2 * KV2_BYTES;
 constexpr int KV_O_OFF = KV_Q_OFF + STAGES * QO2_BYTES;
 constexpr int KV_P_OFF = KV_O_OFF + STAGES * QO2_BYTES;
 constexpr int KV_DS_OFF = KV_P_OFF + PS2_BYTES;
-constexpr int KV_LD_OFF = KV_DS_OFF + PS2_BYTES;   // [STAGES][2][64] floats: lse2, delta
+constexpr int KV_LD_OFF = KV_DS_OFF + PS2_BYTES;   // [STAGES][2][64] floats: lse, delta
 constexpr int KV_BAR_OFF = KV_LD_OFF + STAGES * 2 * BQ2 * 4;
 constexpr int KV_SMEM = KV_BAR_OFF + 128 + 1024;
 
-__global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constant__ CUtensorMap tmK,
+__global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtensorMap tmK,
                                                             const __grid_constant__ CUtensorMap tmQ,
                                                             const __grid_constant__ CUtensorMap tmO,
                                                             const BwdParams p) {
@@ -538,7 +610,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
   const int row0 = b * S, k0 = kt * BK2;
   const int64_t rs = 3 * static_cast<int64_t>(H);
   if (k0 >= len) {  // keys of this tile are all padding: zero gradients
-    for (int i = threadIdx.x; i < BK2 * 8; i += NTHR) {
+    for (int i = threadIdx.x; i < BK2 * 8; i += NTHR_B) {
       const int rr = i >> 3, c = i & 7;
       if (k0 + rr < S) {
         __nv_bfloat16* base = p.dqkv + (static_cast<int64_t>(row0) + k0 + rr) * rs + a * HD + c * 8;
@@ -555,7 +627,8 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
   uint64_t* q_full = kv_full + 1;
   uint64_t* q_empty = q_full + STAGES;
   uint64_t* s_full = q_empty + STAGES;
-  uint64_t* pds_full = s_full + 1;
+  uint64_t* s_free = s_full + 1;
+  uint64_t* pds_full = s_free + 1;
   uint64_t* mm_done = pds_full + 1;
   uint64_t* done = mm_done + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
@@ -569,7 +642,8 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
       ptx::mbar_init(&q_empty[s], 1);
     }
     ptx::mbar_init(s_full, 1);
-    ptx::mbar_init(pds_full, 128);
+    ptx::mbar_init(s_free, NSM_B);
+    ptx::mbar_init(pds_full, NSM_B);
     ptx::mbar_init(mm_done, 1);
     ptx::mbar_init(done, 1);
     ptx::fence_mbar_init();
@@ -586,8 +660,14 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
   const uint32_t tST = tmem, tdPT = tmem + 64, tdV = tmem + 128, tdK = tmem + 192;
 
   if (warp == 0) {
-    // producer: K, V once; per query tile Q_i, dO_i by TMA and lse2 / delta by the warp
+    // producer: K, V once; per query tile Q_i, dO_i by TMA and the tile's
+    // log-sum-exp / delta values by bulk copy (or by the warp's lanes when the
+    // rows are not 16-byte aligned), all completing on q_full
+    const bool bulk = p.lse_bulk != 0;
     if (lane == 0) {
+      ptx::prefetch_tensormap(&tmK);
+      ptx::prefetch_tensormap(&tmQ);
+      ptx::prefetch_tensormap(&tmO);
       ptx::mbar_arrive_expect_tx(kv_full, 2 * KV2_BYTES);
       ptx::tma_load_2d(smem + KV_K_OFF, &tmK, kv_full, H + a * HD, row0 + k0);
       ptx::tma_load_2d(smem + KV_V_OFF, &tmK, kv_full, 2 * H + a * HD, row0 + k0);
@@ -601,17 +681,24 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
       if (lane == 0) ok = ptx::mbar_wait(&q_empty[st], ((i >> 1) & 1) ^ 1u, lim, p.status, kWaitHint);
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
       float* l2 = ldst + st * 2 * BQ2;
-      for (int t = lane; t < BQ2; t += 32) {
-        const int q = i * BQ2 + t;
-        l2[t] = q < S ? lse_b[q] * LOG2E : INFINITY;  // rows past S get P = 0
-        l2[BQ2 + t] = q < S ? del_b[q] : 0.f;
+      const int nq = min(BQ2, S - i * BQ2);  // queries of this tile inside the sequence
+      if (!bulk) {
+        for (int t = lane; t < nq; t += 32) {
+          l2[t] = lse_b[i * BQ2 + t];
+          l2[BQ2 + t] = del_b[i * BQ2 + t];
+        }
       }
       if (lane == 0) {
-        ptx::mbar_arrive_expect_tx(&q_full[st], 2 * QO2_BYTES);
+        const uint32_t lbytes = bulk ? static_cast<uint32_t>(nq) * 4u : 0u;
+        ptx::mbar_arrive_expect_tx(&q_full[st], 2 * QO2_BYTES + 2 * lbytes);
         ptx::tma_load_2d(smem + KV_Q_OFF + st * QO2_BYTES, &tmQ, &q_full[st], a * HD,
                          row0 + i * BQ2);
         ptx::tma_load_2d(smem + KV_O_OFF + st * QO2_BYTES, &tmO, &q_full[st], a * HD,
                          row0 + i * BQ2);
+        if (bulk) {
+          ptx::bulk_load(l2, lse_b + i * BQ2, lbytes, &q_full[st]);
+          ptx::bulk_load(l2 + BQ2, del_b + i * BQ2, lbytes, &q_full[st]);
+        }
       } else {
         ptx::mbar_arrive(&q_full[st]);
       }
@@ -628,11 +715,9 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
       constexpr uint32_t idG = ptx::idesc_bf16_f32(BK2, HD, false, true);
       const uint32_t sk = ptx::smem_u32(smem + KV_K_OFF), sv = ptx::smem_u32(smem + KV_V_OFF);
       const uint32_t sp = ptx::smem_u32(smem + KV_P_OFF), sds = ptx::smem_u32(smem + KV_DS_OFF);
-      bool ok = ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint);
-      for (int i = 0; i < n_qt && ok; ++i) {
+      // S^T_i = K Q_i^T and dP^T_i = V dO_i^T (operands already landed)
+      auto mma_st = [&](int i) {
         const int st = i & 1;
-        if (!ptx::mbar_wait(&q_full[st], (i >> 1) & 1, lim, p.status, kWaitHint)) break;
-        ptx::tc_fence_after();
         const uint32_t sq = ptx::smem_u32(smem + KV_Q_OFF + st * QO2_BYTES);
         const uint32_t so = ptx::smem_u32(smem + KV_O_OFF + st * QO2_BYTES);
 #pragma unroll
@@ -644,8 +729,33 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
           ptx::tc_mma_f16(tdPT, ptx::smem_desc_sw128(sv + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(so + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
         ptx::tc_commit(s_full);
-        if (!ptx::mbar_wait(pds_full, i & 1, lim, p.status, kWaitHint)) break;
+      };
+      bool ok = ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint) &&
+                ptx::mbar_wait(&q_full[0], 0, lim, p.status, kWaitHint);
+      if (ok) {
         ptx::tc_fence_after();
+        mma_st(0);
+      }
+      for (int i = 0; i < n_qt && ok; ++i) {
+        const int st = i & 1;
+        // as in the dQ kernel: tile i+1's S^T / dP^T go in as soon as tile i's
+        // are in registers and Q_{i+1} / dO_{i+1} have landed, without holding
+        // up tile i's dV / dK products
+        const int in = i + 1;
+        bool next_done = in >= n_qt;
+        auto next_ready = [&] {
+          return ptx::mbar_try_wait(s_free, i & 1) &&
+                 ptx::mbar_try_wait(&q_full[in & 1], (in >> 1) & 1);
+        };
+        auto next_issue = [&] {
+          ptx::tc_fence_after();
+          mma_st(in);
+        };
+        if (!ptx::mbar_wait_with(pds_full, i & 1, lim, p.status, kWaitHint, next_done, next_ready, next_issue))
+          break;
+        ptx::tc_fence_after();
+        const uint32_t sq = ptx::smem_u32(smem + KV_Q_OFF + st * QO2_BYTES);
+        const uint32_t so = ptx::smem_u32(smem + KV_O_OFF + st * QO2_BYTES);
 #pragma unroll
         for (int kk = 0; kk < BQ2 / 16; ++kk) {
           ptx::tc_mma_f16(tdV, ptx::smem_desc_sw128(sp + kk * 32, 16, 1024),
@@ -657,13 +767,20 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
         }
         ptx::tc_commit(mm_done);
         ptx::tc_commit(&q_empty[st]);
+        if (!next_done) {
+          if (!ptx::mbar_wait(s_free, i & 1, lim, p.status, kWaitHint) ||
+              !ptx::mbar_wait(&q_full[in & 1], (in >> 1) & 1, lim, p.status, kWaitHint))
+            break;
+          next_issue();
+        }
       }
       ptx::tc_commit(done);
       ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
     }
   } else {
     const int q4 = warp & 3;
-    const int r = q4 * 32 + lane;  // key row within the tile == TMEM lane
+    const int hf = (warp - 2) >> 2;  // column half: queries [32 hf, 32 hf + 32) of a tile
+    const int r = q4 * 32 + lane;    // key row within the tile == TMEM lane
     const int key = k0 + r;
     const bool kvalid = key < len;
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
@@ -679,68 +796,76 @@ __global__ void __launch_bounds__(NTHR, 2) attn_bwd_dkdv_tc(const __grid_constan
       const int st = i & 1;
       if (!wait_all(&q_full[st], (i >> 1) & 1)) { ok = false; break; }
       if (!wait_all(s_full, i & 1)) { ok = false; break; }
-      if (i > 0 && !wait_all(mm_done, (i - 1) & 1)) { ok = false; break; }
       ptx::tc_fence_after();
-      const float* l2 = ldst + st * 2 * BQ2;
+      uint32_t sv[32], dv[32];
+      ptx::tmem_ld_32x32b_x32(tST + lane_base + hf * 32, sv);
+      ptx::tmem_ld_32x32b_x32(tdPT + lane_base + hf * 32, dv);
+      ptx::tmem_ld_wait();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(s_free);
+      const float* l2 = ldst + st * 2 * BQ2 + hf * 32;
+      uint32_t pp[16], dd[16];
 #pragma unroll
-      for (int c = 0; c < BQ2 / 32; ++c) {
-        uint32_t sv[32], dv[32];
-        ptx::tmem_ld_32x32b_x32(tST + lane_base + c * 32, sv);
-        ptx::tmem_ld_32x32b_x32(tdPT + lane_base + c * 32, dv);
-        ptx::tmem_ld_wait();
-        float pt[32], ds[32];
+      for (int t = 0; t < 32; t += 4) {
+        // lse / delta of queries t .. t+3: one broadcast 16-byte load each
+        const float4 lq = *reinterpret_cast<const float4*>(l2 + t);
+        const float4 dq = *reinterpret_cast<const float4*>(l2 + BQ2 + t);
+        const float lv[4] = {lq.x * LOG2E, lq.y * LOG2E, lq.z * LOG2E, lq.w * LOG2E};
+        const float dlv[4] = {dq.x, dq.y, dq.z, dq.w};
+        float pt[4], ds[4];
 #pragma unroll
-        for (int t = 0; t < 32; ++t) {
-          const int qq = c * 32 + t;
-          pt[t] = kvalid ? ptx::ex2_ftz(fmaf(__uint_as_float(sv[t]), sl2, -l2[qq])) : 0.f;
-          ds[t] = pt[t] * (__uint_as_float(dv[t]) - l2[BQ2 + qq]);
+        for (int e = 0; e < 4; ++e) {
+          pt[e] = kvalid ? ptx::ex2_ftz(fmaf(__uint_as_float(sv[t + e]), sl2, -lv[e])) : 0.f;
+          ds[e] = pt[e] * (__uint_as_float(dv[t + e]) - dlv[e]);
         }
+        pp[t >> 1] = ptx::pack_bf16(pt[0], pt[1]);
+        pp[(t >> 1) + 1] = ptx::pack_bf16(pt[2], pt[3]);
+        dd[t >> 1] = ptx::pack_bf16(ds[0], ds[1]);
+        dd[(t >> 1) + 1] = ptx::pack_bf16(ds[2], ds[3]);
+      }
+      const int nq = S - i * BQ2 - hf * 32;  // queries of this half inside the sequence
+      if (nq < 32) {  // warp-uniform: queries past S (their lse / delta slots are stale)
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int unit = c * 4 + u;
-          const int pos = (unit ^ (r & 7)) << 4;
-          *reinterpret_cast<uint4*>(prow + pos) =
-              make_uint4(ptx::pack_bf16(pt[8 * u], pt[8 * u + 1]),
-                         ptx::pack_bf16(pt[8 * u + 2], pt[8 * u + 3]),
-                         ptx::pack_bf16(pt[8 * u + 4], pt[8 * u + 5]),
-                         ptx::pack_bf16(pt[8 * u + 6], pt[8 * u + 7]));
-          *reinterpret_cast<uint4*>(drow + pos) =
-              make_uint4(ptx::pack_bf16(ds[8 * u], ds[8 * u + 1]),
-                         ptx::pack_bf16(ds[8 * u + 2], ds[8 * u + 3]),
-                         ptx::pack_bf16(ds[8 * u + 4], ds[8 * u + 5]),
-                         ptx::pack_bf16(ds[8 * u + 6], ds[8 * u + 7]));
+        for (int t = 0; t < 32; t += 2) {
+          const uint32_t keep = (t < nq ? 0x0000ffffu : 0u) | (t + 1 < nq ? 0xffff0000u : 0u);
+          pp[t >> 1] &= keep;
+          dd[t >> 1] &= keep;
         }
+      }
+      // P^T / dS^T buffers were last read by the dV / dK products of tile i - 1
+      if (i > 0 && !wait_all(mm_done, (i - 1) & 1)) { ok = false; break; }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int pos = ((hf * 4 + u) ^ (r & 7)) << 4;
+        *reinterpret_cast<uint4*>(prow + pos) = make_uint4(pp[4 * u], pp[4 * u + 1], pp[4 * u + 2], pp[4 * u + 3]);
+        *reinterpret_cast<uint4*>(drow + pos) = make_uint4(dd[4 * u], dd[4 * u + 1], dd[4 * u + 2], dd[4 * u + 3]);
       }
       ptx::fence_proxy_async_smem();
       ptx::tc_fence_before();
       ptx::mbar_arrive(pds_full);
     }
+    // epilogue: the low-half warps write dK / sqrt(D), the high-half warps dV
     if (ok && wait_all(mm_done, (n_qt - 1) & 1)) {
       ptx::tc_fence_after();
-      __nv_bfloat16* outk = p.dqkv + (static_cast<int64_t>(row0) + key) * rs + H + a * HD;
-      __nv_bfloat16* outv = outk + H;
+      const uint32_t tacc = hf == 0 ? tdK : tdV;
+      const float sc = hf == 0 ? 0.125f : 1.f;
+      __nv_bfloat16* out = p.dqkv + (static_cast<int64_t>(row0) + key) * rs + (1 + hf) * H + a * HD;
+      uint32_t o[2][32];
+      ptx::tmem_ld_32x32b_x32(tacc + lane_base, o[0]);
+      ptx::tmem_ld_32x32b_x32(tacc + lane_base + 32, o[1]);
+      ptx::tmem_ld_wait();
+      if (key < S) {
 #pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        const uint32_t tacc = which == 0 ? tdK : tdV;
-        const float sc = which == 0 ? 0.125f : 1.f;
-        __nv_bfloat16* out = which == 0 ? outk : outv;
+        for (int c = 0; c < 2; ++c)
 #pragma unroll
-        for (int c = 0; c < HD / 32; ++c) {
-          uint32_t o[32];
-          ptx::tmem_ld_32x32b_x32(tacc + lane_base + c * 32, o);
-          ptx::tmem_ld_wait();
-          if (key < S) {
+          for (int u = 0; u < 4; ++u) {
+            uint32_t w[4];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              uint32_t w[4];
-#pragma unroll
-              for (int t = 0; t < 4; ++t)
-                w[t] = ptx::pack_bf16(__uint_as_float(o[8 * u + 2 * t]) * sc,
-                                      __uint_as_float(o[8 * u + 2 * t + 1]) * sc);
-              *reinterpret_cast<uint4*>(out + c * 32 + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-            }
+            for (int t = 0; t < 4; ++t)
+              w[t] = ptx::pack_bf16(__uint_as_float(o[c][8 * u + 2 * t]) * sc,
+                                    __uint_as_float(o[c][8 * u + 2 * t + 1]) * sc);
+            *reinterpret_cast<uint4*>(out + c * 32 + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
           }
-        }
       }
     }
   }
@@ -796,11 +921,11 @@ sky_status attention_fwd_tc(const void* qkv, const int32_t* lens, int B, int S, 
   SKY_CHECK(head_map(&tq, qkv, T, 3 * H, BQ) && head_map(&tkv, qkv, T, 3 * H, BKV), SKY_ERR_CUDA,
             "cuTensorMapEncodeTiled failed for the attention operands");
   static cudaError_t attr = cudaFuncSetAttribute(attn_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 SMEM_BYTES);
+                                                 F_SMEM);
   if (attr != cudaSuccess) return cuda_fail(attr, "attention smem attribute");
   FwdParams p{S, H, A, lens, static_cast<__nv_bfloat16*>(ctx), lse, status, timeout_ns};
   dim3 grid(ceil_div(S, BQ), A, B);
-  attn_fwd_tc<<<grid, NTHR, SMEM_BYTES, stream>>>(tq, tkv, p);
+  attn_fwd_tc<<<grid, NTHR, F_SMEM, stream>>>(tq, tkv, p);
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "tensor-core attention forward launch");
@@ -822,9 +947,11 @@ sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse,
   static cudaError_t a2 = cudaFuncSetAttribute(attn_bwd_dkdv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, KV_SMEM);
   if (a1 != cudaSuccess) return cuda_fail(a1, "attention dQ smem attribute");
   if (a2 != cudaSuccess) return cuda_fail(a2, "attention dK/dV smem attribute");
-  BwdParams p{S, H, A, lens, lse, delta, static_cast<__nv_bfloat16*>(dqkv), status, timeout_ns};
-  attn_bwd_dkdv_tc<<<dim3(ceil_div(S, BK2), A, B), NTHR, KV_SMEM, stream>>>(tk128, tq64, to64, p);
-  attn_bwd_dq_tc<<<dim3(ceil_div(S, BQ), A, B), NTHR, DQ_SMEM, stream>>>(tq128, tkv64, to128, p);
+  const int bulk = (S % 4 == 0) && (reinterpret_cast<uintptr_t>(lse) & 15) == 0 &&
+                   (reinterpret_cast<uintptr_t>(delta) & 15) == 0;
+  BwdParams p{S, H, A, bulk, lens, lse, delta, static_cast<__nv_bfloat16*>(dqkv), status, timeout_ns};
+  attn_bwd_dkdv_tc<<<dim3(ceil_div(S, BK2), A, B), NTHR_B, KV_SMEM, stream>>>(tk128, tq64, to64, p);
+  attn_bwd_dq_tc<<<dim3(ceil_div(S, BQ), A, B), NTHR_B, DQ_SMEM, stream>>>(tq128, tkv64, to128, p);
   count_launches(2);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "tensor-core attention backward launch");

@@ -79,6 +79,29 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
   }
 }
 
+// mbar_wait that does side work while it waits: `side()` runs once, as soon
+// as `ready()` holds (checked between polls), unless `side_done` is already
+// set; `side_done` reports whether it ran.  Once the side work is done the
+// thread waits with the suspend-time hint like mbar_wait.  Same time bound
+// and status bit as mbar_wait.
+template <class Ready, class Side>
+__device__ __forceinline__ bool mbar_wait_with(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
+                                               int32_t* status, uint32_t hint_ns, bool& side_done,
+                                               Ready ready, Side side) {
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (!side_done && ready()) {
+      side();
+      side_done = true;
+    }
+    if (side_done ? mbar_try_wait(bar, parity, hint_ns) : mbar_try_wait(bar, parity)) return true;
+    if ((it & 15u) == 0 && global_timer_ns() - t0 > limit_ns) {
+      if (status) atomicOr(status, 2);
+      return false;
+    }
+  }
+}
+
 // --------------------------------------------------------------------- TMA
 // 2-D tiled bulk-tensor load global -> shared, completing on `bar` (tx bytes).
 // c0 is the innermost (contiguous) coordinate in elements, c1 the row.
