@@ -236,7 +236,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       float* outf = OUT_F32 ? static_cast<float*>(p.C) +
                                   static_cast<int64_t>(split) * p.M * static_cast<int64_t>(p.N)
                             : nullptr;
-#pragma unroll
+      // The GELU epilogue keeps its chunk loop rolled: unrolled, its
+      // straight-line code overflows the instruction cache.
+#pragma unroll (EPI == SKY_EPI_BIAS_GELU ? 1 : CHUNKS)
       for (int cc = 0; cc < CHUNKS; ++cc) {
         const int c = cc * 32;
         uint32_t r[32];

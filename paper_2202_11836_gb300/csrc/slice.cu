@@ -102,6 +102,15 @@ struct sky_slice {
   void* ws;
   size_t ws_bytes;
   int32_t* d_status;
+  // Weight-gradient GEMMs of a bf16 backward run on a second stream, so they
+  // fill the SMs that the data-gradient chain leaves idle.  ev_in[j]: input j
+  // of the side stream (dU2, dZ, dU1, dQKV) is ready on the caller's stream;
+  // ev_out[j]: the side GEMM reading input j is done, so the next layer may
+  // overwrite that buffer.  ws2: the side GEMMs' split-K scratch.
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_in[4] = {}, ev_out[4] = {}, ev_join = nullptr;
+  void* ws2 = nullptr;
+  size_t ws2_bytes = 0;
   // state of the most recent forward
   bool have_fwd = false;
   int B = 0, S = 0;
@@ -152,6 +161,17 @@ size_t workspace_need(const sky_slice* s, int64_t T) {
   return need;
 }
 
+// Split-K scratch of the weight-gradient GEMMs (their own, so they can run
+// beside the main stream's kernels).
+size_t side_workspace_need(const sky_slice* s, int64_t T) {
+  const int H = s->H, F = s->F;
+  size_t need = 0;
+  const int64_t shapes[4][2] = {{3 * H, H}, {H, H}, {F, H}, {H, F}};
+  for (auto& sh : shapes)
+    need = std::max(need, gemm::workspace_bytes(SKY_GEMM_XTW, (int)sh[0], (int)sh[1], (int)T, true));
+  return need;
+}
+
 cudaEvent_t next_event(sky_slice* s) {
   if (s->event_next == s->event_pool.size()) {
     cudaEvent_t e;
@@ -182,11 +202,16 @@ struct Timed {
 
 sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, int M, int N,
                     int K, const void* A, const void* Bm, void* C, bool out_f32, int epi,
-                    const void* bias, const void* aux, void* aux_out, float* colsum = nullptr) {
+                    const void* bias, const void* aux, void* aux_out, float* colsum = nullptr,
+                    void* ws = nullptr, size_t ws_bytes = 0) {
   Timed t(s, st, cat, 2.0 * M * N * K, 0);
+  if (!ws) {
+    ws = s->ws;
+    ws_bytes = s->ws_bytes;
+  }
   if (s->cfg.dtype == SKY_DTYPE_BF16)
-    return gemm::launch_bf16(form, M, N, K, A, Bm, C, out_f32, epi, bias, aux, aux_out, s->ws,
-                             s->ws_bytes, s->d_status, st, colsum);
+    return gemm::launch_bf16(form, M, N, K, A, Bm, C, out_f32, epi, bias, aux, aux_out, ws,
+                             ws_bytes, s->d_status, st, colsum);
   return gemm::launch_f32(form, M, N, K, static_cast<const float*>(A),
                           static_cast<const float*>(Bm), static_cast<float*>(C), epi,
                           static_cast<const float*>(bias), static_cast<const float*>(aux),
@@ -254,7 +279,7 @@ sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
 // (the caller's dy for the top layer) and dY2 fp32 or null.  Outputs go to
 // dP[k] and dR[k]; for the slice's first layer they are added into dx.
 sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, const float* dY2,
-                          int k, void* dx, cudaStream_t st) {
+                          int k, void* dx, cudaStream_t st, cudaStream_t sw) {
   LayerBufs& Lb = s->layers[i];
   const int B = s->B, S = s->S, H = s->H, A = s->A, F = s->F;
   const int T = B * S;
@@ -263,13 +288,37 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   const double e = (double)s->esz;
   const double dye = (dy_dt == SKY_DTYPE_BF16 ? 2.0 : 4.0) + (dY2 ? 4.0 : 0.0);
   void* dU1b = bf ? s->dU1b : s->dR[k];
+  // Weight gradients go to stream sw (== st when they run in line).  fork(j)
+  // hands input j to sw; reuse(j) makes st wait until the previous layer's
+  // weight-gradient GEMM has finished reading buffer j before st overwrites it;
+  // done(j) marks that GEMM's completion.
+  const bool two = sw != st;
+  auto fork = [&](int j) -> sky_status {
+    if (!two) return SKY_OK;
+    SKY_CUDA(cudaEventRecord(s->ev_in[j], st));
+    SKY_CUDA(cudaStreamWaitEvent(sw, s->ev_in[j], 0));
+    return SKY_OK;
+  };
+  auto reuse = [&](int j) -> sky_status {
+    if (two) SKY_CUDA(cudaStreamWaitEvent(st, s->ev_out[j], 0));
+    return SKY_OK;
+  };
+  auto done = [&](int j) -> sky_status {
+    if (two) SKY_CUDA(cudaEventRecord(s->ev_out[j], sw));
+    return SKY_OK;
+  };
+  void* ws2 = bf ? s->ws2 : nullptr;
+  const size_t ws2b = s->ws2_bytes;
   // a9: LN2 backward -> dU2 (fp32 + dtype), dgamma2, dbeta2, db2
+  SKY_TRY(reuse(0));
   {
     Timed t(s, st, P_LN_BWD, 0, (dye + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(dY, dy_dt, dY2, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
                           bf ? s->dU2_32 : nullptr, s->dU2b, Lb.g[10], Lb.g[11], Lb.g[9], s->ws,
                           s->ws_bytes, st));
   }
+  SKY_TRY(fork(0));
+  SKY_TRY(reuse(1));
   // a10 + a11: dZ = (dU2 W2) * GELU'(Z);  dW2 = dU2^T G
   //          db1 = sum_rows dZ (fused into the bf16 epilogue; a column-sum pass for fp32)
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
@@ -278,26 +327,33 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, st, P_COLSUM, 0, e * T * F);
     SKY_TRY(column_sum(s->dH, T, F, dt, Lb.g[7], s->ws, s->ws_bytes, st));
   }
-  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  SKY_TRY(fork(1));
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
+  SKY_TRY(done(0));
   // a12: P1 = dZ W1 (fp32; dX1 = P1 + dU2 is formed by the LN1 backward);  dW1 = dZ^T X1
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dP1, true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
-  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, F, H, T, s->dH, Lb.X1b, Lb.g[6], true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, F, H, T, s->dH, Lb.X1b, Lb.g[6], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
+  SKY_TRY(done(1));
   // a13: LN1 backward of dX1 = P1 + dU2 -> dU1 (fp32 + dtype), dgamma1, dbeta1, dbo
+  SKY_TRY(reuse(2));
   {
     Timed t(s, st, P_LN_BWD, 0, (4.0 + 4.0 + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? s->dU2_32 : static_cast<float*>(s->dU2b),
                           Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H, dt, bf ? s->dR[k] : nullptr,
                           dU1b, Lb.g[4], Lb.g[5], Lb.g[3], s->ws, s->ws_bytes, st));
   }
+  SKY_TRY(fork(2));
   // a14: dctx = dU1 Wo;  dWo = dU1^T ctx
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, H, dU1b, Lb.p[2], s->dctx, false,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
-  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, H, H, T, dU1b, Lb.ctx, Lb.g[2], true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, H, T, dU1b, Lb.ctx, Lb.g[2], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
+  SKY_TRY(done(2));
   // a15: attention backward -> dQKV
+  SKY_TRY(reuse(3));
   {
     Timed t(s, st, P_ATTN_BWD, 8.0 * H * S * (double)T, e * T * 8.0 * H);
     SKY_TRY(attention_bwd(Lb.QKV, Lb.ctx, s->dctx, Lb.lse, s->d_len, B, S, H, A, dt, s->dqkv,
@@ -307,6 +363,7 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, st, P_COLSUM, 0, e * T * 3.0 * H);
     SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], s->ws, s->ws_bytes, st));
   }
+  SKY_TRY(fork(3));
   // a16: dX = dQKV Wqkv + dU1 (the sum is formed by the next LayerNorm backward,
   // or here for the slice's first layer);  dWqkv = dQKV^T X
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, 3 * H, s->dqkv, Lb.p[0], s->dP[k], true,
@@ -316,8 +373,9 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     SKY_TRY(add_f32(s->dP[k], s->dR[k], (int64_t)T * H,
                     s->cfg.io_fp32 ? SKY_DTYPE_FP32 : dt, dx, st));
   }
-  SKY_TRY(run_gemm(s, st, P_GEMM_WGRAD, SKY_GEMM_XTW, 3 * H, H, T, s->dqkv, Lb.Xb, Lb.g[0], true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, 3 * H, H, T, s->dqkv, Lb.Xb, Lb.g[0], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
+  SKY_TRY(done(3));
   return SKY_OK;
 }
 
@@ -348,16 +406,38 @@ sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
   const void* cur = dy;
   const float* cur2 = nullptr;
   sky_dtype cur_dt = s->cfg.io_fp32 ? SKY_DTYPE_FP32 : s->cfg.dtype;
+  // The side stream is used unless kernels are being timed one by one.  It
+  // joins the caller's stream at the end (and after every layer when the
+  // per-layer cost is being measured), so the caller's stream still orders
+  // everything the backward pass does.
+  cudaStream_t sw = (s->side && !s->prof) ? s->side : st;
+  auto join = [&]() -> sky_status {
+    if (sw == st) return SKY_OK;
+    SKY_CUDA(cudaEventRecord(s->ev_join, sw));
+    SKY_CUDA(cudaStreamWaitEvent(st, s->ev_join, 0));
+    return SKY_OK;
+  };
+  if (sw != st) {  // the side stream starts after everything before this call
+    SKY_CUDA(cudaEventRecord(s->ev_join, st));
+    SKY_CUDA(cudaStreamWaitEvent(sw, s->ev_join, 0));
+  }
   for (int i = s->L - 1; i >= 0; --i) {
     const int k = (s->L - 1 - i) & 1;
     if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i], st));
-    SKY_TRY(backward_layer(s, i, cur, cur_dt, cur2, k, i == 0 ? dx : nullptr, st));
-    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
+    const sky_status rc = backward_layer(s, i, cur, cur_dt, cur2, k, i == 0 ? dx : nullptr, st, sw);
+    if (rc != SKY_OK) {
+      join();
+      return rc;
+    }
+    if (marks) {
+      SKY_TRY(join());
+      SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
+    }
     cur = s->dP[k];
     cur2 = s->dR[k];
     cur_dt = SKY_DTYPE_FP32;
   }
-  return SKY_OK;
+  return join();
 }
 
 int layer_index(const sky_slice* s, int32_t layer) {
@@ -450,9 +530,11 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   s->grad_bytes = gb * s->L;
   s->stash_bytes = stash * s->L;
   s->ws_bytes = align_up(workspace_need(s, T));
-  // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | status
+  s->ws2_bytes = bf ? align_up(side_workspace_need(s, T)) : 0;
+  // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | ws2 | status
   const size_t wk = 6 * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
-                    align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes + 256;
+                    align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes +
+                    s->ws2_bytes + 256;
   s->ws_bytes_total = wk;
   *total = s->param_bytes + s->grad_bytes + s->stash_bytes + wk;
   return SKY_OK;
@@ -558,7 +640,21 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   s->dqkv = take((size_t)T * 3 * s->H * s->esz);
   s->delta = static_cast<float*>(take(lse_b));
   s->ws = take(s->ws_bytes);
+  if (s->ws2_bytes) s->ws2 = take(s->ws2_bytes);
   s->d_status = static_cast<int32_t*>(take(4));
+  if (bf) {
+    // the weight-gradient side stream and its events
+    bool ok = cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) == cudaSuccess;
+    for (int j = 0; j < 4 && ok; ++j)
+      ok = cudaEventCreateWithFlags(&s->ev_in[j], cudaEventDisableTiming) == cudaSuccess &&
+           cudaEventCreateWithFlags(&s->ev_out[j], cudaEventDisableTiming) == cudaSuccess;
+    if (ok) ok = cudaEventCreateWithFlags(&s->ev_join, cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+      const cudaError_t ce = cudaGetLastError();
+      sky_slice_destroy(s);
+      return cuda_fail(ce, "side stream / events");
+    }
+  }
   *out = s;
   return SKY_OK;
   ABI_GUARD_END
@@ -569,6 +665,12 @@ sky_status sky_slice_destroy(sky_slice* s) {
   if (!s) return SKY_OK;
   cudaDeviceSynchronize();
   for (auto e : s->event_pool) cudaEventDestroy(e);
+  for (int j = 0; j < 4; ++j) {
+    if (s->ev_in[j]) cudaEventDestroy(s->ev_in[j]);
+    if (s->ev_out[j]) cudaEventDestroy(s->ev_out[j]);
+  }
+  if (s->ev_join) cudaEventDestroy(s->ev_join);
+  if (s->side) cudaStreamDestroy(s->side);
   if (s->arena) cudaFree(s->arena);
   delete s;
   return SKY_OK;

@@ -45,8 +45,12 @@ def to_host(t):
     return t.float().cpu().numpy().astype(np.float64)
 
 
-def run_gpu_slice(w, X, lens, dY, params, affine_layers, eps=1e-12):
-    """Runs forward+backward of workload ``w`` on the GPU; returns (Y, dX, grads)."""
+def run_gpu_slice(w, X, lens, dY, params, affine_layers, eps=1e-12, steps=1, profiling=False):
+    """Runs forward+backward of workload ``w`` on the GPU; returns (Y, dX, grads).
+
+    ``steps`` > 1 repeats the step back to back on one stream (results of the
+    last one are returned); ``profiling`` runs every kernel in line on the
+    caller's stream (per-kernel timing mode)."""
     import torch
     from paper_2202_11836_gb300.slice import EncoderSlice
     B = X.shape[0]
@@ -54,11 +58,13 @@ def run_gpu_slice(w, X, lens, dY, params, affine_layers, eps=1e-12):
                       B, w.seq, w.dtype, eps) as s:
         for i, p in enumerate(params):
             s.set_params(w.layer_begin + i, p)
+        s.set_profiling(profiling)
         x = to_device(X, w.dtype)
         ln = torch.from_numpy(np.asarray(lens, np.int32)).cuda()
         dy = to_device(dY, w.dtype)
-        y = s.forward(x, ln)
-        dx = s.backward(dy)
+        for _ in range(steps):
+            y = s.forward(x, ln)
+            dx = s.backward(dy)
         s.sync()
         grads = [s.get_grads(w.layer_begin + i) for i in range(len(params))]
         return to_host(y), to_host(dx), grads
