@@ -19,7 +19,15 @@
 //               tile's main loop.
 // K-major operands (x and W in y = x W^T) and MN-major operands (W in
 // dy W, and both operands of dy^T x) are read directly through the
-// descriptors' major-ness bit, so no transpose pass exists.  Weight gradients
+// descriptors' major-ness bit, so no transpose pass exists.
+// Large problems run the CTA-pair variant: a cluster of two CTAs on two SMs
+// computes a 256 x 256 tile with tcgen05.mma.cta_group::2 (M = 256); each CTA
+// loads its 128 rows of A and half of the tile's B columns, so every SM moves
+// a third less operand data per FLOP through shared memory and L2 than with
+// the single-CTA 128 x 256 tile.  The leader CTA's thread issues the MMAs;
+// both CTAs' TMA loads complete on the leader's stage barrier, and the
+// leader's commits arrive on both CTAs' stage-empty and accumulator barriers.
+// Weight gradients
 // (fp32 output) may split the token dimension over CTAs; partials go to a
 // workspace and are summed in a fixed order, so results are deterministic.
 #include <cuda.h>
@@ -48,6 +56,11 @@ constexpr int EPI_BYTES = NUM_EPI_WARPS * 32 * 32 * 4;
 constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
 constexpr int SMEM_BYTES = BAR_OFF + 256 /*barriers*/ + 1024 /*alignment slack*/;
 constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
+// CTA-pair variant: per CTA and stage A 128 x 64 + B 128 x 64 (32 KiB), six
+// stages in the same 192 KiB
+constexpr int PAIR_STAGES = 6;
+constexpr int PAIR_STAGE_BYTES = A_BYTES + (BN / 2) * BK * 2;
+static_assert(PAIR_STAGES * PAIR_STAGE_BYTES == STAGES * STAGE_BYTES, "same ring size");
 constexpr uint32_t kSleepNs = 20000;         // suspend hint of the epilogue's accumulator wait
 
 struct Params {
@@ -72,42 +85,60 @@ __device__ __forceinline__ uint2 ld_nc_u2(const void* p) {
   return v;
 }
 
-template <bool A_MN, bool B_MN, int EPI, bool OUT_F32>
+// PAIR: the CTA-pair variant (launched in clusters of two; p.m_tiles counts
+// 256-row tiles).
+template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA,
                    const __grid_constant__ CUtensorMap tmB, const Params p) {
+  constexpr int NST = PAIR ? PAIR_STAGES : STAGES;
+  constexpr int SBYTES = PAIR ? PAIR_STAGE_BYTES : STAGE_BYTES;
+  constexpr int B_ROWS = PAIR ? BN / 2 : BN;  // B rows (tile columns) this CTA loads
+  constexpr int TILE_M = PAIR ? 2 * BM : BM;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + BAR_OFF);
-  uint64_t* empty = full + STAGES;
-  uint64_t* tfull = empty + STAGES;
+  uint64_t* empty = full + NST;
+  uint64_t* tfull = empty + NST;
   uint64_t* tempty = tfull + 2;
   uint64_t* done = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR ? ptx::cluster_ctarank() : 0u;
+  const bool leader = rank == 0;
+  const int cid = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int ncl = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < NST; ++s) {
       ptx::mbar_init(&full[s], 1);
       ptx::mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(&tfull[a], 1);
-      ptx::mbar_init(&tempty[a], 32 * NUM_EPI_WARPS);
+      ptx::mbar_init(&tempty[a], (PAIR ? 2 : 1) * 32 * NUM_EPI_WARPS);
     }
     ptx::mbar_init(done, 1);
-    ptx::fence_mbar_init();
+    if constexpr (PAIR) ptx::fence_mbar_init_cluster();
+    else ptx::fence_mbar_init();
     ptx::fence_proxy_async_smem();
     ptx::prefetch_tensormap(&tmA);
     ptx::prefetch_tensormap(&tmB);
   }
   if (warp == 1) {
-    ptx::tmem_alloc(tmem_slot, TMEM_COLS);
-    ptx::tmem_relinquish();
+    if constexpr (PAIR) {
+      ptx::tmem_alloc_pair(tmem_slot, TMEM_COLS);
+      ptx::tmem_relinquish_pair();
+    } else {
+      ptx::tmem_alloc(tmem_slot, TMEM_COLS);
+      ptx::tmem_relinquish();
+    }
   }
   ptx::tc_fence_before();
-  __syncthreads();
+  __syncwarp();
+  if constexpr (PAIR) ptx::cluster_sync();  // barriers of both CTAs initialised
+  else __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -122,63 +153,81 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      for (int u = cid; u < units && ok; u += ncl) {
         const int split = u / tiles, rem = u % tiles;
-        const int m0 = (rem / p.n_tiles) * BM, n0 = (rem % p.n_tiles) * BN;
+        const int m0 = (rem / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
+        const int n0 = (rem % p.n_tiles) * BN + static_cast<int>(rank) * (BN - B_ROWS);
         const int kb0 = split * p.kb_per_split;
         const int kb1 = min(p.k_blocks, kb0 + p.kb_per_split);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, lim, p.status)) { ok = false; break; }
-          uint8_t* sa = smem + stage * STAGE_BYTES;
+          uint8_t* sa = smem + stage * SBYTES;
           uint8_t* sb = sa + A_BYTES;
-          ptx::mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+          // the leader's stage barrier expects both CTAs' bytes
+          if (leader) ptx::mbar_arrive_expect_tx(&full[stage], (PAIR ? 2 : 1) * SBYTES);
           if (!p.skip_loads) {
             const int k0 = kb * BK;
+            auto load = [&](void* dst, const CUtensorMap* map, int c0, int c1) {
+              if constexpr (PAIR)
+                ptx::tma_load_2d_pair(dst, map, ptx::mapa_shared(ptx::smem_u32(&full[stage]), 0),
+                                      c0, c1);
+              else
+                ptx::tma_load_2d(dst, map, &full[stage], c0, c1);
+            };
             if (A_MN) {
-              ptx::tma_load_2d(sa, &tmA, &full[stage], m0, k0);
-              ptx::tma_load_2d(sa + MN_CHUNK_BYTES, &tmA, &full[stage], m0 + 64, k0);
+              load(sa, &tmA, m0, k0);
+              load(sa + MN_CHUNK_BYTES, &tmA, m0 + 64, k0);
             } else {
-              ptx::tma_load_2d(sa, &tmA, &full[stage], k0, m0);
+              load(sa, &tmA, k0, m0);
             }
             if (B_MN) {
 #pragma unroll
-              for (int j = 0; j < BN / 64; ++j)
-                ptx::tma_load_2d(sb + j * MN_CHUNK_BYTES, &tmB, &full[stage], n0 + 64 * j, k0);
+              for (int j = 0; j < B_ROWS / 64; ++j)
+                load(sb + j * MN_CHUNK_BYTES, &tmB, n0 + 64 * j, k0);
             } else {
-              ptx::tma_load_2d(sb, &tmB, &full[stage], k0, n0);
+              load(sb, &tmB, k0, n0);
             }
           }
           ++issued;
-          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+          if (++stage == NST) { stage = 0; phase ^= 1u; }
         }
       }
       // Drain: wait (bounded) for the loads still in flight before exiting.
-      const int n_tail = issued < STAGES ? issued : STAGES;
+      // The leader's stage barriers count the peer's loads too; the peer
+      // stays resident until the leader has drained (final cluster barrier).
+      const int n_tail = !leader ? 0 : (issued < NST ? issued : NST);
       for (int i = 0; i < n_tail; ++i) {
-        if (--stage < 0) { stage = STAGES - 1; phase ^= 1u; }
+        if (--stage < 0) { stage = NST - 1; phase ^= 1u; }
         ptx::mbar_wait(&full[stage], phase, lim, p.status);
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------- MMA issue
-    if (lane == 0) {
-      constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, BN, A_MN, B_MN);
+    if (lane == 0 && leader) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(TILE_M, BN, A_MN, B_MN);
+      auto commit = [&](uint64_t* bar) {  // to this barrier in both CTAs of a pair
+        if constexpr (PAIR) ptx::tc_commit_pair(bar, 3);
+        else ptx::tc_commit(bar);
+      };
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
       uint32_t aphase = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      for (int u = cid; u < units && ok; u += ncl) {
         const int split = u / tiles;
         const int kb0 = split * p.kb_per_split;
         const int kb1 = min(p.k_blocks, kb0 + p.kb_per_split);
-        if (!ptx::mbar_wait(&tempty[acc], aphase ^ 1u, lim, p.status)) break;
+        // both CTAs' epilogues have drained this accumulator
+        if (!(PAIR ? ptx::mbar_wait_cluster(&tempty[acc], aphase ^ 1u, lim, p.status)
+                   : ptx::mbar_wait(&tempty[acc], aphase ^ 1u, lim, p.status)))
+          break;
         ptx::tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!ptx::mbar_wait(&full[stage], phase, lim, p.status)) { ok = false; break; }
           ptx::tc_fence_after();
-          const uint32_t sa = ptx::smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sa = ptx::smem_u32(smem + stage * SBYTES);
           const uint32_t sb = sa + A_BYTES;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
@@ -186,17 +235,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                      : ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
             const uint64_t bd = B_MN ? ptx::smem_desc_sw128(sb + kk * 2048, MN_CHUNK_BYTES, 1024)
                                      : ptx::smem_desc_sw128(sb + kk * 32, 16, 1024);
-            ptx::tc_mma_f16(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+            if constexpr (PAIR)
+              ptx::tc_mma_f16_pair(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+            else
+              ptx::tc_mma_f16(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
           }
-          ptx::tc_commit(&empty[stage]);
-          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+          commit(&empty[stage]);
+          if (++stage == NST) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        ptx::tc_commit(&tfull[acc]);
+        commit(&tfull[acc]);
         if (++acc == 2) { acc = 0; aphase ^= 1u; }
       }
       // All issued MMAs must finish before TMEM is released.
-      ptx::tc_commit(done);
+      if constexpr (PAIR) ptx::tc_commit_pair(done, 1);
+      else ptx::tc_commit(done);
       ptx::mbar_wait(done, 0, lim, p.status);
     }
   } else {
@@ -212,9 +265,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int rsub = lane >> 3;       // row within each group of 4 rows
     int acc = 0;
     uint32_t aphase = 0;
-    for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    for (int u = cid; u < units; u += ncl) {
       const int split = u / tiles, rem = u % tiles;
-      const int m0 = (rem / p.n_tiles) * BM, n0 = (rem % p.n_tiles) * BN + hf * HALF;
+      const int m0 = (rem / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
+      const int n0 = (rem % p.n_tiles) * BN + hf * HALF;
       // GELU' input of this warp's whole sub-tile, fetched before the wait
       uint2 pre[EPI == SKY_EPI_GELU_BWD ? CHUNKS : 1][8];
       if constexpr (EPI == SKY_EPI_GELU_BWD) {
@@ -327,16 +381,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
       }
       ptx::tc_fence_before();
-      ptx::mbar_arrive(&tempty[acc]);
+      if (leader) ptx::mbar_arrive(&tempty[acc]);
+      else ptx::mbar_arrive_cluster(ptx::mapa_shared(ptx::smem_u32(&tempty[acc]), 0));
       if (++acc == 2) { acc = 0; aphase ^= 1u; }
     }
   }
 
   ptx::tc_fence_before();
-  __syncthreads();
+  __syncwarp();
+  if constexpr (PAIR) ptx::cluster_sync();  // no CTA leaves while its peer may still signal it
+  else __syncthreads();
   if (warp == 1) {
     ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem_base, TMEM_COLS);
+    if constexpr (PAIR) ptx::tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else ptx::tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -391,32 +449,72 @@ bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, in
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool A_MN, bool B_MN, int EPI, bool OUT_F32>
-cudaError_t launch_variant(dim3 grid, const CUtensorMap& ta, const CUtensorMap& tb,
+// Launches `units` work units on a persistent grid: one CTA per SM, or for
+// the pair variant one two-CTA cluster per SM pair, capped by how many such
+// clusters the device can hold at once (so the grid is a single wave).
+template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR>
+cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
                            const Params& p, cudaStream_t stream) {
-  static cudaError_t attr = cudaFuncSetAttribute(gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 SMEM_BYTES);
+  auto kern = gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32, PAIR>;
+  static cudaError_t attr =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (attr != cudaSuccess) return attr;
-  gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
-  return cudaGetLastError();
-}
-
-// One instantiation per (operand majorness, epilogue, output type) keeps
-// every kernel's code to the epilogue it runs.
-template <bool A_MN, bool B_MN>
-cudaError_t launch_form(dim3 grid, const CUtensorMap& ta, const CUtensorMap& tb, const Params& p,
-                        int epi, bool out_f32, cudaStream_t stream) {
-  if (out_f32) return launch_variant<A_MN, B_MN, SKY_EPI_STORE, true>(grid, ta, tb, p, stream);
-  switch (epi) {
-    case SKY_EPI_BIAS_GELU:
-      return launch_variant<A_MN, B_MN, SKY_EPI_BIAS_GELU, false>(grid, ta, tb, p, stream);
-    case SKY_EPI_GELU_BWD:
-      return launch_variant<A_MN, B_MN, SKY_EPI_GELU_BWD, false>(grid, ta, tb, p, stream);
-    default:
-      return launch_variant<A_MN, B_MN, SKY_EPI_STORE, false>(grid, ta, tb, p, stream);
+  if constexpr (!PAIR) {
+    const int grid = units < sms ? units : sms;
+    kern<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
+    return cudaGetLastError();
+  } else {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(NUM_THREADS);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    static int max_clusters = [&] {
+      cudaLaunchConfig_t q = cfg;
+      q.gridDim = dim3(2 * (sms / 2));
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, kern, &q) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+      }
+      return n;
+    }();
+    if (max_clusters < 1) return cudaErrorLaunchOutOfResources;
+    const int clusters = units < max_clusters ? units : max_clusters;
+    cfg.gridDim = dim3(2 * clusters);
+    return cudaLaunchKernelEx(&cfg, kern, ta, tb, p);
   }
 }
+
+// One instantiation per (operand majorness, epilogue, output type, pairing)
+// keeps every kernel's code to the epilogue it runs.
+template <bool A_MN, bool B_MN, bool PAIR>
+cudaError_t launch_form(int units, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
+                        const Params& p, int epi, bool out_f32, cudaStream_t stream) {
+  if (out_f32)
+    return launch_variant<A_MN, B_MN, SKY_EPI_STORE, true, PAIR>(units, sms, ta, tb, p, stream);
+  switch (epi) {
+    case SKY_EPI_BIAS_GELU:
+      return launch_variant<A_MN, B_MN, SKY_EPI_BIAS_GELU, false, PAIR>(units, sms, ta, tb, p,
+                                                                        stream);
+    case SKY_EPI_GELU_BWD:
+      return launch_variant<A_MN, B_MN, SKY_EPI_GELU_BWD, false, PAIR>(units, sms, ta, tb, p,
+                                                                       stream);
+    default:
+      return launch_variant<A_MN, B_MN, SKY_EPI_STORE, false, PAIR>(units, sms, ta, tb, p, stream);
+  }
+}
+
+// The pair variant serves every problem with at least one full 256-row tile,
+// except the bias+GELU epilogue: that kernel is bound by its epilogue math,
+// and pairing makes each accumulator wait for the slower CTA's epilogue.
+bool use_pair(int M, int epi) { return M >= 2 * BM && epi != SKY_EPI_BIAS_GELU; }
 
 uint64_t g_timeout_ns = 2000000000ull;  // 2 s per wait
 int g_skip_loads = 0;
@@ -444,9 +542,11 @@ int choose_splits(int tiles, int k_blocks, int sms) {
 
 size_t workspace_bytes(sky_gemm_form form, int M, int N, int K, bool out_f32) {
   if (!out_f32) return 0;
-  const int tiles = ceil_div(M, BM) * ceil_div(N, BN);
+  const bool pair = use_pair(M, SKY_EPI_STORE);  // fp32 outputs use the STORE epilogue
+  const int tiles = ceil_div(M, pair ? 2 * BM : BM) * ceil_div(N, BN);
   const int kb = ceil_div(K, BK);
-  const int s = choose_splits(tiles, kb, sm_count() > 0 ? sm_count() : 148);
+  const int sms = sm_count() > 0 ? sm_count() : 148;
+  const int s = choose_splits(tiles, kb, pair ? sms / 2 : sms);
   (void)form;
   return s > 1 ? static_cast<size_t>(s) * M * N * sizeof(float) : 0;
 }
@@ -479,17 +579,18 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   CUtensorMap ta, tb;
   const bool a_mn = form == SKY_GEMM_XTW;
   const bool b_mn = form != SKY_GEMM_XWT;
+  const bool pair = use_pair(M, epi);
   bool ok = a_mn ? make_map(&ta, A, K, M, 64) : make_map(&ta, A, M, K, BM);
-  ok = ok && (b_mn ? make_map(&tb, B, K, N, 64) : make_map(&tb, B, N, K, BN));
+  ok = ok && (b_mn ? make_map(&tb, B, K, N, 64) : make_map(&tb, B, N, K, pair ? BN / 2 : BN));
   SKY_CHECK(ok, SKY_ERR_CUDA, "cuTensorMapEncodeTiled failed (M=%d N=%d K=%d)", M, N, K);
 
   Params p{};
   p.M = M; p.N = N; p.K = K;
-  p.m_tiles = ceil_div(M, BM);
+  p.m_tiles = ceil_div(M, pair ? 2 * BM : BM);
   p.n_tiles = ceil_div(N, BN);
   p.k_blocks = ceil_div(K, BK);
   const bool may_split = out_f32 && epi == SKY_EPI_STORE && bias == nullptr;
-  p.splits = may_split ? choose_splits(p.m_tiles * p.n_tiles, p.k_blocks, sms) : 1;
+  p.splits = may_split ? choose_splits(p.m_tiles * p.n_tiles, p.k_blocks, pair ? sms / 2 : sms) : 1;
   if (p.splits > 1) {  // never more partials than the workspace holds
     const size_t cap = ws_bytes / (static_cast<size_t>(M) * N * sizeof(float));
     p.splits = cap < 2 ? 1 : (p.splits < (int)cap ? p.splits : (int)cap);
@@ -502,7 +603,7 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   p.C = p.splits > 1 ? ws : C;
   // optional fused column sum of C (bf16 outputs only): per-warp partials in
   // the workspace, added in a fixed order after the kernel
-  const int colpart_rows = p.m_tiles * 4;
+  const int colpart_rows = p.m_tiles * (pair ? 8 : 4);  // one per 32 rows of every tile
   if (colsum) {
     SKY_CHECK(!out_f32 && p.splits == 1, SKY_ERR_UNSUPPORTED, "fused column sum needs a bf16 output");
     SKY_CHECK(ws && ws_bytes >= static_cast<size_t>(colpart_rows) * N * sizeof(float),
@@ -517,14 +618,22 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   p.skip_loads = g_skip_loads;
 
   const int units = p.m_tiles * p.n_tiles * p.splits;
-  const int grid = units < sms ? units : sms;
   cudaError_t e;
-  if (form == SKY_GEMM_XWT)
-    e = launch_form<false, false>(grid, ta, tb, p, epi, out_f32, stream);
-  else if (form == SKY_GEMM_XW)
-    e = launch_form<false, true>(grid, ta, tb, p, epi, out_f32, stream);
-  else
-    e = launch_form<true, true>(grid, ta, tb, p, epi, out_f32, stream);
+  if (pair) {
+    if (form == SKY_GEMM_XWT)
+      e = launch_form<false, false, true>(units, sms, ta, tb, p, epi, out_f32, stream);
+    else if (form == SKY_GEMM_XW)
+      e = launch_form<false, true, true>(units, sms, ta, tb, p, epi, out_f32, stream);
+    else
+      e = launch_form<true, true, true>(units, sms, ta, tb, p, epi, out_f32, stream);
+  } else {
+    if (form == SKY_GEMM_XWT)
+      e = launch_form<false, false, false>(units, sms, ta, tb, p, epi, out_f32, stream);
+    else if (form == SKY_GEMM_XW)
+      e = launch_form<false, true, false>(units, sms, ta, tb, p, epi, out_f32, stream);
+    else
+      e = launch_form<true, true, false>(units, sms, ta, tb, p, epi, out_f32, stream);
+  }
   count_launches(1);
   if (e != cudaSuccess) return cuda_fail(e, "gemm_tc_kernel launch");
   if (colsum) {
