@@ -9,11 +9,17 @@ namespace gemm {
 
 // bf16 inputs on tcgen05; C is bf16 unless out_f32.
 // colsum (optional, bf16 output, no split): also writes out[n] = sum_m C[m, n]
-// (before rounding), with fixed-order partials in `ws` (m_tiles*4 x N fp32).
+// (before rounding), with fixed-order partials (one row per 32 rows of C) in
+// `ws`.  With `deferred_rows`, the partials go to `colpart` instead, no sum is
+// launched and *deferred_rows reports their row count (for reduce_rows_f32,
+// possibly on another stream ordered after this launch).
 sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
-                       cudaStream_t stream, float* colsum = nullptr);
+                       cudaStream_t stream, float* colsum = nullptr, float* colpart = nullptr,
+                       size_t colpart_bytes = 0, int* deferred_rows = nullptr);
+// Rows of column partials a bf16 GEMM with M rows writes (upper bound).
+int colpart_rows_max(int M);
 // out[n] = sum over r of part[r][n] in order r = 0, 1, ... (rowwise.cu).
 cudaError_t reduce_rows_f32(const float* part, int rows, int N, float* out, cudaStream_t stream);
 size_t workspace_bytes(sky_gemm_form form, int M, int N, int K, bool out_f32);

@@ -525,6 +525,10 @@ void set_debug(uint64_t timeout_ns, int skip_loads) {
   g_skip_loads = skip_loads;
 }
 
+int colpart_rows_max(int M) {
+  return std::max(ceil_div(M, BM) * 4, ceil_div(M, 2 * BM) * 8);
+}
+
 int choose_splits(int tiles, int k_blocks, int sms) {
   // Estimated makespan (in k-block units) of `tiles * s` units on `sms` CTAs
   // plus a small per-unit cost; the fixed-order reduce is charged per split.
@@ -554,7 +558,8 @@ size_t workspace_bytes(sky_gemm_form form, int M, int N, int K, bool out_f32) {
 sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
-                       cudaStream_t stream, float* colsum) {
+                       cudaStream_t stream, float* colsum, float* colpart, size_t colpart_bytes,
+                       int* deferred_rows) {
   // TMA row pitches and the 16-byte epilogue stores need the contiguous
   // dimensions to be multiples of 8 elements; the token dimension is free.
   const bool dims_ok = N % 8 == 0 && (form == SKY_GEMM_XTW ? M % 8 == 0 : K % 8 == 0);
@@ -604,11 +609,14 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   // optional fused column sum of C (bf16 outputs only): per-warp partials in
   // the workspace, added in a fixed order after the kernel
   const int colpart_rows = p.m_tiles * (pair ? 8 : 4);  // one per 32 rows of every tile
-  if (colsum) {
+  if (colsum || deferred_rows) {
     SKY_CHECK(!out_f32 && p.splits == 1, SKY_ERR_UNSUPPORTED, "fused column sum needs a bf16 output");
-    SKY_CHECK(ws && ws_bytes >= static_cast<size_t>(colpart_rows) * N * sizeof(float),
+    float* buf = deferred_rows ? colpart : static_cast<float*>(ws);
+    const size_t cap = deferred_rows ? colpart_bytes : ws_bytes;
+    SKY_CHECK(buf && cap >= static_cast<size_t>(colpart_rows) * N * sizeof(float),
               SKY_ERR_INVALID_ARG, "GEMM column-sum workspace too small");
-    p.colpart = static_cast<float*>(ws);
+    p.colpart = buf;
+    if (deferred_rows) *deferred_rows = colpart_rows;
   }
   p.bias = static_cast<const __nv_bfloat16*>(bias);
   p.aux = epi == SKY_EPI_GELU_BWD ? static_cast<const __half*>(aux) : nullptr;
@@ -636,7 +644,7 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   }
   count_launches(1);
   if (e != cudaSuccess) return cuda_fail(e, "gemm_tc_kernel launch");
-  if (colsum) {
+  if (colsum && !deferred_rows) {
     e = reduce_rows_f32(p.colpart, colpart_rows, N, colsum, stream);
     if (e != cudaSuccess) return cuda_fail(e, "column-sum reduce launch");
   }

@@ -549,7 +549,8 @@ size_t layernorm_bwd_ws(int rows, int H) {
 sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, const float* u,
                          const void* gamma, const float* mean, const float* rstd, int rows, int H,
                          sky_dtype dt, float* du32, void* du, float* dgamma, float* dbeta,
-                         float* dbias, void* ws, size_t ws_bytes, cudaStream_t st) {
+                         float* dbias, void* ws, size_t ws_bytes, cudaStream_t st,
+                         int* deferred_parts) {
   SKY_CHECK(H % rw::V == 0 && lane_vectors(H) <= kMaxNV && (dt == SKY_DTYPE_BF16 || H <= 1024),
             SKY_ERR_UNSUPPORTED, "LayerNorm width %d unsupported", H);
   SKY_CHECK(du32 || du, SKY_ERR_INVALID_ARG, "LayerNorm backward needs an output");
@@ -580,11 +581,14 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
           static_cast<const float*>(dy), dy2, u, static_cast<const __nv_bfloat16*>(gamma), mean,
           rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, nullptr);
     }
-    dim3 grid(ceil_div(H, 32), 3);
-    rw::reduce_partials<<<grid, 256, 0, st>>>(part, sb, H, dgamma, dbeta, dbias);
-    count_launches(2);
+    count_launches(1);
     const cudaError_t e = cudaGetLastError();
-    return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward launch");
+    if (e != cudaSuccess) return cuda_fail(e, "layernorm backward launch");
+    if (deferred_parts) {
+      *deferred_parts = sb;
+      return SKY_OK;
+    }
+    return layernorm_bwd_reduce(part, sb, H, dgamma, dbeta, dbias, st);
   }
   if (dt == SKY_DTYPE_BF16) {
     if (dy_dt == SKY_DTYPE_BF16) {
@@ -604,11 +608,24 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
     if (du32 && du && du != du32)
       SKY_CUDA(cudaMemcpyAsync(du, du32, (size_t)rows * H * 4, cudaMemcpyDeviceToDevice, st));
   }
-  dim3 grid(ceil_div(H, 32), 3);
-  rw::reduce_partials<<<grid, 256, 0, st>>>(part, nblk, H, dgamma, dbeta, dbias);
-  count_launches(2);
+  count_launches(1);
   const cudaError_t e = cudaGetLastError();
-  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward launch");
+  if (e != cudaSuccess) return cuda_fail(e, "layernorm backward launch");
+  if (deferred_parts) {
+    *deferred_parts = nblk;
+    return SKY_OK;
+  }
+  return layernorm_bwd_reduce(part, nblk, H, dgamma, dbeta, dbias, st);
+}
+
+sky_status layernorm_bwd_reduce(const void* ws, int parts, int H, float* dgamma, float* dbeta,
+                                float* dbias, cudaStream_t st) {
+  dim3 grid(ceil_div(H, 32), 3);
+  rw::reduce_partials<<<grid, 256, 0, st>>>(static_cast<const float*>(ws), parts, H, dgamma,
+                                            dbeta, dbias);
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward reduce launch");
 }
 
 namespace gemm {

@@ -20,7 +20,13 @@ size_t layernorm_bwd_ws(int rows, int H);
 sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, const float* u,
                          const void* gamma, const float* mean, const float* rstd, int rows, int H,
                          sky_dtype dt, float* du32, void* du, float* dgamma, float* dbeta,
-                         float* dbias, void* ws, size_t ws_bytes, cudaStream_t st);
+                         float* dbias, void* ws, size_t ws_bytes, cudaStream_t st,
+                         int* deferred_parts = nullptr);
+// With `deferred_parts`, layernorm_bwd leaves dgamma / dbeta / dbias as
+// per-CTA partials in `ws` (*deferred_parts rows each) and this call, possibly
+// on another stream ordered after it, adds them in a fixed order.
+sky_status layernorm_bwd_reduce(const void* ws, int parts, int H, float* dgamma, float* dbeta,
+                                float* dbias, cudaStream_t st);
 sky_status add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dt, void* out,
                    cudaStream_t st);
 sky_status f32_to_bf16(const float* x, int64_t n, void* out, cudaStream_t st);

@@ -111,6 +111,13 @@ struct sky_slice {
   cudaEvent_t ev_in[4] = {}, ev_out[4] = {}, ev_join = nullptr;
   void* ws2 = nullptr;
   size_t ws2_bytes = 0;
+  // Column partials whose fixed-order reduction (a bias / LayerNorm-parameter
+  // gradient, needed by nothing downstream) also runs on the side stream:
+  // lnp[0] / lnp[1] of the LN2 / LN1 backward, db1p of the fused db1.
+  void* lnp[2] = {nullptr, nullptr};
+  size_t lnp_bytes = 0;
+  float* db1p = nullptr;
+  size_t db1p_bytes = 0;
   // state of the most recent forward
   bool have_fwd = false;
   int B = 0, S = 0;
@@ -165,7 +172,7 @@ size_t workspace_need(const sky_slice* s, int64_t T) {
 // beside the main stream's kernels).
 size_t side_workspace_need(const sky_slice* s, int64_t T) {
   const int H = s->H, F = s->F;
-  size_t need = 0;
+  size_t need = column_sum_ws((int)T, 3 * H);  // dbqkv
   const int64_t shapes[4][2] = {{3 * H, H}, {H, H}, {F, H}, {H, F}};
   for (auto& sh : shapes)
     need = std::max(need, gemm::workspace_bytes(SKY_GEMM_XTW, (int)sh[0], (int)sh[1], (int)T, true));
@@ -309,28 +316,47 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   };
   void* ws2 = bf ? s->ws2 : nullptr;
   const size_t ws2b = s->ws2_bytes;
+  // bf16: the column-sum reductions of this layer's bias / LayerNorm-parameter
+  // gradients run on sw too, from partials in buffers of their own
+  int ln_parts = 0, db1_rows = 0;
+  auto ln_reduce = [&](int j, float* dg, float* db, float* dbias) -> sky_status {
+    Timed t(s, sw, P_COLSUM, 0, 3.0 * ln_parts * H * 4.0);
+    return layernorm_bwd_reduce(s->lnp[j], ln_parts, H, dg, db, dbias, sw);
+  };
   // a9: LN2 backward -> dU2 (fp32 + dtype), dgamma2, dbeta2, db2
   SKY_TRY(reuse(0));
   {
     Timed t(s, st, P_LN_BWD, 0, (dye + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(dY, dy_dt, dY2, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
-                          bf ? s->dU2_32 : nullptr, s->dU2b, Lb.g[10], Lb.g[11], Lb.g[9], s->ws,
-                          s->ws_bytes, st));
+                          bf ? s->dU2_32 : nullptr, s->dU2b, Lb.g[10], Lb.g[11], Lb.g[9],
+                          bf ? s->lnp[0] : s->ws, bf ? s->lnp_bytes : s->ws_bytes, st,
+                          bf ? &ln_parts : nullptr));
   }
   SKY_TRY(fork(0));
+  if (bf) SKY_TRY(ln_reduce(0, Lb.g[10], Lb.g[11], Lb.g[9]));
+  // a10 + a11: dW2 = dU2^T G (on sw, beside the data gradient);
+  //            dZ = (dU2 W2) * GELU'(Z);
+  //            db1 = sum_rows dZ (fused into the bf16 epilogue; a column-sum pass for fp32)
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
+  SKY_TRY(done(0));
   SKY_TRY(reuse(1));
-  // a10 + a11: dZ = (dU2 W2) * GELU'(Z);  dW2 = dU2^T G
-  //          db1 = sum_rows dZ (fused into the bf16 epilogue; a column-sum pass for fp32)
-  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
-                   SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr, bf ? Lb.g[7] : nullptr));
-  if (!bf) {
+  if (bf) {
+    Timed t(s, st, P_GEMM_DGRAD, 2.0 * T * F * H, 0);
+    SKY_TRY(gemm::launch_bf16(SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
+                              SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr, s->ws, s->ws_bytes,
+                              s->d_status, st, nullptr, s->db1p, s->db1p_bytes, &db1_rows));
+  } else {
+    SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
+                     SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr));
     Timed t(s, st, P_COLSUM, 0, e * T * F);
     SKY_TRY(column_sum(s->dH, T, F, dt, Lb.g[7], s->ws, s->ws_bytes, st));
   }
   SKY_TRY(fork(1));
-  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
-  SKY_TRY(done(0));
+  if (bf) {  // db1 = sum of the fused partials
+    Timed t(s, sw, P_COLSUM, 0, 4.0 * db1_rows * F);
+    SKY_CUDA(gemm::reduce_rows_f32(s->db1p, db1_rows, F, Lb.g[7], sw));
+  }
   // a12: P1 = dZ W1 (fp32; dX1 = P1 + dU2 is formed by the LN1 backward);  dW1 = dZ^T X1
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dP1, true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
@@ -343,9 +369,11 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, st, P_LN_BWD, 0, (4.0 + 4.0 + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? s->dU2_32 : static_cast<float*>(s->dU2b),
                           Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H, dt, bf ? s->dR[k] : nullptr,
-                          dU1b, Lb.g[4], Lb.g[5], Lb.g[3], s->ws, s->ws_bytes, st));
+                          dU1b, Lb.g[4], Lb.g[5], Lb.g[3], bf ? s->lnp[1] : s->ws,
+                          bf ? s->lnp_bytes : s->ws_bytes, st, bf ? &ln_parts : nullptr));
   }
   SKY_TRY(fork(2));
+  if (bf) SKY_TRY(ln_reduce(1, Lb.g[4], Lb.g[5], Lb.g[3]));
   // a14: dctx = dU1 Wo;  dWo = dU1^T ctx
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, H, dU1b, Lb.p[2], s->dctx, false,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
@@ -359,11 +387,12 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     SKY_TRY(attention_bwd(Lb.QKV, Lb.ctx, s->dctx, Lb.lse, s->d_len, B, S, H, A, dt, s->dqkv,
                           s->delta, s->d_status, st));
   }
-  {
-    Timed t(s, st, P_COLSUM, 0, e * T * 3.0 * H);
-    SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], s->ws, s->ws_bytes, st));
-  }
   SKY_TRY(fork(3));
+  {  // dbqkv = column sums of dQKV (on sw for bf16, with sw's scratch)
+    Timed t(s, sw, P_COLSUM, 0, e * T * 3.0 * H);
+    SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], bf ? s->ws2 : s->ws,
+                       bf ? s->ws2_bytes : s->ws_bytes, sw));
+  }
   // a16: dX = dQKV Wqkv + dU1 (the sum is formed by the next LayerNorm backward,
   // or here for the slice's first layer);  dWqkv = dQKV^T X
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, 3 * H, s->dqkv, Lb.p[0], s->dP[k], true,
@@ -531,10 +560,13 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   s->stash_bytes = stash * s->L;
   s->ws_bytes = align_up(workspace_need(s, T));
   s->ws2_bytes = bf ? align_up(side_workspace_need(s, T)) : 0;
-  // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | ws2 | status
+  s->lnp_bytes = bf ? align_up(layernorm_bwd_ws((int)T, s->H)) : 0;
+  s->db1p_bytes = bf ? align_up((size_t)gemm::colpart_rows_max((int)T) * s->F * 4) : 0;
+  // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | ws2 | lnp[2] |
+  // db1p | status
   const size_t wk = 6 * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
                     align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes +
-                    s->ws2_bytes + 256;
+                    s->ws2_bytes + 2 * s->lnp_bytes + s->db1p_bytes + 256;
   s->ws_bytes_total = wk;
   *total = s->param_bytes + s->grad_bytes + s->stash_bytes + wk;
   return SKY_OK;
@@ -641,6 +673,11 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   s->delta = static_cast<float*>(take(lse_b));
   s->ws = take(s->ws_bytes);
   if (s->ws2_bytes) s->ws2 = take(s->ws2_bytes);
+  if (s->lnp_bytes) {
+    s->lnp[0] = take(s->lnp_bytes);
+    s->lnp[1] = take(s->lnp_bytes);
+  }
+  if (s->db1p_bytes) s->db1p = static_cast<float*>(take(s->db1p_bytes));
   s->d_status = static_cast<int32_t*>(take(4));
   if (bf) {
     // the weight-gradient side stream and its events
