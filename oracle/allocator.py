@@ -33,17 +33,29 @@ Readings of the paper where it is silent or inconsistent:
 4. Alg. 2 recomputes device workloads from the current ``pi`` at every test
    (a move at boundary ``i`` is visible when boundary ``i+1`` is examined);
    the target (mean workload over all D devices) is computed once per sweep;
-   "memory satisfied after change" means both devices touched by the move
-   stay within their memory.
+   "memory satisfied after change" means every device is within its memory
+   after the move (only the two devices it touches can change).
 5. Alg. 2 stops after a sweep that changes nothing, or after ``max_iter``
    sweeps.  (Its inner test ``counter == max_iter`` can never hold inside
    ``while counter < max_iter``; the loop bound is what limits the sweeps.)
 6. The MILP leaves device order free and lets a device hold no layer (an
    empty device still contributes ``ct_i`` to ``q``, as the constraint reads).
+7. Every sum (a device's memory or workload, the total workload) is
+   accumulated left to right in index order (``_sum``), so the comparisons
+   that decide a move round the same way wherever they are evaluated
+   (Python's built-in ``sum`` compensates rounding from 3.12 on).
 """
 from __future__ import annotations
 
 import itertools
+
+
+def _sum(values) -> float:
+    """Plain left-to-right accumulation (reading 7)."""
+    s = 0.0
+    for v in values:
+        s += v
+    return s
 
 
 def even_partition(L: int, D: int) -> list:
@@ -63,7 +75,7 @@ def num_layers(pi: list, i: int) -> int:
 
 def allocated_memory(lm: list, pi: list) -> list:
     """``am[i]``: memory of the layers device ``i`` holds (Alg. 1)."""
-    return [sum(lm[pi[i]:pi[i + 1]]) for i in range(len(pi) - 1)]
+    return [_sum(lm[pi[i]:pi[i + 1]]) for i in range(len(pi) - 1)]
 
 
 def memory_satisfied(dm: list, lm: list, pi: list) -> bool:
@@ -105,7 +117,7 @@ def layer_workload(dt: list, lf: list, ct: list, i: int, j: int) -> float:
 
 def device_workload(dt: list, lf: list, ct: list, pi: list, i: int) -> float:
     """Sum of the layer workloads of device ``i`` (reading 1)."""
-    return sum(layer_workload(dt, lf, ct, i, j) for j in range(pi[i], pi[i + 1]))
+    return _sum(layer_workload(dt, lf, ct, i, j) for j in range(pi[i], pi[i + 1]))
 
 
 def finetune(dt: list, dm: list, ct: list, lf: list, lm: list, pi: list, max_iter: int) -> list:
@@ -121,7 +133,7 @@ def finetune(dt: list, dm: list, ct: list, lf: list, lm: list, pi: list, max_ite
     pi = list(pi)
     counter = 0
     while counter < max_iter:
-        target = sum(device_workload(dt, lf, ct, pi, i) for i in range(D)) / D
+        target = _sum(device_workload(dt, lf, ct, pi, i) for i in range(D)) / D
         before = list(pi)
         for i in range(D - 1):
             w_this = device_workload(dt, lf, ct, pi, i)
@@ -152,7 +164,7 @@ def milp_objective(dt: list, ct: list, lf: list, owner: list) -> float:
     """``q = max_i (dt_i * sum_j x_ij lf_j + ct_i)`` of Sec. IV-C for the
     assignment ``owner[j] = i`` (``x_ij = 1``)."""
     D = len(dt)
-    return max(dt[i] * sum(lf[j] for j in range(len(lf)) if owner[j] == i) + ct[i]
+    return max(dt[i] * _sum(lf[j] for j in range(len(lf)) if owner[j] == i) + ct[i]
                for i in range(D))
 
 
@@ -177,7 +189,7 @@ def milp_brute_force(dt: list, dm: list, ct: list, lf: list, lm: list):
             if idx and idx[-1] - idx[0] != len(idx) - 1:
                 ok = False
                 break
-            if sum(lm[j] for j in idx) > dm[i]:
+            if _sum(lm[j] for j in idx) > dm[i]:
                 ok = False
                 break
         if not ok:
