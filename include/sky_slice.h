@@ -50,7 +50,8 @@ typedef enum {
   SKY_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed            */
   SKY_ERR_STATE = 4,        /* e.g. backward without a matching forward     */
   SKY_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up           */
-  SKY_ERR_UNSUPPORTED = 6   /* valid but not implemented (e.g. D != 64 bf16)*/
+  SKY_ERR_UNSUPPORTED = 6,  /* valid but not implemented (e.g. D != 64 bf16)*/
+  SKY_ERR_INFEASIBLE = 7    /* allocator: no partition fits the memory limits */
 } sky_status;
 
 typedef enum { SKY_DTYPE_BF16 = 0, SKY_DTYPE_FP32 = 1 } sky_dtype;

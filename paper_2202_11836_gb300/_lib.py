@@ -14,7 +14,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(PKG, "libsky_slice.so")
 
 SKY_OK, SKY_ERR_INVALID_ARG, SKY_ERR_OOM, SKY_ERR_CUDA, SKY_ERR_STATE, SKY_ERR_TIMEOUT, \
-    SKY_ERR_UNSUPPORTED = range(7)
+    SKY_ERR_UNSUPPORTED, SKY_ERR_INFEASIBLE = range(8)
 SKY_DTYPE_BF16, SKY_DTYPE_FP32 = 0, 1
 SKY_GEMM_XWT, SKY_GEMM_XW, SKY_GEMM_XTW = 0, 1, 2
 SKY_EPI_STORE, SKY_EPI_BIAS_GELU, SKY_EPI_GELU_BWD = 0, 1, 2
@@ -50,7 +50,16 @@ class SkyError(RuntimeError):
 STATUS_NAMES = {SKY_OK: "SKY_OK", SKY_ERR_INVALID_ARG: "SKY_ERR_INVALID_ARG",
                 SKY_ERR_OOM: "SKY_ERR_OOM", SKY_ERR_CUDA: "SKY_ERR_CUDA",
                 SKY_ERR_STATE: "SKY_ERR_STATE", SKY_ERR_TIMEOUT: "SKY_ERR_TIMEOUT",
-                SKY_ERR_UNSUPPORTED: "SKY_ERR_UNSUPPORTED"}
+                SKY_ERR_UNSUPPORTED: "SKY_ERR_UNSUPPORTED", SKY_ERR_INFEASIBLE: "SKY_ERR_INFEASIBLE"}
+
+class SkyAllocProblem(C.Structure):
+    _fields_ = [("devices", C.c_int32), ("layers", C.c_int32),
+                ("dt", C.POINTER(C.c_double)), ("dm", C.POINTER(C.c_double)),
+                ("ct", C.POINTER(C.c_double)), ("lf", C.POINTER(C.c_double)),
+                ("lm", C.POINTER(C.c_double))]
+
+
+SKY_COST_CT_PER_DEVICE, SKY_COST_CT_PER_LAYER = 0, 1
 
 _VP, _I32, _SZ = C.c_void_p, C.c_int32, C.c_size_t
 _SIGNATURES = {
@@ -92,6 +101,17 @@ _SIGNATURES = {
     "sky_column_sum_noalloc": (C.c_int, [_VP, _I32, _I32, C.c_int, _VP, _VP]),
     "sky_debug_gemm_fault": (None, [C.c_uint64, C.c_int32]),
     "sky_device_sm_count": (_I32, []),
+    "sky_alloc_even": (C.c_int, [_I32, _I32, C.POINTER(_I32)]),
+    "sky_alloc_coarse": (C.c_int, [C.POINTER(SkyAllocProblem), C.POINTER(_I32)]),
+    "sky_alloc_finetune": (C.c_int, [C.POINTER(SkyAllocProblem), _I32, C.POINTER(_I32),
+                                     C.POINTER(_I32)]),
+    "sky_alloc_heuristic": (C.c_int, [C.POINTER(SkyAllocProblem), _I32, C.POINTER(_I32)]),
+    "sky_alloc_workloads": (C.c_int, [C.POINTER(SkyAllocProblem), C.POINTER(_I32), C.c_int,
+                                      C.POINTER(C.c_double)]),
+    "sky_alloc_best_ordered": (C.c_int, [C.POINTER(SkyAllocProblem), C.POINTER(_I32),
+                                         C.POINTER(C.c_double)]),
+    "sky_alloc_milp_exact": (C.c_int, [C.POINTER(SkyAllocProblem), C.POINTER(_I32),
+                                       C.POINTER(C.c_double)]),
 }
 
 _lib = None

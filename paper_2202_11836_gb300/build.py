@@ -1,6 +1,7 @@
 """Builds libsky_slice.so (the C-ABI library) in-tree with nvcc for sm_103a.
 
-Each translation unit under ``csrc/`` compiles in parallel into ``_build/``;
+Each translation unit under ``csrc/`` (CUDA ``.cu`` and host-only ``.cpp``)
+compiles in parallel into ``_build/``;
 the objects link into ``libsky_slice.so`` next to this file.  A source whose
 object is newer than it (and than every header) is not recompiled.
 """
@@ -18,8 +19,11 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsky_slice.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+# Host code is compiled without floating-point contraction, so the allocator's
+# sums and comparisons round the same way on every host architecture.
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
-         "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]
+         "-Xcompiler", "-ffp-contract=off", "--expt-relaxed-constexpr",
+         "-I", os.path.join(ROOT, "include")]
 
 
 def nvcc() -> str:
@@ -53,7 +57,7 @@ def _compile(src: str, extra: list, verbose: bool) -> str:
 def build(verbose: bool = False, extra: list | None = None) -> str:
     """Compiles every csrc/*.cu and links libsky_slice.so; returns its path."""
     os.makedirs(BUILD, exist_ok=True)
-    srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
+    srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")) + glob.glob(os.path.join(CSRC, "*.cpp")))
     extra = list(extra or [])
     with cf.ThreadPoolExecutor(max_workers=min(8, len(srcs))) as ex:
         objs = list(ex.map(lambda s: _compile(s, extra, verbose), srcs))

@@ -525,6 +525,7 @@ const char* sky_status_string(sky_status st) {
     case SKY_ERR_STATE: return "SKY_ERR_STATE";
     case SKY_ERR_TIMEOUT: return "SKY_ERR_TIMEOUT";
     case SKY_ERR_UNSUPPORTED: return "SKY_ERR_UNSUPPORTED";
+    case SKY_ERR_INFEASIBLE: return "SKY_ERR_INFEASIBLE";
   }
   return "SKY_ERR_UNKNOWN";
 }
