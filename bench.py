@@ -70,6 +70,38 @@ def gemm_traffic(workload):
     return GEMM_TRAFFIC["bytes_per_launch"]
 
 
+def allocation_plan(rec, layers=160, devices=64, seed=2022):
+    """The paper's allocator on the measured layer costs (Sec. IV).
+
+    The layer table is the median per-layer cost of the benchmark slice
+    (time of fwd + bwd on this GPU, parameter + gradient + stash bytes),
+    repeated for a 160-layer model; the device table has 64 devices whose time
+    ratios are drawn like the paper's slow-down factors (normal, clipped to
+    [1, 7]) and whose memory holds 1.5 to 4 times an even share.  Reports the
+    predicted per-step makespan (slowest device, ms) of the even split, the
+    heuristic (Alg. 1 + Alg. 2) and the exact best partition in device order,
+    and the C++ heuristic's run time."""
+    import random
+    from paper_2202_11836_gb300 import allocator
+    t_layer = statistics.median([r["fwd_ms"] + r["bwd_ms"] for r in rec])
+    m_layer = float(statistics.median([r["param_bytes"] + r["grad_bytes"] + r["stash_bytes"]
+                                       for r in rec]))
+    rng = random.Random(seed)
+    dt = [min(7.0, max(1.0, rng.gauss(4.0, 1.5))) for _ in range(devices)]
+    share = m_layer * layers / devices
+    dm = [rng.uniform(1.5, 4.0) * share for _ in range(devices)]
+    P = allocator.Problem(dt, dm, [0.0] * devices, [t_layer] * layers, [m_layer] * layers)
+    t0 = time.perf_counter()
+    pi = P.heuristic(100)
+    t_heur = (time.perf_counter() - t0) * 1e3
+    _, q_best = P.best_ordered()
+    return {"layers": layers, "devices": devices, "layer_ms": round(t_layer, 4),
+            "makespan_ms": {"even": round(P.makespan(allocator.even(layers, devices)), 3),
+                            "heuristic": round(P.makespan(pi), 3),
+                            "best_in_device_order": round(q_best, 3)},
+            "heuristic_run_ms": round(t_heur, 3)}
+
+
 def algorithmic_flops(w, lens):
     """Matmul FLOPs of one step (forward + backward) over all layers."""
     T, H, F, S = w.batch * w.seq, w.hidden, w.ffn, w.seq
@@ -354,6 +386,7 @@ def run_gpu(args, w):
             "pct_bf16_peak_end_to_end": round(100 * total_f / (ms_step / 1e3) / 1e12 / pk["bf16"], 2),
             "tokens_per_s_per_layer": tokens / (per_layer_ms / 1e3),
             "per_layer_ms": per_layer_ms,
+            "allocation": allocation_plan(rec),
             "valid_tokens_per_s": world * int(np.sum(lens)) * args.steps / (ms / 1e3),
             "roofline": {"kernel": "gemm_tc_kernel (all GEMM launches of the step)",
                          "bound": "tensor", "achieved": round(achieved, 1),

@@ -24,7 +24,9 @@ def lib():
 
 def declared_functions():
     names = set()
-    for h in ("sky_slice.h", "sky_ops.h"):
+    for h in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if not h.endswith(".h"):
+            continue
         src = open(os.path.join(ROOT, "include", h)).read()
         src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
         names |= set(re.findall(r"\b(sky_\w+)\s*\(", src))

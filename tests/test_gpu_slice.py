@@ -198,3 +198,27 @@ def test_layer_cost_and_linearity():
     pred = alpha + beta * n
     r2 = 1 - ((t - pred) ** 2).sum() / ((t - t.mean()) ** 2).sum()
     assert r2 >= 0.99, (times, r2)
+
+
+def test_layer_cost_feeds_allocator():
+    """The per-layer records of sky_slice_layer_cost are the model benchmark
+    of Sec. IV-B: their time and bytes form the allocator's layer table, and
+    a slow device gets fewer layers than a fast one."""
+    from paper_2202_11836_gb300 import allocator
+    from paper_2202_11836_gb300.slice import EncoderSlice
+    w = synth.WORKLOADS["base-s128-b16"]
+    lb, le = 0, 6
+    with EncoderSlice(w.hidden, w.heads, w.ffn, lb, le, w.batch, w.seq) as s:
+        for l in range(lb, le):
+            s.set_params(l, synth.layer_params(l, w.hidden, w.ffn, "bf16"))
+        rec = s.layer_cost(w.batch, w.seq, iters=3)
+    lf, lm = allocator.layer_table(rec)
+    assert all(f > 0 for f in lf) and all(m > 0 for m in lm)
+    t = [r["fwd_ms"] + r["bwd_ms"] for r in rec]
+    # three devices, the middle one three times slower; memory for 4 layers each
+    P = allocator.Problem([1.0, 3.0, 1.0], [4 * max(lm)] * 3, [0.0] * 3, t, lm)
+    pi = P.heuristic()
+    counts = [pi[i + 1] - pi[i] for i in range(3)]
+    assert pi[0] == 0 and pi[-1] == le - lb and min(counts) >= 1
+    assert counts[1] <= min(counts[0], counts[2])
+    assert P.makespan(pi) <= P.makespan(allocator.even(le - lb, 3))
