@@ -348,6 +348,27 @@ def run_gpu(args, w):
     rec = s.layer_cost(w.batch, w.seq, iters=5)
     per_layer_ms = statistics.median([r["fwd_ms"] + r["bwd_ms"] for r in rec])
 
+    # 3b. the local parameter update (Sec. III), timed on its own: AdamW over
+    # every parameter of the slice, an HBM stream of 30 bytes per parameter
+    s.optimizer_init("adamw", lr=2e-5, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01)
+    n_params = sum(int(np.prod(v)) for v in s.shapes().values()) * w.layers
+    for _ in range(3):
+        s.optimizer_step(2e-5, stream)
+    sync()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    n_upd = 10
+    t0.record(stream)
+    for _ in range(n_upd):
+        s.optimizer_step(2e-5, stream)
+    t1.record(stream)
+    t1.synchronize()
+    upd_ms = t0.elapsed_time(t1) / n_upd
+    upd_gbs = 30.0 * n_params / (upd_ms / 1e3) / 1e9
+    optimizer = {"kind": "adamw", "params": n_params, "ms": round(upd_ms, 4),
+                 "bytes_per_param": 30, "achieved_gbs": round(upd_gbs, 1),
+                 "peak_gbs": pk["hbm"], "frac": round(upd_gbs / pk["hbm"], 4)}
+
     # 4. end to end through the public API with host buffers
     xh = torch.from_numpy(X).to(tdt).pin_memory()
     dyh = torch.from_numpy(dY).to(tdt).pin_memory()
@@ -387,6 +408,7 @@ def run_gpu(args, w):
             "tokens_per_s_per_layer": tokens / (per_layer_ms / 1e3),
             "per_layer_ms": per_layer_ms,
             "allocation": allocation_plan(rec),
+            "optimizer": optimizer,
             "valid_tokens_per_s": world * int(np.sum(lens)) * args.steps / (ms / 1e3),
             "roofline": {"kernel": "gemm_tc_kernel (all GEMM launches of the step)",
                          "bound": "tensor", "achieved": round(achieved, 1),

@@ -174,6 +174,48 @@ sky_status sky_slice_kernel_stats(sky_slice* s, sky_kernel_stat* out, int32_t n_
 sky_status sky_slice_memory(const sky_slice* s, uint64_t* param_bytes, uint64_t* grad_bytes,
                             uint64_t* stash_bytes, uint64_t* workspace_bytes);
 
+/* ---- Local parameter update (Sec. III) ------------------------------------
+ * After its backward pass a device updates the weights of its own layers with
+ * the gradients it computed (Sec. III); nothing is sent anywhere.  The paper
+ * names no optimizer; two rules are provided:
+ *   ADAMW: Adam with bias-corrected moments and decoupled weight decay
+ *          (w <- w - lr wd w; w <- w - lr m_hat / (sqrt(v_hat) + eps)),
+ *   SGD:   heavy-ball momentum with the decay added to the gradient
+ *          (b <- momentum b + g + wd w; w <- w - lr b).
+ * Weight decay applies to Wqkv, Wo, W1 and W2 only (BERT's choice), not to
+ * biases or LayerNorm parameters.  Updates run on fp32 master weights; a bf16
+ * slice's parameters are the master weights rounded to nearest bf16 after
+ * every step. */
+typedef enum { SKY_OPT_SGD = 0, SKY_OPT_ADAMW = 1 } sky_optimizer_kind;
+typedef struct {
+  int32_t kind;        /* sky_optimizer_kind                         */
+  float lr;            /* learning rate (sky_slice_optimizer_step may override) */
+  float beta1, beta2;  /* ADAMW moment decay rates, in [0, 1)        */
+  float eps;           /* ADAMW denominator term, > 0                */
+  float weight_decay;  /* >= 0                                       */
+  float momentum;      /* SGD, in [0, 1)                             */
+} sky_optimizer_config;
+
+/* Allocates the fp32 master weights (copied from the current parameters) and
+ * zeroed optimizer state (AdamW: 2, SGD: 1 fp32 copy of every parameter; a
+ * bf16 slice also keeps the master copy) and resets the step count.  Calling
+ * it again re-initialises.  Synchronises the device; the memory is freed by
+ * sky_slice_destroy.  Errors: INVALID_ARG for a bad config, OOM, UNSUPPORTED
+ * when a parameter tensor's size is not a multiple of 4. */
+sky_status sky_slice_optimizer_init(sky_slice* s, const sky_optimizer_config* cfg);
+
+/* One update of every parameter from the gradients of the most recent
+ * sky_slice_backward, with learning rate `lr` (a schedule is the caller's),
+ * enqueued on `stream`.  The slice's parameters are rewritten.  STATE if the
+ * optimizer is not initialised. */
+sky_status sky_slice_optimizer_step(sky_slice* s, float lr, void* stream);
+
+/* Host copies of one layer's fp32 optimizer tensors, 12 in parameter order:
+ * which = 0 master weights, 1 first state (AdamW m, SGD momentum),
+ * 2 second state (AdamW v).  Synchronises. */
+sky_status sky_slice_get_optimizer_state(sky_slice* s, int32_t layer, int32_t which,
+                                         void* const* dst);
+
 /* Host-side cap (bytes) on what sky_slice_create may allocate; 0 = no cap.
  * Lets the out-of-memory path be tested without exhausting a device. */
 void sky_debug_set_alloc_cap(uint64_t bytes);

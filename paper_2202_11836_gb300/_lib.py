@@ -60,6 +60,13 @@ class SkyAllocProblem(C.Structure):
 
 
 SKY_COST_CT_PER_DEVICE, SKY_COST_CT_PER_LAYER = 0, 1
+SKY_OPT_SGD, SKY_OPT_ADAMW = 0, 1
+
+
+class SkyOptimizerConfig(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("lr", C.c_float), ("beta1", C.c_float),
+                ("beta2", C.c_float), ("eps", C.c_float), ("weight_decay", C.c_float),
+                ("momentum", C.c_float)]
 
 _VP, _I32, _SZ = C.c_void_p, C.c_int32, C.c_size_t
 _SIGNATURES = {
@@ -101,6 +108,9 @@ _SIGNATURES = {
     "sky_column_sum_noalloc": (C.c_int, [_VP, _I32, _I32, C.c_int, _VP, _VP]),
     "sky_debug_gemm_fault": (None, [C.c_uint64, C.c_int32]),
     "sky_device_sm_count": (_I32, []),
+    "sky_slice_optimizer_init": (C.c_int, [_VP, C.POINTER(SkyOptimizerConfig)]),
+    "sky_slice_optimizer_step": (C.c_int, [_VP, C.c_float, _VP]),
+    "sky_slice_get_optimizer_state": (C.c_int, [_VP, _I32, _I32, C.POINTER(_VP)]),
     "sky_alloc_even": (C.c_int, [_I32, _I32, C.POINTER(_I32)]),
     "sky_alloc_coarse": (C.c_int, [C.POINTER(SkyAllocProblem), C.POINTER(_I32)]),
     "sky_alloc_finetune": (C.c_int, [C.POINTER(SkyAllocProblem), _I32, C.POINTER(_I32),

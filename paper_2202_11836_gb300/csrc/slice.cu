@@ -11,6 +11,7 @@
 // calls documented as synchronous.
 #include <algorithm>
 #include <atomic>
+#include <cmath>
 #include <cstdarg>
 #include <cstring>
 #include <exception>
@@ -20,6 +21,7 @@
 
 #include "common.cuh"
 #include "gemm.h"
+#include "optimizer.h"
 #include "rowwise.h"
 
 namespace sky {
@@ -118,6 +120,16 @@ struct sky_slice {
   size_t lnp_bytes = 0;
   float* db1p = nullptr;
   size_t db1p_bytes = 0;
+  // local parameter update (Sec. III): fp32 master weights and state in one
+  // allocation, the tensor and chunk tables the update kernel walks
+  bool opt_ready = false;
+  sky_optimizer_config opt_cfg{};
+  int64_t opt_t = 0;
+  void* opt_mem = nullptr;
+  std::vector<sky::opt::Tensor> opt_tensors;
+  sky::opt::Tensor* d_opt_tensors = nullptr;
+  sky::opt::Chunk* d_opt_chunks = nullptr;
+  int opt_chunks = 0;
   // state of the most recent forward
   bool have_fwd = false;
   int B = 0, S = 0;
@@ -709,6 +721,7 @@ sky_status sky_slice_destroy(sky_slice* s) {
   }
   if (s->ev_join) cudaEventDestroy(s->ev_join);
   if (s->side) cudaStreamDestroy(s->side);
+  if (s->opt_mem) cudaFree(s->opt_mem);
   if (s->arena) cudaFree(s->arena);
   delete s;
   return SKY_OK;
@@ -901,6 +914,149 @@ sky_status sky_slice_set_profiling(sky_slice* s, int enable) {
   for (int k = 0; k < P_NCAT; ++k) {
     s->cat_ms[k] = s->cat_flops[k] = s->cat_bytes[k] = 0;
     s->cat_n[k] = 0;
+  }
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_optimizer_init(sky_slice* s, const sky_optimizer_config* cfg) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s && cfg, SKY_ERR_INVALID_ARG, "null argument");
+  const sky_optimizer_config c = *cfg;
+  SKY_CHECK(c.kind == SKY_OPT_SGD || c.kind == SKY_OPT_ADAMW, SKY_ERR_INVALID_ARG,
+            "unknown optimizer kind %d", c.kind);
+  SKY_CHECK(c.lr >= 0.f && c.weight_decay >= 0.f, SKY_ERR_INVALID_ARG, "lr and weight_decay must be >= 0");
+  SKY_CHECK(c.kind != SKY_OPT_ADAMW || (c.beta1 >= 0.f && c.beta1 < 1.f && c.beta2 >= 0.f &&
+                                        c.beta2 < 1.f && c.eps > 0.f),
+            SKY_ERR_INVALID_ARG, "AdamW needs beta1, beta2 in [0, 1) and eps > 0");
+  SKY_CHECK(c.kind != SKY_OPT_SGD || (c.momentum >= 0.f && c.momentum < 1.f), SKY_ERR_INVALID_ARG,
+            "SGD momentum must be in [0, 1)");
+  for (int k = 0; k < SKY_NUM_PARAMS; ++k)
+    SKY_CHECK(param_elems(s, k) % 4 == 0, SKY_ERR_UNSUPPORTED,
+              "parameter %d has %zu elements, not a multiple of 4", k, param_elems(s, k));
+  if (s->last_stream) SKY_CUDA(cudaStreamSynchronize(s->last_stream));
+  SKY_CUDA(cudaDeviceSynchronize());
+  if (s->opt_mem) {
+    cudaFree(s->opt_mem);
+    s->opt_mem = nullptr;
+  }
+  s->opt_ready = false;
+  const bool bf = s->cfg.dtype == SKY_DTYPE_BF16;
+  const int nstate = c.kind == SKY_OPT_ADAMW ? 2 : 1;
+  const int copies = nstate + (bf ? 1 : 0);  // fp32 slices update their parameters in place
+  size_t per_layer = 0;
+  for (int k = 0; k < SKY_NUM_PARAMS; ++k) per_layer += align_up(param_elems(s, k) * 4) * copies;
+  const size_t ntens = (size_t)s->L * SKY_NUM_PARAMS;
+  std::vector<opt::Tensor> ts;
+  ts.reserve(ntens);
+  // tables first (sizes known once the tensors are listed), then the tensors
+  const size_t state_bytes = per_layer * s->L;
+  const size_t tab_bytes = align_up(ntens * sizeof(opt::Tensor));
+  // chunk count: one chunk per kChunk float4 groups of every tensor
+  size_t nchunks = 0;
+  for (int l = 0; l < s->L; ++l)
+    for (int k = 0; k < SKY_NUM_PARAMS; ++k)
+      nchunks += (size_t)ceil_div((int64_t)param_elems(s, k) / 4, opt::kChunk);
+  const size_t total = state_bytes + tab_bytes + align_up(nchunks * sizeof(opt::Chunk));
+  if (g_alloc_cap && total > g_alloc_cap) {
+    set_error("optimizer state needs %zu bytes, above the allocation cap", total);
+    return SKY_ERR_OOM;
+  }
+  cudaError_t e = cudaMalloc(&s->opt_mem, total);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    s->opt_mem = nullptr;
+    set_error("cudaMalloc(%zu) for optimizer state: %s", total, cudaGetErrorString(e));
+    return e == cudaErrorMemoryAllocation ? SKY_ERR_OOM : SKY_ERR_CUDA;
+  }
+  SKY_CUDA(cudaMemset(s->opt_mem, 0, state_bytes));
+  char* q = static_cast<char*>(s->opt_mem);
+  for (int l = 0; l < s->L; ++l) {
+    LayerBufs& Lb = s->layers[l];
+    for (int k = 0; k < SKY_NUM_PARAMS; ++k) {
+      const size_t n = param_elems(s, k);
+      auto take = [&]() {
+        float* r = reinterpret_cast<float*>(q);
+        q += align_up(n * 4);
+        return r;
+      };
+      opt::Tensor t{};
+      t.n = (int64_t)n;
+      t.g = Lb.g[k];
+      if (bf) {
+        t.w = take();
+        t.p = Lb.p[k];
+        SKY_TRY(to_f32(Lb.p[k], (int64_t)n, SKY_DTYPE_BF16, t.w, nullptr));
+      } else {
+        t.w = static_cast<float*>(Lb.p[k]);
+        t.p = nullptr;
+      }
+      t.s0 = take();
+      t.s1 = nstate == 2 ? take() : nullptr;
+      t.decay = (k == 0 || k == 2 || k == 6 || k == 8) ? 1 : 0;  // Wqkv, Wo, W1, W2
+      ts.push_back(t);
+    }
+  }
+  std::vector<opt::Chunk> chunks;
+  opt::make_chunks(ts, &chunks);
+  s->d_opt_tensors = reinterpret_cast<opt::Tensor*>(q);
+  q += tab_bytes;
+  s->d_opt_chunks = reinterpret_cast<opt::Chunk*>(q);
+  SKY_CUDA(cudaMemcpy(s->d_opt_tensors, ts.data(), ts.size() * sizeof(opt::Tensor),
+                      cudaMemcpyHostToDevice));
+  SKY_CUDA(cudaMemcpy(s->d_opt_chunks, chunks.data(), chunks.size() * sizeof(opt::Chunk),
+                      cudaMemcpyHostToDevice));
+  SKY_CUDA(cudaDeviceSynchronize());
+  s->opt_tensors = ts;
+  s->opt_chunks = (int)chunks.size();
+  s->opt_cfg = c;
+  s->opt_t = 0;
+  s->opt_ready = true;
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_optimizer_step(sky_slice* s, float lr, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s, SKY_ERR_INVALID_ARG, "null handle");
+  SKY_CHECK(s->opt_ready, SKY_ERR_STATE, "optimizer not initialised");
+  SKY_CHECK(lr >= 0.f, SKY_ERR_INVALID_ARG, "lr must be >= 0");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const sky_optimizer_config& c = s->opt_cfg;
+  s->opt_t += 1;
+  s->last_stream = st;
+  double bytes = 0;
+  for (const auto& t : s->opt_tensors)
+    bytes += (double)t.n * (c.kind == SKY_OPT_ADAMW ? 28.0 : 20.0) + (t.p ? 2.0 * t.n : 0.0);
+  Timed tm(s, st, P_COPY, 0, bytes);
+  if (c.kind == SKY_OPT_ADAMW) {
+    opt::AdamArgs a{lr, c.beta1, c.beta2, c.eps, c.weight_decay,
+                    (float)(1.0 - std::pow((double)c.beta1, (double)s->opt_t)),
+                    (float)(1.0 - std::pow((double)c.beta2, (double)s->opt_t))};
+    return opt::launch_adamw(s->d_opt_tensors, s->d_opt_chunks, s->opt_chunks, a, st);
+  }
+  opt::SgdArgs a{lr, c.momentum, c.weight_decay, s->opt_t == 1 ? 1 : 0};
+  return opt::launch_sgd(s->d_opt_tensors, s->d_opt_chunks, s->opt_chunks, a, st);
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_get_optimizer_state(sky_slice* s, int32_t layer, int32_t which,
+                                         void* const* dst) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s && dst, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(s->opt_ready, SKY_ERR_STATE, "optimizer not initialised");
+  const int li = layer_index(s, layer);
+  SKY_CHECK(li >= 0, SKY_ERR_INVALID_ARG, "layer %d outside the slice", layer);
+  SKY_CHECK(which >= 0 && which <= 2, SKY_ERR_INVALID_ARG, "which must be 0, 1 or 2");
+  SKY_CHECK(which != 2 || s->opt_cfg.kind == SKY_OPT_ADAMW, SKY_ERR_INVALID_ARG,
+            "SGD keeps one state tensor");
+  if (s->last_stream) SKY_CUDA(cudaStreamSynchronize(s->last_stream));
+  SKY_CUDA(cudaDeviceSynchronize());
+  for (int k = 0; k < SKY_NUM_PARAMS; ++k) {
+    const opt::Tensor& t = s->opt_tensors[(size_t)li * SKY_NUM_PARAMS + k];
+    const float* src = which == 0 ? t.w : (which == 1 ? t.s0 : t.s1);
+    SKY_CHECK(dst[k], SKY_ERR_INVALID_ARG, "tensor %d is null", k);
+    SKY_CUDA(cudaMemcpy(dst[k], src, (size_t)t.n * 4, cudaMemcpyDeviceToHost));
   }
   return SKY_OK;
   ABI_GUARD_END

@@ -80,6 +80,26 @@ class EncoderSlice:
         """fp32 gradients of the 12 tensors of `layer` from the last backward."""
         return self._get("sky_slice_get_grads", layer, True)
 
+    # ---------------------------------------------------- local update (Sec. III)
+    def optimizer_init(self, kind: str = "adamw", lr: float = 1e-4, beta1: float = 0.9,
+                       beta2: float = 0.999, eps: float = 1e-6, weight_decay: float = 0.01,
+                       momentum: float = 0.9) -> None:
+        """fp32 master weights and zeroed AdamW / SGD state (see sky_slice.h)."""
+        k = {"adamw": L.SKY_OPT_ADAMW, "sgd": L.SKY_OPT_SGD}[kind]
+        cfg = L.SkyOptimizerConfig(k, lr, beta1, beta2, eps, weight_decay, momentum)
+        L.call("sky_slice_optimizer_init", self.h, C.byref(cfg))
+
+    def optimizer_step(self, lr: float, stream=None) -> None:
+        """One update from the gradients of the last backward."""
+        L.call("sky_slice_optimizer_step", self.h, C.c_float(lr), _stream_ptr(stream))
+
+    def optimizer_state(self, layer: int, which: int) -> dict:
+        """fp32 master weights (0), first (1) or second (2) state of `layer`."""
+        bufs = [np.empty(self.shapes()[n], dtype=np.float32) for n in PARAM_NAMES]
+        arr = (C.c_void_p * 12)(*[b.ctypes.data for b in bufs])
+        L.call("sky_slice_get_optimizer_state", self.h, layer, which, arr)
+        return dict(zip(PARAM_NAMES, bufs))
+
     # -------------------------------------------------------------- compute
     def forward(self, x, lens, y=None, stream=None):
         """x: device [B, S, H] tensor (slice dtype); lens: device int32 [B]."""
