@@ -178,3 +178,16 @@ def test_paper_scale_160_layers_64_devices():
     print(f"\nD={D} L={L_}: even q={q_even:.3f}, heuristic q={q_heur:.3f}, "
           f"best in device order q={q_best:.3f}; heuristic {t_cpp*1e3:.2f} ms (C++) "
           f"vs {t_py*1e3:.1f} ms (oracle)")
+
+
+def test_gpipe_makespan_closed_forms():
+    from paper_2202_11836_gb300.pipeline import gpipe_makespan
+    # identical stages: (M + D - 1) forward slots, then (M + D - 1) backward slots
+    for D in (1, 2, 5):
+        for M in (1, 3, 8):
+            assert gpipe_makespan([2.0] * D, [3.0] * D, M) == pytest.approx((M + D - 1) * 5.0)
+    # one micro-batch: the devices run one after the other
+    assert gpipe_makespan([1.0, 2.0, 4.0], [2.0, 1.0, 3.0], 1) == pytest.approx(13.0)
+    # many micro-batches: the slowest stage sets the pace
+    t = gpipe_makespan([1.0, 5.0, 1.0], [1.0, 5.0, 1.0], 100)
+    assert t == pytest.approx(2 * (5.0 * 100 + 1.0 + 1.0))
