@@ -24,6 +24,8 @@ using bf16 = __nv_bfloat16;
 // shuffles.  Requires D == 64.
 __global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __restrict__ dctx, int S,
                                 int H, int A, int64_t rows, float* __restrict__ delta) {
+  pdl_trigger();
+  pdl_wait();
   const int64_t row = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
   const int l = threadIdx.x & 31;
   if (row >= rows) return;
@@ -224,10 +226,11 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
   const int dblocks = ceil_div(rows * A * 32, 256);
   if (dt == SKY_DTYPE_BF16) {
     SKY_CHECK(D == attn::HD, SKY_ERR_UNSUPPORTED, "bf16 attention needs head dim 64 (got %d)", D);
-    attn::attn_delta_bf16<<<ceil_div(rows * 32, 256), 256, 0, stream>>>(
-        static_cast<const __nv_bfloat16*>(ctx), static_cast<const __nv_bfloat16*>(dctx), S, H, A,
-        rows, delta);
+    const cudaError_t le = launch_pdl(attn::attn_delta_bf16, dim3(ceil_div(rows * 32, 256)), dim3(256),
+                                      0, stream, 1, static_cast<const __nv_bfloat16*>(ctx),
+                                      static_cast<const __nv_bfloat16*>(dctx), S, H, A, rows, delta);
     count_launches(1);
+    if (le != cudaSuccess) return cuda_fail(le, "attention delta launch");
     return attention_bwd_tc(qkv, dctx, lse, delta, lens, B, S, H, A, dqkv, status, 2000000000ull,
                             stream);
   } else {

@@ -72,6 +72,8 @@ struct FwdParams {
 __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ CUtensorMap tmQ,
                                                     const __grid_constant__ CUtensorMap tmKV,
                                                     const FwdParams p) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
@@ -351,6 +353,12 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
                                                           const __grid_constant__ CUtensorMap tmKV,
                                                           const __grid_constant__ CUtensorMap tmO,
                                                           const BwdParams p) {
+  // Launched right behind the dK/dV kernel, which it does not depend on (it
+  // writes the other columns of dQKV): it starts once every dK/dV CTA has
+  // started -- and so has seen the delta pre-pass complete -- runs beside it,
+  // and waits for it only before exiting, so the next kernel, which waits
+  // for this one, also sees dK and dV.
+  pdl_trigger();
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
@@ -569,6 +577,7 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, 256);
   }
+  pdl_wait();
 }
 
 // --------------------------------------------------------- backward, dK dV
@@ -598,6 +607,10 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
                                                             const __grid_constant__ CUtensorMap tmQ,
                                                             const __grid_constant__ CUtensorMap tmO,
                                                             const BwdParams p) {
+  // wait first, then let the dQ kernel start: once every CTA here has passed
+  // the wait, the delta pre-pass (and everything before it) is complete
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ uint8_t smem_raw[];
   const int kt = blockIdx.x, a = blockIdx.y, b = blockIdx.z;
   const int S = p.S, H = p.H;
@@ -925,9 +938,8 @@ sky_status attention_fwd_tc(const void* qkv, const int32_t* lens, int B, int S, 
   if (attr != cudaSuccess) return cuda_fail(attr, "attention smem attribute");
   FwdParams p{S, H, A, lens, static_cast<__nv_bfloat16*>(ctx), lse, status, timeout_ns};
   dim3 grid(ceil_div(S, BQ), A, B);
-  attn_fwd_tc<<<grid, NTHR, F_SMEM, stream>>>(tq, tkv, p);
+  const cudaError_t e = launch_pdl(attn_fwd_tc, grid, dim3(NTHR), F_SMEM, stream, 1, tq, tkv, p);
   count_launches(1);
-  const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "tensor-core attention forward launch");
 }
 
@@ -950,10 +962,12 @@ sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse,
   const int bulk = (S % 4 == 0) && (reinterpret_cast<uintptr_t>(lse) & 15) == 0 &&
                    (reinterpret_cast<uintptr_t>(delta) & 15) == 0;
   BwdParams p{S, H, A, bulk, lens, lse, delta, static_cast<__nv_bfloat16*>(dqkv), status, timeout_ns};
-  attn_bwd_dkdv_tc<<<dim3(ceil_div(S, BK2), A, B), NTHR_B, KV_SMEM, stream>>>(tk128, tq64, to64, p);
-  attn_bwd_dq_tc<<<dim3(ceil_div(S, BQ), A, B), NTHR_B, DQ_SMEM, stream>>>(tq128, tkv64, to128, p);
+  cudaError_t e = launch_pdl(attn_bwd_dkdv_tc, dim3(ceil_div(S, BK2), A, B), dim3(NTHR_B), KV_SMEM,
+                             stream, 1, tk128, tq64, to64, p);
+  if (e == cudaSuccess)
+    e = launch_pdl(attn_bwd_dq_tc, dim3(ceil_div(S, BQ), A, B), dim3(NTHR_B), DQ_SMEM, stream, 1,
+                   tq128, tkv64, to128, p);
   count_launches(2);
-  const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "tensor-core attention backward launch");
 }
 

@@ -94,4 +94,49 @@ int sm_count();  // cached per device
 // Number of kernels this library has launched (all threads, all devices).
 void count_launches(int n);
 
+// ---- Programmatic dependent launch ------------------------------------------
+// Hot-path kernels launch with programmatic stream serialization: the next
+// kernel on the stream may be scheduled once every CTA of the current one
+// has started (each calls pdl_trigger() first), and it runs pdl_wait() --
+// which returns when the previous grid has completed and its memory is
+// visible -- before it reads anything that grid wrote or writes anything it
+// reads.  Its launch and set-up then overlap the previous kernel's tail
+// instead of following its completion.  SKY_PDL=0 in the environment turns
+// the attribute off (plain stream order).
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+bool pdl_enabled();
+
+// cudaLaunchKernelEx with the programmatic-serialization attribute (when
+// enabled) and optionally a cluster of `cluster_x` CTAs.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, int cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[2];
+  int n = 0;
+  if (pdl_enabled()) {
+    at[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  if (cluster_x > 1) {
+    at[n].id = cudaLaunchAttributeClusterDimension;
+    at[n].val.clusterDim.x = cluster_x;
+    at[n].val.clusterDim.y = 1;
+    at[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.attrs = at;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 }  // namespace sky

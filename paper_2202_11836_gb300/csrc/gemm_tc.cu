@@ -105,6 +105,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint64_t* done = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
 
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = PAIR ? ptx::cluster_ctarank() : 0u;
   const bool leader = rank == 0;
@@ -141,6 +142,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   else __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();  // the set-up above overlapped the previous kernel; its outputs are visible now
 
   const int tiles = p.m_tiles * p.n_tiles;
   const int units = tiles * p.splits;
@@ -401,6 +403,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // Fixed-order sum of split-K partials: out[i] = sum_s ws[s][i].
 __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int splits, int64_t n,
                                      float* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   const int64_t n4 = n / 4;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4;
        i += (int64_t)gridDim.x * blockDim.x) {
@@ -461,22 +465,19 @@ cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUte
   if (attr != cudaSuccess) return attr;
   if constexpr (!PAIR) {
     const int grid = units < sms ? units : sms;
-    kern<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(ta, tb, p);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(grid), dim3(NUM_THREADS), SMEM_BYTES, stream, 1, ta, tb, p);
   } else {
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute at[1];
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = 2;
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    cfg.blockDim = dim3(NUM_THREADS);
-    cfg.dynamicSmemBytes = SMEM_BYTES;
-    cfg.stream = stream;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
     static int max_clusters = [&] {
-      cudaLaunchConfig_t q = cfg;
+      cudaLaunchConfig_t q = {};
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 2;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      q.blockDim = dim3(NUM_THREADS);
+      q.dynamicSmemBytes = SMEM_BYTES;
+      q.attrs = at;
+      q.numAttrs = 1;
       q.gridDim = dim3(2 * (sms / 2));
       int n = 0;
       if (cudaOccupancyMaxActiveClusters(&n, kern, &q) != cudaSuccess) {
@@ -487,8 +488,8 @@ cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUte
     }();
     if (max_clusters < 1) return cudaErrorLaunchOutOfResources;
     const int clusters = units < max_clusters ? units : max_clusters;
-    cfg.gridDim = dim3(2 * clusters);
-    return cudaLaunchKernelEx(&cfg, kern, ta, tb, p);
+    return launch_pdl(kern, dim3(2 * clusters), dim3(NUM_THREADS), SMEM_BYTES, stream, 2, ta, tb,
+                      p);
   }
 }
 
@@ -651,10 +652,9 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   if (p.splits > 1) {
     const int64_t n = static_cast<int64_t>(M) * N;
     const int blocks = static_cast<int>(std::min<int64_t>(ceil_div(n / 4 + 1, 256), sms * 8));
-    splitk_reduce_kernel<<<blocks, 256, 0, stream>>>(static_cast<const float*>(ws), p.splits, n,
-                                                     static_cast<float*>(C));
+    e = launch_pdl(splitk_reduce_kernel, dim3(blocks), dim3(256), 0, stream, 1,
+                   static_cast<const float*>(ws), p.splits, n, static_cast<float*>(C));
     count_launches(1);
-    e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "splitk_reduce launch");
   }
   return SKY_OK;

@@ -34,6 +34,8 @@ __device__ __forceinline__ void store_param(void* p, int64_t i4, const float4& w
 __global__ void __launch_bounds__(kThreads) adamw_kernel(const Tensor* __restrict__ ts,
                                                          const Chunk* __restrict__ chunks,
                                                          int n_chunks, AdamArgs a) {
+  pdl_trigger();
+  pdl_wait();
   for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
     const Chunk ch = chunks[c];
     const Tensor t = ts[ch.tensor];
@@ -65,6 +67,8 @@ __global__ void __launch_bounds__(kThreads) adamw_kernel(const Tensor* __restric
 __global__ void __launch_bounds__(kThreads) sgd_kernel(const Tensor* __restrict__ ts,
                                                        const Chunk* __restrict__ chunks,
                                                        int n_chunks, SgdArgs a) {
+  pdl_trigger();
+  pdl_wait();
   for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
     const Chunk ch = chunks[c];
     const Tensor t = ts[ch.tensor];
@@ -103,7 +107,7 @@ sky_status launch_adamw(const Tensor* d_ts, const Chunk* d_chunks, int n_chunks,
                         cudaStream_t st) {
   const int blocks = std::min(n_chunks, 8 * (sm_count() > 0 ? sm_count() : 148));
   if (blocks <= 0) return SKY_OK;
-  adamw_kernel<<<blocks, kThreads, 0, st>>>(d_ts, d_chunks, n_chunks, a);
+  launch_pdl(adamw_kernel, dim3(blocks), dim3(kThreads), 0, st, 1, d_ts, d_chunks, n_chunks, a);
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "AdamW update launch");
@@ -113,7 +117,7 @@ sky_status launch_sgd(const Tensor* d_ts, const Chunk* d_chunks, int n_chunks, c
                       cudaStream_t st) {
   const int blocks = std::min(n_chunks, 8 * (sm_count() > 0 ? sm_count() : 148));
   if (blocks <= 0) return SKY_OK;
-  sgd_kernel<<<blocks, kThreads, 0, st>>>(d_ts, d_chunks, n_chunks, a);
+  launch_pdl(sgd_kernel, dim3(blocks), dim3(kThreads), 0, st, 1, d_ts, d_chunks, n_chunks, a);
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "SGD update launch");

@@ -52,6 +52,8 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_fwd_kernel(
     const T* __restrict__ beta, int rows, int H, float eps, float* u_out,
     float* __restrict__ y32, T* __restrict__ yT, float* __restrict__ mean_out,
     float* __restrict__ rstd_out) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int warp = blockIdx.x * LN_WARPS + (threadIdx.x >> 5);
   const int nwarps = gridDim.x * LN_WARPS;
@@ -124,6 +126,8 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_bwd_kernel(
     const T* __restrict__ gamma,
     const float* __restrict__ mean, const float* __restrict__ rstd, int rows, int H,
     float* __restrict__ du32, T* __restrict__ duT, float* __restrict__ part) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ float red[];  // [LN_WARPS][3][H]
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const int warp = blockIdx.x * LN_WARPS + wib;
@@ -205,6 +209,8 @@ __global__ void __launch_bounds__(LN_WARPS * 32) ln_bwd_kernel(
 template <typename T>
 __global__ void add_kernel(const float* __restrict__ a, const float* __restrict__ b, int64_t n,
                            T* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
     out[i] = from_f32<T>(a[i] + b[i]);
@@ -212,6 +218,8 @@ __global__ void add_kernel(const float* __restrict__ a, const float* __restrict_
 
 __global__ void to_bf16_kernel(const float* __restrict__ x, int64_t n,
                                __nv_bfloat16* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
     out[i] = __float2bfloat16_rn(x[i]);
@@ -219,6 +227,8 @@ __global__ void to_bf16_kernel(const float* __restrict__ x, int64_t n,
 
 template <typename T>
 __global__ void to_f32_kernel(const T* __restrict__ x, int64_t n, float* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
     out[i] = to_f32(x[i]);
@@ -261,6 +271,8 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
     const __nv_bfloat16* __restrict__ gamma, const float* __restrict__ mean,
     const float* __restrict__ rstd, int rows, int H, float* __restrict__ du32,
     __nv_bfloat16* __restrict__ duT, float* __restrict__ part, int32_t* status) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ uint8_t sm_raw[];
   uint8_t* sm = sm_raw + ((128 - (ptx::smem_u32(sm_raw) & 127)) & 127);
   uint64_t* full = reinterpret_cast<uint64_t*>(sm + SB_RING * SB_ROW_BYTES);
@@ -381,6 +393,8 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
 __global__ void __launch_bounds__(256) reduce_partials(const float* __restrict__ part, int nblk,
                                                        int N, float* out0, float* out1,
                                                        float* out2) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[8][33];
   const int k = blockIdx.y;
   float* out = k == 0 ? out0 : (k == 1 ? out1 : out2);
@@ -409,6 +423,8 @@ __global__ void __launch_bounds__(256) reduce_partials(const float* __restrict__
 template <typename T>
 __global__ void __launch_bounds__(256) colsum_partial(const T* __restrict__ x, int rows, int N,
                                                       float* __restrict__ part) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[8][256];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int col = blockIdx.x * 256 + lane * 8;
@@ -480,7 +496,7 @@ template <typename T, int NV>
 void ln_fwd_launch(const float* a, const float* r, const void* gm, const void* bt, int rows, int H,
                    float eps, float* u_out, float* y32, void* y, float* mean, float* rstd,
                    cudaStream_t st) {
-  ln_fwd_kernel<T, NV><<<ln_blocks(rows), LN_WARPS * 32, 0, st>>>(
+  launch_pdl(ln_fwd_kernel<T, NV>, dim3(ln_blocks(rows)), dim3(LN_WARPS * 32), 0, st, 1, 
       a, r, static_cast<const T*>(gm), static_cast<const T*>(bt), rows, H, eps, u_out, y32,
       static_cast<T*>(y), mean, rstd);
 }
@@ -492,7 +508,7 @@ void ln_bwd_launch(const void* dy, const float* dy2, const float* u, const void*
   if (smem > 48 * 1024)
     cudaFuncSetAttribute(ln_bwd_kernel<TDY, T, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);
-  ln_bwd_kernel<TDY, T, NV><<<nblk, LN_WARPS * 32, smem, st>>>(
+  launch_pdl(ln_bwd_kernel<TDY, T, NV>, dim3(nblk), dim3(LN_WARPS * 32), smem, st, 1, 
       static_cast<const TDY*>(dy), dy2, u, static_cast<const T*>(gm), mean, rstd, rows, H, du32,
       static_cast<T*>(du), part);
 }
@@ -570,14 +586,14 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
       static cudaError_t a = cudaFuncSetAttribute(rw::ln_bwd_stream_kernel<__nv_bfloat16>,
                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
       if (a != cudaSuccess) return cuda_fail(a, "LayerNorm backward smem attribute");
-      rw::ln_bwd_stream_kernel<__nv_bfloat16><<<sb, threads, smem, st>>>(
+      launch_pdl(rw::ln_bwd_stream_kernel<__nv_bfloat16>, dim3(sb), dim3(threads), smem, st, 1, 
           static_cast<const __nv_bfloat16*>(dy), dy2, u, static_cast<const __nv_bfloat16*>(gamma),
           mean, rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, nullptr);
     } else {
       static cudaError_t a = cudaFuncSetAttribute(rw::ln_bwd_stream_kernel<float>,
                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
       if (a != cudaSuccess) return cuda_fail(a, "LayerNorm backward smem attribute");
-      rw::ln_bwd_stream_kernel<float><<<sb, threads, smem, st>>>(
+      launch_pdl(rw::ln_bwd_stream_kernel<float>, dim3(sb), dim3(threads), smem, st, 1, 
           static_cast<const float*>(dy), dy2, u, static_cast<const __nv_bfloat16*>(gamma), mean,
           rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, nullptr);
     }
@@ -621,7 +637,7 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
 sky_status layernorm_bwd_reduce(const void* ws, int parts, int H, float* dgamma, float* dbeta,
                                 float* dbias, cudaStream_t st) {
   dim3 grid(ceil_div(H, 32), 3);
-  rw::reduce_partials<<<grid, 256, 0, st>>>(static_cast<const float*>(ws), parts, H, dgamma,
+  launch_pdl(rw::reduce_partials, dim3(grid), dim3(256), 0, st, 1, static_cast<const float*>(ws), parts, H, dgamma,
                                             dbeta, dbias);
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
@@ -630,7 +646,7 @@ sky_status layernorm_bwd_reduce(const void* ws, int parts, int H, float* dgamma,
 
 namespace gemm {
 cudaError_t reduce_rows_f32(const float* part, int rows, int N, float* out, cudaStream_t stream) {
-  rw::reduce_partials<<<dim3(ceil_div(N, 32), 1), 256, 0, stream>>>(part, rows, N, out, nullptr,
+  launch_pdl(rw::reduce_partials, dim3(dim3(ceil_div(N, 32), 1)), dim3(256), 0, stream, 1, part, rows, N, out, nullptr,
                                                                   nullptr);
   count_launches(1);
   return cudaGetLastError();
@@ -642,9 +658,9 @@ sky_status add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dt, 
   if (n <= 0) return SKY_OK;
   const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
   if (out_dt == SKY_DTYPE_BF16)
-    rw::add_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(a, b, n, static_cast<__nv_bfloat16*>(out));
+    launch_pdl(rw::add_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, st, 1, a, b, n, static_cast<__nv_bfloat16*>(out));
   else
-    rw::add_kernel<float><<<blocks, 256, 0, st>>>(a, b, n, static_cast<float*>(out));
+    launch_pdl(rw::add_kernel<float>, dim3(blocks), dim3(256), 0, st, 1, a, b, n, static_cast<float*>(out));
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "add launch");
@@ -653,7 +669,7 @@ sky_status add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dt, 
 sky_status f32_to_bf16(const float* x, int64_t n, void* out, cudaStream_t st) {
   if (n <= 0) return SKY_OK;
   const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
-  rw::to_bf16_kernel<<<blocks, 256, 0, st>>>(x, n, static_cast<__nv_bfloat16*>(out));
+  launch_pdl(rw::to_bf16_kernel, dim3(blocks), dim3(256), 0, st, 1, x, n, static_cast<__nv_bfloat16*>(out));
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "narrow launch");
@@ -663,10 +679,10 @@ sky_status to_f32(const void* x, int64_t n, sky_dtype dt, float* out, cudaStream
   if (n <= 0) return SKY_OK;
   const int blocks = (int)std::min<int64_t>(ceil_div(n, 256), 8 * 148);
   if (dt == SKY_DTYPE_BF16)
-    rw::to_f32_kernel<__nv_bfloat16><<<blocks, 256, 0, st>>>(
+    launch_pdl(rw::to_f32_kernel<__nv_bfloat16>, dim3(blocks), dim3(256), 0, st, 1, 
         static_cast<const __nv_bfloat16*>(x), n, out);
   else
-    rw::to_f32_kernel<float><<<blocks, 256, 0, st>>>(static_cast<const float*>(x), n, out);
+    launch_pdl(rw::to_f32_kernel<float>, dim3(blocks), dim3(256), 0, st, 1, static_cast<const float*>(x), n, out);
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "widen launch");
@@ -696,11 +712,11 @@ sky_status column_sum(const void* x, int rows, int N, sky_dtype dt, float* out, 
   float* part = static_cast<float*>(ws);
   dim3 grid(ceil_div(N, 256), groups);
   if (dt == SKY_DTYPE_BF16)
-    rw::colsum_partial<__nv_bfloat16><<<grid, 256, 0, st>>>(
+    launch_pdl(rw::colsum_partial<__nv_bfloat16>, dim3(grid), dim3(256), 0, st, 1, 
         static_cast<const __nv_bfloat16*>(x), rows, N, part);
   else
-    rw::colsum_partial<float><<<grid, 256, 0, st>>>(static_cast<const float*>(x), rows, N, part);
-  rw::reduce_partials<<<dim3(ceil_div(N, 32), 1), 256, 0, st>>>(part, groups, N, out, nullptr,
+    launch_pdl(rw::colsum_partial<float>, dim3(grid), dim3(256), 0, st, 1, static_cast<const float*>(x), rows, N, part);
+  launch_pdl(rw::reduce_partials, dim3(dim3(ceil_div(N, 32), 1)), dim3(256), 0, st, 1, part, groups, N, out, nullptr,
                                                                 nullptr);
   count_launches(2);
   const cudaError_t e = cudaGetLastError();

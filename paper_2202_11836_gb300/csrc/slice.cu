@@ -13,6 +13,7 @@
 #include <atomic>
 #include <cmath>
 #include <cstdarg>
+#include <cstdlib>
 #include <cstring>
 #include <exception>
 #include <new>
@@ -31,6 +32,14 @@ thread_local std::string g_last_error;
 uint64_t g_alloc_cap = 0;
 std::atomic<int64_t> g_launches{0};
 }  // namespace
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("SKY_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
 
 void count_launches(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
