@@ -49,18 +49,27 @@ constexpr int A_BYTES = BM * BK * 2;        // 16 KiB
 constexpr int B_BYTES = BN * BK * 2;        // 32 KiB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;           // two fp32 accumulators of 128 x 256
-constexpr int NUM_EPI_WARPS = 8;            // two per TMEM lane quarter
-constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
-constexpr int EPI_OFF = STAGES * STAGE_BYTES;           // per epilogue warp: 32 x 32 fp32 staging
-constexpr int EPI_BYTES = NUM_EPI_WARPS * 32 * 32 * 4;
-constexpr int BAR_OFF = EPI_OFF + EPI_BYTES;
-constexpr int SMEM_BYTES = BAR_OFF + 256 /*barriers*/ + 1024 /*alignment slack*/;
+constexpr int NUM_EPI_WARPS = 8;            // two per TMEM lane quarter (default)
 constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
 // CTA-pair variant: per CTA and stage A 128 x 64 + B 128 x 64 (32 KiB), six
 // stages in the same 192 KiB
 constexpr int PAIR_STAGES = 6;
 constexpr int PAIR_STAGE_BYTES = A_BYTES + (BN / 2) * BK * 2;
 static_assert(PAIR_STAGES * PAIR_STAGE_BYTES == STAGES * STAGE_BYTES, "same ring size");
+
+// Launch shape per instantiation: epilogue warps (a multiple of 4, one group
+// per TMEM lane quarter), ring stages and shared memory.
+template <int EPI, bool PAIR>
+struct Shape {
+  static constexpr int EW = NUM_EPI_WARPS;
+  static constexpr int THREADS = 64 + 32 * EW;
+  static constexpr int NST = PAIR ? PAIR_STAGES : (EW == 16 ? 3 : STAGES);
+  static constexpr int SBYTES = PAIR ? PAIR_STAGE_BYTES : STAGE_BYTES;
+  static constexpr int EPI_OFF = NST * SBYTES;               // per epilogue warp: 32 x 32 fp32 staging
+  static constexpr int BAR_OFF = EPI_OFF + EW * 32 * 32 * 4;
+  static constexpr int SMEM = BAR_OFF + 256 /*barriers*/ + 1024 /*alignment slack*/;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
+};
 constexpr uint32_t kSleepNs = 20000;         // suspend hint of the epilogue's accumulator wait
 
 struct Params {
@@ -88,17 +97,19 @@ __device__ __forceinline__ uint2 ld_nc_u2(const void* p) {
 // PAIR: the CTA-pair variant (launched in clusters of two; p.m_tiles counts
 // 256-row tiles).
 template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA,
                    const __grid_constant__ CUtensorMap tmB, const Params p) {
-  constexpr int NST = PAIR ? PAIR_STAGES : STAGES;
-  constexpr int SBYTES = PAIR ? PAIR_STAGE_BYTES : STAGE_BYTES;
+  using SH = Shape<EPI, PAIR>;
+  constexpr int NST = SH::NST;
+  constexpr int SBYTES = SH::SBYTES;
+  constexpr int EW = SH::EW;
   constexpr int B_ROWS = PAIR ? BN / 2 : BN;  // B rows (tile columns) this CTA loads
   constexpr int TILE_M = PAIR ? 2 * BM : BM;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + BAR_OFF);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + SH::BAR_OFF);
   uint64_t* empty = full + NST;
   uint64_t* tfull = empty + NST;
   uint64_t* tempty = tfull + 2;
@@ -118,7 +129,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(&tfull[a], 1);
-      ptx::mbar_init(&tempty[a], (PAIR ? 2 : 1) * 32 * NUM_EPI_WARPS);
+      ptx::mbar_init(&tempty[a], (PAIR ? 2 : 1) * 32 * EW);
     }
     ptx::mbar_init(done, 1);
     if constexpr (PAIR) ptx::fence_mbar_init_cluster();
@@ -260,9 +271,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     // column half hf of the tile.  Per 32-column chunk: tcgen05.ld (thread =
     // row) -> XOR-swizzled smem tile -> read back so that 8 lanes cover one
     // row's 32 columns, then the fused epilogue and coalesced stores.
-    constexpr int HALF = BN / 2, CHUNKS = HALF / 32;
+    constexpr int HALF = BN / (EW / 4), CHUNKS = HALF / 32;  // columns of a warp, 32-column chunks
     const int q = warp & 3, hf = (warp - 2) >> 2;
-    float* stage = reinterpret_cast<float*>(smem + EPI_OFF) + (warp - 2) * 32 * 32;
+    float* stage = reinterpret_cast<float*>(smem + SH::EPI_OFF) + (warp - 2) * 32 * 32;
     const int c4 = lane & 7;          // this lane's 4-column group in a chunk
     const int rsub = lane >> 3;       // row within each group of 4 rows
     int acc = 0;
@@ -460,12 +471,13 @@ template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR>
 cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
                            const Params& p, cudaStream_t stream) {
   auto kern = gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32, PAIR>;
+  using SH = Shape<EPI, PAIR>;
   static cudaError_t attr =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SH::SMEM);
   if (attr != cudaSuccess) return attr;
   if constexpr (!PAIR) {
     const int grid = units < sms ? units : sms;
-    return launch_pdl(kern, dim3(grid), dim3(NUM_THREADS), SMEM_BYTES, stream, 1, ta, tb, p);
+    return launch_pdl(kern, dim3(grid), dim3(SH::THREADS), SH::SMEM, stream, 1, ta, tb, p);
   } else {
     static int max_clusters = [&] {
       cudaLaunchConfig_t q = {};
@@ -474,8 +486,8 @@ cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUte
       at[0].val.clusterDim.x = 2;
       at[0].val.clusterDim.y = 1;
       at[0].val.clusterDim.z = 1;
-      q.blockDim = dim3(NUM_THREADS);
-      q.dynamicSmemBytes = SMEM_BYTES;
+      q.blockDim = dim3(SH::THREADS);
+      q.dynamicSmemBytes = SH::SMEM;
       q.attrs = at;
       q.numAttrs = 1;
       q.gridDim = dim3(2 * (sms / 2));
@@ -488,8 +500,7 @@ cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUte
     }();
     if (max_clusters < 1) return cudaErrorLaunchOutOfResources;
     const int clusters = units < max_clusters ? units : max_clusters;
-    return launch_pdl(kern, dim3(2 * clusters), dim3(NUM_THREADS), SMEM_BYTES, stream, 2, ta, tb,
-                      p);
+    return launch_pdl(kern, dim3(2 * clusters), dim3(SH::THREADS), SH::SMEM, stream, 2, ta, tb, p);
   }
 }
 
