@@ -36,7 +36,6 @@ namespace attn_tc {
 constexpr int BQ = 128, BKV = 64, HD = 64;
 constexpr int Q_BYTES = BQ * HD * 2;    // 16 KiB
 constexpr int KV_BYTES = BKV * HD * 2;  // 8 KiB per K or V tile
-constexpr int P_BYTES = BQ * BKV * 2;   // 16 KiB
 constexpr int STAGES = 2;               // backward operand rings
 constexpr int NTHR = 192;               // warp 0 TMA, warp 1 MMA, warps 2..5 softmax
 // The backward kernels run eight softmax warps: warps w and w + 4 share TMEM
@@ -54,10 +53,11 @@ constexpr uint32_t kWaitHint = 10000;
 constexpr int F_STAGES = 3;
 constexpr int F_Q_OFF = 0;
 constexpr int F_KV_OFF = F_Q_OFF + Q_BYTES;                  // [F_STAGES] x {K, V}
-constexpr int F_P_OFF = F_KV_OFF + F_STAGES * 2 * KV_BYTES;  // [2] P tiles
-constexpr int F_BAR_OFF = F_P_OFF + 2 * P_BYTES;
+constexpr int F_BAR_OFF = F_KV_OFF + F_STAGES * 2 * KV_BYTES;
 constexpr int F_SMEM = F_BAR_OFF + 256 + 1024;
-constexpr int F_TMEM_COLS = 256;  // S_0: [0, 64), S_1: [64, 128), O: [128, 192)
+// S_0: [0, 64), S_1: [64, 128), O: [128, 192), P_0: [192, 224), P_1: [224, 256)
+// (P as bf16 pairs: the A operand of P V read from tensor memory)
+constexpr int F_TMEM_COLS = 256;
 constexpr float kRescaleLog2 = 8.f;
 
 struct FwdParams {
@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS = tmem, tO = tmem + 128;
+  const uint32_t tS = tmem, tO = tmem + 128, tP = tmem + 192;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -152,7 +152,6 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
       constexpr uint32_t idO = ptx::idesc_bf16_f32(BQ, HD, false, true);
       const uint32_t sq = ptx::smem_u32(smem + F_Q_OFF);
       const uint32_t skv = ptx::smem_u32(smem + F_KV_OFF);
-      const uint32_t sp = ptx::smem_u32(smem + F_P_OFF);
       // S_j = Q K_j^T into S buffer j & 1 (K_j already landed)
       auto mma_s = [&](int j) {
         const uint32_t sk = skv + (j % F_STAGES) * 2 * KV_BYTES;
@@ -187,12 +186,11 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
           break;
         ptx::tc_fence_after();
         const uint32_t sv = skv + (j % F_STAGES) * 2 * KV_BYTES + KV_BYTES;
-        const uint32_t spj = sp + (j & 1) * P_BYTES;
+        const uint32_t tpj = tP + (j & 1) * (BKV / 2);
 #pragma unroll
         for (int kk = 0; kk < BKV / 16; ++kk)
-          ptx::tc_mma_f16(tO, ptx::smem_desc_sw128(spj + kk * 32, 16, 1024),
-                          ptx::smem_desc_sw128(sv + kk * 2048, 8192, 1024), idO,
-                          (j > 0 || kk > 0) ? 1u : 0u);
+          ptx::tc_mma_f16_tmem_a(tO, tpj + kk * 8, ptx::smem_desc_sw128(sv + kk * 2048, 8192, 1024),
+                                 idO, (j > 0 || kk > 0) ? 1u : 0u);
         ptx::tc_commit(&pv_done[j & 1]);
         ptx::tc_commit(&kv_empty[j % F_STAGES]);
         if (!s_done) {  // S_{j+1} is needed before P_{j+1} can exist
@@ -267,24 +265,25 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
         l *= alpha;
         m = m_new;
       }
-      // P buffer j & 1 was last read by P_{j-2} V_{j-2}
-      if (j >= 2 && !wait_all(&pv_done[j & 1], ((j - 2) >> 1) & 1)) { ok = false; break; }
-      // P = exp2(s * sl2 - m) as bf16, row r of the swizzled K-major tile
-      uint8_t* prow = smem + F_P_OFF + (j & 1) * P_BYTES + r * 128;
+      // P = exp2(s * sl2 - m) as bf16 pairs into this row's lane of P buffer
+      // j & 1 in tensor memory
       const float nm = -m;
       float ls = 0.f;
+      uint32_t pk[BKV / 2];
 #pragma unroll
-      for (int u = 0; u < BKV / 8; ++u) {  // 16-byte unit u holds keys 8u .. 8u+7
+      for (int u = 0; u < BKV / 8; ++u) {
         float e[8];
 #pragma unroll
         for (int t = 0; t < 8; ++t) e[t] = ptx::ex2_ftz(fmaf(__uint_as_float(v[8 * u + t]), sl2, nm));
         ls += ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
-        *reinterpret_cast<uint4*>(prow + ((u ^ (r & 7)) << 4)) =
-            make_uint4(ptx::pack_bf16(e[0], e[1]), ptx::pack_bf16(e[2], e[3]),
-                       ptx::pack_bf16(e[4], e[5]), ptx::pack_bf16(e[6], e[7]));
+#pragma unroll
+        for (int t = 0; t < 4; ++t) pk[4 * u + t] = ptx::pack_bf16(e[2 * t], e[2 * t + 1]);
       }
       l += ls;
-      ptx::fence_proxy_async_smem();
+      // P buffer j & 1 was last read by P_{j-2} V_{j-2}
+      if (j >= 2 && !wait_all(&pv_done[j & 1], ((j - 2) >> 1) & 1)) { ok = false; break; }
+      ptx::tmem_st_32x32b_x32(tP + (j & 1) * (BKV / 2) + lane_base, pk);
+      ptx::tmem_st_wait();
       ptx::tc_fence_before();
       ptx::mbar_arrive(&p_full[j & 1]);
     }
@@ -334,8 +333,7 @@ constexpr int DQ_STAGES = 3;
 constexpr int DQ_QD_BYTES = 2 * Q_BYTES;  // Q and dO tiles (128 x 64 each)
 constexpr int DQ_Q_OFF = 0, DQ_DO_OFF = Q_BYTES;
 constexpr int DQ_KV_OFF = DQ_QD_BYTES;                           // [DQ_STAGES] x {K, V}
-constexpr int DQ_DS_OFF = DQ_KV_OFF + DQ_STAGES * 2 * KV_BYTES;  // dS tile
-constexpr int DQ_BAR_OFF = DQ_DS_OFF + P_BYTES;
+constexpr int DQ_BAR_OFF = DQ_KV_OFF + DQ_STAGES * 2 * KV_BYTES;
 constexpr int DQ_SMEM = DQ_BAR_OFF + 256 + 1024;
 
 struct BwdParams {
@@ -406,7 +404,9 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS = tmem, tdP = tmem + 64, tdQ = tmem + 128;
+  // S: [0, 64), dP: [64, 128), dQ: [128, 192), dS as bf16 pairs (the A
+  // operand of dS K, read from tensor memory): [192, 224)
+  const uint32_t tS = tmem, tdP = tmem + 64, tdQ = tmem + 128, tdS = tmem + 192;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -437,7 +437,6 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
       constexpr uint32_t idQ = ptx::idesc_bf16_f32(BQ, HD, false, true);
       const uint32_t sq = ptx::smem_u32(smem + DQ_Q_OFF), so = ptx::smem_u32(smem + DQ_DO_OFF);
       const uint32_t skv = ptx::smem_u32(smem + DQ_KV_OFF);
-      const uint32_t sds = ptx::smem_u32(smem + DQ_DS_OFF);
       // S_j = Q K_j^T and dP_j = dO V_j^T (operands already landed)
       auto mma_sdp = [&](int j) {
         const uint32_t sk = skv + (j % DQ_STAGES) * 2 * KV_BYTES, sv = sk + KV_BYTES;
@@ -477,12 +476,10 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
           break;
         ptx::tc_fence_after();
         const uint32_t sk = skv + (j % DQ_STAGES) * 2 * KV_BYTES;
-        const uint32_t sdj = sds;
 #pragma unroll
         for (int kk = 0; kk < BKV / 16; ++kk)
-          ptx::tc_mma_f16(tdQ, ptx::smem_desc_sw128(sdj + kk * 32, 16, 1024),
-                          ptx::smem_desc_sw128(sk + kk * 2048, 8192, 1024), idQ,
-                          (j > 0 || kk > 0) ? 1u : 0u);
+          ptx::tc_mma_f16_tmem_a(tdQ, tdS + kk * 8, ptx::smem_desc_sw128(sk + kk * 2048, 8192, 1024),
+                                 idQ, (j > 0 || kk > 0) ? 1u : 0u);
         ptx::tc_commit(dq_done);
         ptx::tc_commit(&kv_empty[j % DQ_STAGES]);
         if (!next_done) {
@@ -506,7 +503,6 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
     const int64_t sidx = (static_cast<int64_t>(b) * p.A + a) * S + (q < S ? q : 0);
     const float nlse2 = q < S ? -p.lse[sidx] * LOG2E : -INFINITY;  // P = 0 on rows past S
     const float dl = q < S ? p.delta[sidx] : 0.f;
-    uint8_t* drow = smem + DQ_DS_OFF + r * 128;
     bool ok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
       const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, kWaitHint);
@@ -543,11 +539,11 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
       }
       // the dS buffer was last read by the dQ product of tile j - 1
       if (j >= 1 && !wait_all(dq_done, (j - 1) & 1)) { ok = false; break; }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        *reinterpret_cast<uint4*>(drow + (((hf * 4 + u) ^ (r & 7)) << 4)) =
-            make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-      ptx::fence_proxy_async_smem();
+      {  // this half's 32 keys = 16 columns of the row's lane
+        uint32_t (&p0)[16] = *reinterpret_cast<uint32_t(*)[16]>(&pk[0]);
+        ptx::tmem_st_32x32b_x16(tdS + hf * 16 + lane_base, p0);
+      }
+      ptx::tmem_st_wait();
       ptx::tc_fence_before();
       ptx::mbar_arrive(ds_full);
     }
