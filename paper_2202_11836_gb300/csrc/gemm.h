@@ -13,11 +13,14 @@ namespace gemm {
 // `ws`.  With `deferred_rows`, the partials go to `colpart` instead, no sum is
 // launched and *deferred_rows reports their row count (for reduce_rows_f32,
 // possibly on another stream ordered after this launch).
+// resid (optional, fp32 output of the STORE epilogue, no split): C = acc +
+// bias + resid[m, n], added in that order (the residual branch of Sec. II-C).
 sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
                        cudaStream_t stream, float* colsum = nullptr, float* colpart = nullptr,
-                       size_t colpart_bytes = 0, int* deferred_rows = nullptr);
+                       size_t colpart_bytes = 0, int* deferred_rows = nullptr,
+                       const float* resid = nullptr);
 // Rows of column partials a bf16 GEMM with M rows writes (upper bound).
 int colpart_rows_max(int M);
 // out[n] = sum over r of part[r][n] in order r = 0, 1, ... (rowwise.cu).

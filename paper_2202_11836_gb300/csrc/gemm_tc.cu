@@ -80,6 +80,7 @@ struct Params {
   const __half* aux;              // [M,N] GELU'(z) (GELU_BWD) or null
   __half* aux_out;                // [M,N] GELU'(z) (BIAS_GELU) or null
   float* colpart;                 // [m_tiles * 4][N] per-warp column sums of C, or null
+  const float* resid;             // [M,N] fp32 added after the bias (fp32 outputs), or null
   int32_t* status;
   uint64_t timeout_ns;
   int skip_loads;                 // fault injection: producer never issues TMA
@@ -90,6 +91,13 @@ __device__ __forceinline__ uint2 ld_nc_u2(const void* p) {
   uint2 v;
   asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0, %1}, [%2];"
                : "=r"(v.x), "=r"(v.y)
+               : "l"(p));
+  return v;
+}
+__device__ __forceinline__ float4 ld_nc_f4(const float* p) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
                : "l"(p));
   return v;
 }
@@ -297,6 +305,22 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
           }
         }
       }
+      // fp32 residual (post-LN residual branch), one 32-column chunk ahead:
+      // chunk 0 before the accumulator wait, chunk cc+1 while cc is stored
+      const float* rp = OUT_F32 ? p.resid : nullptr;
+      float4 res[OUT_F32 ? 8 : 1];
+      auto load_res = [&](int cc, float4* d) {
+        const int col = n0 + cc * 32 + 4 * c4;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int row = m0 + q * 32 + 4 * i + rsub;
+          d[i] = (col < p.N && row < p.M) ? ld_nc_f4(rp + static_cast<int64_t>(row) * p.N + col)
+                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      };
+      if constexpr (OUT_F32) {
+        if (rp) load_res(0, res);
+      }
       if (!ptx::mbar_wait(&tfull[acc], aphase, lim, p.status, kSleepNs)) break;
       ptx::tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN + hf * HALF;
@@ -331,12 +355,25 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
         }
         // all 8 rows x 4 columns first (independent, branch-free), then the
         // bounds-checked stores
+        float4 nxt[OUT_F32 ? 8 : 1];
+        if constexpr (OUT_F32) {
+          if (rp && cc + 1 < CHUNKS) load_res(cc + 1, nxt);
+        }
         float v[8][4];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           const int rl = 4 * i + rsub;
           const float4 t4 = *reinterpret_cast<const float4*>(stage + rl * 32 + ((c4 ^ (rl & 7)) << 2));
           v[i][0] = t4.x + b4[0]; v[i][1] = t4.y + b4[1]; v[i][2] = t4.z + b4[2]; v[i][3] = t4.w + b4[3];
+        }
+        if constexpr (OUT_F32) {
+          if (rp) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              v[i][0] += res[i].x; v[i][1] += res[i].y; v[i][2] += res[i].z; v[i][3] += res[i].w;
+              res[i] = nxt[i];
+            }
+          }
         }
         if constexpr (EPI == SKY_EPI_GELU_BWD) {
 #pragma unroll
@@ -571,7 +608,7 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
                        cudaStream_t stream, float* colsum, float* colpart, size_t colpart_bytes,
-                       int* deferred_rows) {
+                       int* deferred_rows, const float* resid) {
   // TMA row pitches and the 16-byte epilogue stores need the contiguous
   // dimensions to be multiples of 8 elements; the token dimension is free.
   const bool dims_ok = N % 8 == 0 && (form == SKY_GEMM_XTW ? M % 8 == 0 : K % 8 == 0);
@@ -590,6 +627,9 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   SKY_CHECK(epi != SKY_EPI_BIAS_GELU || (bias && aux_out), SKY_ERR_INVALID_ARG,
             "BIAS_GELU epilogue needs bias and aux_out");
   SKY_CHECK(epi != SKY_EPI_GELU_BWD || aux, SKY_ERR_INVALID_ARG, "GELU' epilogue needs aux");
+  SKY_CHECK(!resid || (out_f32 && epi == SKY_EPI_STORE && !colsum && !deferred_rows &&
+                       (reinterpret_cast<uintptr_t>(resid) & 15) == 0),
+            SKY_ERR_UNSUPPORTED, "a residual needs a 16-byte aligned fp32 output of the STORE epilogue");
   const int sms = sm_count();
   SKY_CHECK(sms > 0, SKY_ERR_CUDA, "no CUDA device");
 
@@ -606,7 +646,7 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   p.m_tiles = ceil_div(M, pair ? 2 * BM : BM);
   p.n_tiles = ceil_div(N, BN);
   p.k_blocks = ceil_div(K, BK);
-  const bool may_split = out_f32 && epi == SKY_EPI_STORE && bias == nullptr;
+  const bool may_split = out_f32 && epi == SKY_EPI_STORE && bias == nullptr && resid == nullptr;
   p.splits = may_split ? choose_splits(p.m_tiles * p.n_tiles, p.k_blocks, pair ? sms / 2 : sms) : 1;
   if (p.splits > 1) {  // never more partials than the workspace holds
     const size_t cap = ws_bytes / (static_cast<size_t>(M) * N * sizeof(float));
@@ -631,6 +671,7 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
     if (deferred_rows) *deferred_rows = colpart_rows;
   }
   p.bias = static_cast<const __nv_bfloat16*>(bias);
+  p.resid = resid;
   p.aux = epi == SKY_EPI_GELU_BWD ? static_cast<const __half*>(aux) : nullptr;
   p.aux_out = static_cast<__half*>(aux_out);
   p.status = status;

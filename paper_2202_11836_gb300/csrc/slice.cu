@@ -231,7 +231,7 @@ struct Timed {
 sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, int M, int N,
                     int K, const void* A, const void* Bm, void* C, bool out_f32, int epi,
                     const void* bias, const void* aux, void* aux_out, float* colsum = nullptr,
-                    void* ws = nullptr, size_t ws_bytes = 0) {
+                    void* ws = nullptr, size_t ws_bytes = 0, const float* resid = nullptr) {
   Timed t(s, st, cat, 2.0 * M * N * K, 0);
   if (!ws) {
     ws = s->ws;
@@ -239,7 +239,7 @@ sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, 
   }
   if (s->cfg.dtype == SKY_DTYPE_BF16)
     return gemm::launch_bf16(form, M, N, K, A, Bm, C, out_f32, epi, bias, aux, aux_out, ws,
-                             ws_bytes, s->d_status, st, colsum);
+                             ws_bytes, s->d_status, st, colsum, nullptr, 0, nullptr, resid);
   return gemm::launch_f32(form, M, N, K, static_cast<const float*>(A),
                           static_cast<const float*>(Bm), static_cast<float*>(C), epi,
                           static_cast<const float*>(bias), static_cast<const float*>(aux),
@@ -268,35 +268,39 @@ sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
     Timed t(s, st, P_ATTN_FWD, 4.0 * H * S * (double)T, e * T * 4.0 * H);
     SKY_TRY(attention_fwd(Lb.QKV, s->d_len, B, S, H, A, dt, Lb.ctx, Lb.lse, s->d_status, st));
   }
-  // a3: U1 = ctx Wo^T + bo  (fp32; the residual is added by the LayerNorm)
+  // a3 + a4: U1 = ctx Wo^T + bo + X (fp32).  bf16: the residual X is added
+  // by the GEMM epilogue; fp32: by the LayerNorm.  X1 = LN(U1)
+  const bool bf = dt == SKY_DTYPE_BF16;
   SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, H, Lb.ctx, Lb.p[2], Lb.U1, true,
-                   SKY_EPI_STORE, Lb.p[3], nullptr, nullptr));
-  // a4: U1 += X; X1 = LN(U1)
+                   SKY_EPI_STORE, Lb.p[3], nullptr, nullptr, nullptr, nullptr, 0,
+                   bf ? Lb.X32 : nullptr));
   {
-    Timed t(s, st, P_LN_FWD, 0, 12.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
-    SKY_TRY(layernorm_fwd(Lb.U1, Lb.X32, Lb.p[4], Lb.p[5], T, H, s->cfg.ln_eps, dt, Lb.U1,
-                          dt == SKY_DTYPE_BF16 ? Lb.X1_32 : nullptr, Lb.X1b, Lb.mean1, Lb.rstd1,
-                          st));
+    Timed t(s, st, P_LN_FWD, 0, (bf ? 4.0 : 12.0) * T * H + (4.0 + e) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_fwd(Lb.U1, bf ? nullptr : Lb.X32, Lb.p[4], Lb.p[5], T, H, s->cfg.ln_eps,
+                          dt, bf ? nullptr : Lb.U1, bf ? Lb.X1_32 : nullptr, Lb.X1b, Lb.mean1,
+                          Lb.rstd1, st));
   }
   // a5 + a6: Z = X1 W1^T + b1; G = GELU(Z) and GELU'(Z) for the backward (fused epilogue)
   SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, F, H, Lb.X1b, Lb.p[6], Lb.G, false,
                    SKY_EPI_BIAS_GELU, Lb.p[7], nullptr, Lb.Gp));
-  // a7: U2 = G W2^T + b2  (fp32)
+  // a7 + a8: U2 = G W2^T + b2 + X1 (fp32; the residual as in a3).  Y = LN(U2)
+  // -> next layer's input (fp32 + dtype copy) or the caller's y
   SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, F, Lb.G, Lb.p[8], Lb.U2, true,
-                   SKY_EPI_STORE, Lb.p[9], nullptr, nullptr));
-  // a8: U2 += X1; Y = LN(U2) -> next layer's input (fp32 + dtype copy) or the caller's y
+                   SKY_EPI_STORE, Lb.p[9], nullptr, nullptr, nullptr, nullptr, 0,
+                   bf ? Lb.X1_32 : nullptr));
   {
-    Timed t(s, st, P_LN_FWD, 0, 12.0 * T * H + (4.0 + e) * T * H + 8.0 * T);
+    Timed t(s, st, P_LN_FWD, 0, (bf ? 4.0 : 12.0) * T * H + (4.0 + e) * T * H + 8.0 * T);
+    const float* r2 = bf ? nullptr : Lb.X1_32;
+    float* u2 = bf ? nullptr : Lb.U2;
     if (y_out) {
-      const bool f32 = dt == SKY_DTYPE_BF16 && s->cfg.io_fp32;
-      SKY_TRY(layernorm_fwd(Lb.U2, Lb.X1_32, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, Lb.U2,
+      const bool f32 = bf && s->cfg.io_fp32;
+      SKY_TRY(layernorm_fwd(Lb.U2, r2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, u2,
                             f32 ? static_cast<float*>(y_out) : nullptr, f32 ? nullptr : y_out,
                             Lb.mean2, Lb.rstd2, st));
     } else {
       LayerBufs& Nx = s->layers[i + 1];
-      SKY_TRY(layernorm_fwd(Lb.U2, Lb.X1_32, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, Lb.U2,
-                            dt == SKY_DTYPE_BF16 ? Nx.X32 : nullptr, Nx.Xb, Lb.mean2, Lb.rstd2,
-                            st));
+      SKY_TRY(layernorm_fwd(Lb.U2, r2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, u2,
+                            bf ? Nx.X32 : nullptr, Nx.Xb, Lb.mean2, Lb.rstd2, st));
     }
   }
   return SKY_OK;
