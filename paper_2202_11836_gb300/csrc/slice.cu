@@ -104,9 +104,10 @@ struct sky_slice {
   void* arena = nullptr;
   uint64_t param_bytes = 0, grad_bytes = 0, stash_bytes = 0, ws_bytes_total = 0;
   std::vector<sky::LayerBufs> layers;
-  // fp32 gradient stream.  Between layers it travels as two terms that the
-  // next LayerNorm backward adds: dP[k] (dQKV Wqkv) and dR[k] (dU1, the
-  // residual branch); k alternates per layer.
+  // fp32 gradient stream; k alternates per layer.  bf16: dP[k] holds the
+  // whole input gradient dQKV Wqkv + dU1 (the GEMM epilogue adds dR[k] = dU1).
+  // fp32: it travels as the two terms dP[k], dR[k] that the next LayerNorm
+  // backward adds.
   float *dP[2], *dR[2], *dU2_32, *dP1;
   void *dU2b, *dU1b, *dH, *dctx, *dqkv;           // dtype copies / branch gradients
   float* delta;
@@ -309,7 +310,8 @@ sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
 // ----------------------------------------------------------------- backward
 // One layer, steps a9..a16.  The upstream gradient is dY + dY2: dY in dy_dt
 // (the caller's dy for the top layer) and dY2 fp32 or null.  Outputs go to
-// dP[k] and dR[k]; for the slice's first layer they are added into dx.
+// dP[k] (bf16: the whole input gradient) and dR[k] (fp32: the second term);
+// for the slice's first layer they end in dx.
 sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, const float* dY2,
                           int k, void* dx, cudaStream_t st, cudaStream_t sw) {
   LayerBufs& Lb = s->layers[i];
@@ -382,17 +384,19 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, sw, P_COLSUM, 0, 4.0 * db1_rows * F);
     SKY_CUDA(gemm::reduce_rows_f32(s->db1p, db1_rows, F, Lb.g[7], sw));
   }
-  // a12: P1 = dZ W1 (fp32; dX1 = P1 + dU2 is formed by the LN1 backward);  dW1 = dZ^T X1
+  // a12: dX1 = dZ W1 + dU2 (fp32; bf16: dU2 added by the GEMM epilogue, fp32:
+  // by the LN1 backward);  dW1 = dZ^T X1
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dP1, true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
+                   SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, nullptr, 0,
+                   bf ? s->dU2_32 : nullptr));
   SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, F, H, T, s->dH, Lb.X1b, Lb.g[6], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
   SKY_TRY(done(1));
   // a13: LN1 backward of dX1 = P1 + dU2 -> dU1 (fp32 + dtype), dgamma1, dbeta1, dbo
   SKY_TRY(reuse(2));
   {
-    Timed t(s, st, P_LN_BWD, 0, (4.0 + 4.0 + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
-    SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? s->dU2_32 : static_cast<float*>(s->dU2b),
+    Timed t(s, st, P_LN_BWD, 0, (bf ? 4.0 : 8.0) * T * H + (4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? nullptr : static_cast<float*>(s->dU2b),
                           Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H, dt, bf ? s->dR[k] : nullptr,
                           dU1b, Lb.g[4], Lb.g[5], Lb.g[3], bf ? s->lnp[1] : s->ws,
                           bf ? s->lnp_bytes : s->ws_bytes, st, bf ? &ln_parts : nullptr));
@@ -418,14 +422,22 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], bf ? s->ws2 : s->ws,
                        bf ? s->ws2_bytes : s->ws_bytes, sw));
   }
-  // a16: dX = dQKV Wqkv + dU1 (the sum is formed by the next LayerNorm backward,
-  // or here for the slice's first layer);  dWqkv = dQKV^T X
-  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, 3 * H, s->dqkv, Lb.p[0], s->dP[k], true,
-                   SKY_EPI_STORE, nullptr, nullptr, nullptr));
-  if (dx) {
-    Timed t(s, st, P_COPY, 0, (8.0 + ((bf && !s->cfg.io_fp32) ? 2.0 : 4.0)) * T * H);
-    SKY_TRY(add_f32(s->dP[k], s->dR[k], (int64_t)T * H,
-                    s->cfg.io_fp32 ? SKY_DTYPE_FP32 : dt, dx, st));
+  // a16: dX = dQKV Wqkv + dU1;  dWqkv = dQKV^T X.  bf16: dU1 is added by the
+  // GEMM epilogue (straight into dx for the slice's first layer with fp32
+  // I/O); fp32: by the next LayerNorm backward, or here for the first layer
+  const bool direct = bf && dx && s->cfg.io_fp32 && (reinterpret_cast<uintptr_t>(dx) & 15) == 0;
+  SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, 3 * H, s->dqkv, Lb.p[0],
+                   direct ? dx : s->dP[k], true, SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr,
+                   nullptr, 0, bf ? s->dR[k] : nullptr));
+  if (dx && !direct) {
+    const sky_dtype odt = s->cfg.io_fp32 ? SKY_DTYPE_FP32 : dt;
+    Timed t(s, st, P_COPY, 0, ((bf ? 4.0 : 8.0) + (odt == SKY_DTYPE_BF16 ? 2.0 : 4.0)) * T * H);
+    if (!bf)
+      SKY_TRY(add_f32(s->dP[k], s->dR[k], (int64_t)T * H, odt, dx, st));
+    else if (odt == SKY_DTYPE_BF16)
+      SKY_TRY(f32_to_bf16(s->dP[k], (int64_t)T * H, dx, st));
+    else
+      SKY_CUDA(cudaMemcpyAsync(dx, s->dP[k], (size_t)T * H * 4, cudaMemcpyDeviceToDevice, st));
   }
   SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, 3 * H, H, T, s->dqkv, Lb.Xb, Lb.g[0], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
@@ -488,7 +500,7 @@ sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
       SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
     }
     cur = s->dP[k];
-    cur2 = s->dR[k];
+    cur2 = s->cfg.dtype == SKY_DTYPE_BF16 ? nullptr : s->dR[k];  // bf16: already in dP[k]
     cur_dt = SKY_DTYPE_FP32;
   }
   return join();
