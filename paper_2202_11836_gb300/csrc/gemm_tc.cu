@@ -10,7 +10,8 @@
 //               K=16) into a TMEM accumulator; two accumulators (512 TMEM
 //               columns) let the epilogue of one tile overlap the next,
 //   warps 2..9  epilogue (two warps per TMEM lane quarter, one per half of
-//               the tile's columns): tcgen05.ld of the accumulator, a
+//               the tile's columns; 2..17 and a quarter of the columns each
+//               for bias + GELU): tcgen05.ld of the accumulator, a
 //               transpose through shared memory so stores coalesce, fused
 //               bias / GELU, store to global memory.  The forward GELU
 //               epilogue also stores GELU'(z) (fp16); the backward epilogue
@@ -58,15 +59,19 @@ constexpr int PAIR_STAGE_BYTES = A_BYTES + (BN / 2) * BK * 2;
 static_assert(PAIR_STAGES * PAIR_STAGE_BYTES == STAGES * STAGE_BYTES, "same ring size");
 
 // Launch shape per instantiation: epilogue warps (a multiple of 4, one group
-// per TMEM lane quarter), ring stages and shared memory.
+// per TMEM lane quarter), epilogue chunk width, ring stages and shared memory.
+// The bias+GELU epilogue is bound by its own math: it runs 16 warps (four per
+// lane quarter, 64 columns each) on 16-column chunks, which keeps it at about
+// 100 registers a thread (576 threads leave 112).
 template <int EPI, bool PAIR>
 struct Shape {
-  static constexpr int EW = NUM_EPI_WARPS;
+  static constexpr int EW = EPI == SKY_EPI_BIAS_GELU ? 16 : NUM_EPI_WARPS;
+  static constexpr int CW = EW == 16 ? 16 : 32;              // epilogue chunk width (columns)
   static constexpr int THREADS = 64 + 32 * EW;
-  static constexpr int NST = PAIR ? PAIR_STAGES : (EW == 16 ? 3 : STAGES);
+  static constexpr int NST = PAIR ? PAIR_STAGES : STAGES;
   static constexpr int SBYTES = PAIR ? PAIR_STAGE_BYTES : STAGE_BYTES;
-  static constexpr int EPI_OFF = NST * SBYTES;               // per epilogue warp: 32 x 32 fp32 staging
-  static constexpr int BAR_OFF = EPI_OFF + EW * 32 * 32 * 4;
+  static constexpr int EPI_OFF = NST * SBYTES;               // per epilogue warp: 32 x CW fp32 staging
+  static constexpr int BAR_OFF = EPI_OFF + EW * 32 * CW * 4;
   static constexpr int SMEM = BAR_OFF + 256 /*barriers*/ + 1024 /*alignment slack*/;
   static_assert(SMEM <= 232448, "shared memory per CTA");
 };
@@ -281,7 +286,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
     // row's 32 columns, then the fused epilogue and coalesced stores.
     constexpr int HALF = BN / (EW / 4), CHUNKS = HALF / 32;  // columns of a warp, 32-column chunks
     const int q = warp & 3, hf = (warp - 2) >> 2;
-    float* stage = reinterpret_cast<float*>(smem + SH::EPI_OFF) + (warp - 2) * 32 * 32;
+    float* stage = reinterpret_cast<float*>(smem + SH::EPI_OFF) + (warp - 2) * 32 * SH::CW;
     const int c4 = lane & 7;          // this lane's 4-column group in a chunk
     const int rsub = lane >> 3;       // row within each group of 4 rows
     int acc = 0;
@@ -327,9 +332,51 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
       float* outf = OUT_F32 ? static_cast<float*>(p.C) +
                                   static_cast<int64_t>(split) * p.M * static_cast<int64_t>(p.N)
                             : nullptr;
-      // The GELU epilogue keeps its chunk loop rolled: unrolled, its
-      // straight-line code overflows the instruction cache.
-#pragma unroll (EPI == SKY_EPI_BIAS_GELU ? 1 : CHUNKS)
+      if constexpr (EPI == SKY_EPI_BIAS_GELU) {
+        // CW-column chunks: LPR lanes cover a row's CW columns, RPI rows per step
+        constexpr int CW = SH::CW, LPR = CW / 4, RPI = 32 / LPR, NI = 32 / RPI;
+        const int g4 = lane % LPR, grs = lane / LPR;
+        auto swz = [](int row) { return CW == 32 ? (row & 7) : ((row >> 1) & 3); };
+#pragma unroll 1
+        for (int c = 0; c < HALF; c += CW) {
+          uint32_t r[CW];
+          __syncwarp();
+          if constexpr (CW == 16) ptx::tmem_ld_32x32b_x16(taddr + c, *reinterpret_cast<uint32_t(*)[16]>(r));
+          else ptx::tmem_ld_32x32b_x32(taddr + c, *reinterpret_cast<uint32_t(*)[32]>(r));
+          ptx::tmem_ld_wait();
+          if (n0 + c >= p.N) continue;  // warp-uniform
+#pragma unroll
+          for (int j = 0; j < CW / 4; ++j)
+            *reinterpret_cast<float4*>(stage + lane * CW + ((j ^ swz(lane)) << 2)) =
+                make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                            __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+          __syncwarp();
+          const int col = n0 + c + 4 * g4;
+          if (col >= p.N) continue;
+          const uint2 braw = *reinterpret_cast<const uint2*>(p.bias + col);
+          const __nv_bfloat162* bh = reinterpret_cast<const __nv_bfloat162*>(&braw);
+          const float2 bf0 = __bfloat1622float2(bh[0]), bf1 = __bfloat1622float2(bh[1]);
+          const float b4[4] = {bf0.x, bf0.y, bf1.x, bf1.y};
+#pragma unroll
+          for (int i = 0; i < NI; ++i) {
+            const int rl = RPI * i + grs;
+            const float4 t4 = *reinterpret_cast<const float4*>(stage + rl * CW + ((g4 ^ swz(rl)) << 2));
+            float z[4] = {t4.x + b4[0], t4.y + b4[1], t4.z + b4[2], t4.w + b4[3]}, gp[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) gelu_and_grad_as(z[j], z[j], gp[j]);
+            const int row = m0 + q * 32 + rl;
+            if (row < p.M) {
+              const int64_t off = static_cast<int64_t>(row) * p.N + col;
+              const __half2 h0 = __floats2half2_rn(gp[0], gp[1]), h1 = __floats2half2_rn(gp[2], gp[3]);
+              *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.C) + off) =
+                  make_uint2(ptx::pack_bf16(z[0], z[1]), ptx::pack_bf16(z[2], z[3]));
+              *reinterpret_cast<uint2*>(p.aux_out + off) =
+                  make_uint2(*reinterpret_cast<const uint32_t*>(&h0), *reinterpret_cast<const uint32_t*>(&h1));
+            }
+          }
+        }
+      } else
+#pragma unroll CHUNKS
       for (int cc = 0; cc < CHUNKS; ++cc) {
         const int c = cc * 32;
         uint32_t r[32];
@@ -560,10 +607,8 @@ cudaError_t launch_form(int units, int sms, const CUtensorMap& ta, const CUtenso
   }
 }
 
-// The pair variant serves every problem with at least one full 256-row tile,
-// except the bias+GELU epilogue: that kernel is bound by its epilogue math,
-// and pairing makes each accumulator wait for the slower CTA's epilogue.
-bool use_pair(int M, int epi) { return M >= 2 * BM && epi != SKY_EPI_BIAS_GELU; }
+// The pair variant serves every problem with at least one full 256-row tile.
+bool use_pair(int M, int /*epi*/) { return M >= 2 * BM; }
 
 uint64_t g_timeout_ns = 2000000000ull;  // 2 s per wait
 int g_skip_loads = 0;
