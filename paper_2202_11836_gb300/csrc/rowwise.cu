@@ -237,36 +237,45 @@ __global__ void to_f32_kernel(const T* __restrict__ x, int64_t n, float* __restr
 // LayerNorm backward, streamed through shared memory (bf16 slices, H = 1024
 // or less, H % 256 == 0).  One persistent CTA per SM owns a contiguous block
 // of rows.  A producer thread keeps RING rows of (u, dy, dy2) in flight with
-// 1-D bulk copies into a shared-memory ring; 8 consumer warps take rows
-// round-robin, each lane holding 32 columns (four 8-wide chunks), compute
+// 1-D bulk copies into a shared-memory ring; 8 pairs of consumer warps take
+// rows round-robin, the two warps of a pair one half of the row's columns
+// each (16 per lane, two 8-wide chunks), and compute
 //   du = rstd * (g - mean(g) - xhat * mean(g * xhat)),  g = (dy + dy2) * gamma
-// and keep the column sums of dy*xhat, dy and du in registers.  At the end
-// the 8 warps' sums are added in order into part[k][blockIdx.x][:].
-constexpr int SB_WARPS = 8, SB_RING = 16, SB_NV = 4;  // 32 columns per lane: H <= 1024
-constexpr int SB_ROW_BYTES = 3 * 1024 * 4;            // u, dy, dy2 (fp32 capacity)
+// The pair adds its two halves' row sums in a fixed order through shared
+// memory (one named barrier per row), and each warp keeps the column sums of
+// dy*xhat, dy and du for its columns in registers -- 48 a lane, which lets 16
+// consumer warps share an SM.  At the end the 8 pairs' sums are added in
+// order into part[k][blockIdx.x][:].
+constexpr int SB_PAIRS = 8, SB_WARPS = 2 * SB_PAIRS, SB_RING = 16, SB_NV = 2;  // H <= 1024
+constexpr int SB_ROW_BYTES = 3 * 1024 * 4;                                     // u, dy, dy2 (fp32)
 
-// part[k][blockIdx.x][:] = sum over the consumer warps (in order) of acc.
+// part[k][blockIdx.x][:] = sum over the consumer pairs (in order) of acc.
 __device__ __forceinline__ void sb_flush(const float (&acc)[SB_NV][8], int k, float* red,
                                          float* __restrict__ part, int H) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp < SB_WARPS) {
+    const int pr = warp >> 1, hh = warp & 1, half = H / 2;
 #pragma unroll
     for (int c = 0; c < SB_NV; ++c) {
       const int col = (c * 32 + lane) * 8;
-      if (col < H) store8(red + warp * H + col, acc[c]);
+      if (col < half) store8(red + pr * H + hh * half + col, acc[c]);
     }
   }
   __syncthreads();
   for (int col = threadIdx.x; col < H; col += blockDim.x) {
     float s = 0.f;
-    for (int w = 0; w < SB_WARPS; ++w) s += red[w * H + col];
+    for (int w = 0; w < SB_PAIRS; ++w) s += red[w * H + col];
     part[(static_cast<int64_t>(k) * gridDim.x + blockIdx.x) * H + col] = s;
   }
   __syncthreads();
 }
 
+__device__ __forceinline__ void pair_sync(int pair) {
+  asm volatile("bar.sync %0, 64;" ::"r"(1 + pair) : "memory");
+}
+
 template <typename TDY>
-__global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
+__global__ void __launch_bounds__(32 * (SB_WARPS + 1), 1) ln_bwd_stream_kernel(
     const TDY* __restrict__ dy, const float* __restrict__ dy2, const float* __restrict__ u,
     const __nv_bfloat16* __restrict__ gamma, const float* __restrict__ mean,
     const float* __restrict__ rstd, int rows, int H, float* __restrict__ du32,
@@ -277,7 +286,9 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
   uint8_t* sm = sm_raw + ((128 - (ptx::smem_u32(sm_raw) & 127)) & 127);
   uint64_t* full = reinterpret_cast<uint64_t*>(sm + SB_RING * SB_ROW_BYTES);
   uint64_t* empty = full + SB_RING;
-  float* sgm = reinterpret_cast<float*>(empty + SB_RING);  // gamma as fp32 [H]
+  // per pair, row parity and half: {partial sum of g, of g * xhat, ok flag}
+  float* xch = reinterpret_cast<float*>(empty + SB_RING);
+  float* sgm = xch + SB_PAIRS * 2 * 2 * 4;  // gamma as fp32 [H]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int per = (rows + gridDim.x - 1) / gridDim.x;
   const int r0 = blockIdx.x * per, r1 = min(rows, r0 + per);
@@ -288,7 +299,7 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
   if (threadIdx.x == 0) {
     for (int s = 0; s < SB_RING; ++s) {
       ptx::mbar_init(&full[s], 1);
-      ptx::mbar_init(&empty[s], 32);
+      ptx::mbar_init(&empty[s], 64);  // the two warps of the row's pair
     }
     ptx::fence_mbar_init();
     ptx::fence_proxy_async_smem();
@@ -315,17 +326,18 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
         ptx::mbar_wait(&full[i % SB_RING], (i / SB_RING) & 1, lim, status, 5000);
   } else {
     const float invH = 1.f / H;
-    for (int i = warp; i < n; i += SB_WARPS) {
+    const int pr = warp >> 1, hh = warp & 1, half = H / 2;
+    for (int i = pr, it = 0; i < n; i += SB_PAIRS, ++it) {
       const int s = i % SB_RING;
       const int64_t row = r0 + i;
       const float mu = mean[row], rs = rstd[row];
-      const bool ok = ptx::mbar_wait(&full[s], (i / SB_RING) & 1, lim, status, 5000);
-      if (!__all_sync(0xffffffffu, ok)) break;
+      const bool ok = __all_sync(0xffffffffu, ptx::mbar_wait(&full[s], (i / SB_RING) & 1, lim, status, 5000));
       const uint8_t* slot = sm + s * SB_ROW_BYTES;
-      const float* su = reinterpret_cast<const float*>(slot);
-      const TDY* sdy = reinterpret_cast<const TDY*>(slot + 4096);
-      const float* sd2 = reinterpret_cast<const float*>(slot + 8192);
-      // x-hat and dy (+ dy2) of 8 columns, read from the slot
+      const float* su = reinterpret_cast<const float*>(slot) + hh * half;
+      const TDY* sdy = reinterpret_cast<const TDY*>(slot + 4096) + hh * half;
+      const float* sd2 = reinterpret_cast<const float*>(slot + 8192) + hh * half;
+      const float* sg = sgm + hh * half;
+      // x-hat and dy (+ dy2) of 8 columns of this warp's half, read from the slot
       auto fetch = [&](int col, float (&xh)[8], float (&d)[8]) {
         load8(su + col, xh);
         load8(sdy + col, d);
@@ -342,10 +354,10 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
 #pragma unroll
       for (int c = 0; c < SB_NV; ++c) {
         const int col = (c * 32 + lane) * 8;
-        if (col < H) {
+        if (col < half) {
           float xh[8], d[8], gm[8];
           fetch(col, xh, d);
-          load8(sgm + col, gm);
+          load8(sg + col, gm);
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             const float g = d[k] * gm[k];
@@ -354,15 +366,26 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
           }
         }
       }
-      const float mg = warp_sum(s1) * invH, mgx = warp_sum(s2) * invH;
+      s1 = warp_sum(s1);
+      s2 = warp_sum(s2);
+      // the pair's two halves, added in a fixed order (low half first)
+      float* xp = xch + ((pr * 2 + (it & 1)) * 2) * 4;
+      if (lane == 0) {
+        xp[hh * 4 + 0] = s1;
+        xp[hh * 4 + 1] = s2;
+        xp[hh * 4 + 2] = ok ? 1.f : 0.f;
+      }
+      pair_sync(pr);
+      if (xp[2] == 0.f || xp[4 + 2] == 0.f) break;  // either warp timed out: the pair stops
+      const float mg = (xp[0] + xp[4]) * invH, mgx = (xp[1] + xp[4 + 1]) * invH;
       // second pass re-reads the slot instead of holding the row in registers
 #pragma unroll
       for (int c = 0; c < SB_NV; ++c) {
         const int col = (c * 32 + lane) * 8;
-        if (col < H) {
+        if (col < half) {
           float xh[8], d[8], gm[8], o[8];
           fetch(col, xh, d);
-          load8(sgm + col, gm);
+          load8(sg + col, gm);
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             o[k] = rs * (d[k] * gm[k] - mg - xh[k] * mgx);
@@ -370,18 +393,19 @@ __global__ void __launch_bounds__(288, 1) ln_bwd_stream_kernel(
             pb[c][k] += d[k];
             pu[c][k] += o[k];
           }
-          if (du32) store8(du32 + row * H + col, o);
-          if (duT) store8(duT + row * H + col, o);
+          const int64_t off = row * H + hh * half + col;
+          if (du32) store8(du32 + off, o);
+          if (duT) store8(duT + off, o);
         }
       }
       __syncwarp();
-      ptx::mbar_arrive(&empty[s]);  // slot s may be refilled
+      ptx::mbar_arrive(&empty[s]);  // slot s may be refilled once both warps are done
     }
   }
   // every row's copy has landed and been consumed: the ring is free for the
-  // CTA's fixed-order reduction of the 8 warps' column sums
+  // CTA's fixed-order reduction of the 8 pairs' column sums
   __syncthreads();
-  float* red = reinterpret_cast<float*>(sm);  // [SB_WARPS][H]
+  float* red = reinterpret_cast<float*>(sm);  // [SB_PAIRS][H]
   sb_flush(pg, 0, red, part, H);
   sb_flush(pb, 1, red, part, H);
   sb_flush(pu, 2, red, part, H);
@@ -578,9 +602,11 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
   if (dt == SKY_DTYPE_BF16 && H <= 1024 && H % 256 == 0 && rw::stream_blocks() <= nblk) {
     // streamed variant: one CTA per SM, rows staged through shared memory
     const int sb = rw::stream_blocks();
-    const size_t smem = (size_t)rw::SB_RING * rw::SB_ROW_BYTES + 2 * rw::SB_RING * 8 + (size_t)H * 4 + 128;
+    const size_t fixed = (size_t)rw::SB_RING * rw::SB_ROW_BYTES + 2 * rw::SB_RING * 8 +
+                         (size_t)rw::SB_PAIRS * 2 * 2 * 4 * 4 + 128;
+    const size_t smem = fixed + (size_t)H * 4;
     // the attribute is set once, for the largest H this variant takes
-    const size_t smem_max = (size_t)rw::SB_RING * rw::SB_ROW_BYTES + 2 * rw::SB_RING * 8 + 1024 * 4 + 128;
+    const size_t smem_max = fixed + 1024 * 4;
     const int threads = 32 * (rw::SB_WARPS + 1);
     if (dy_dt == SKY_DTYPE_BF16) {
       static cudaError_t a = cudaFuncSetAttribute(rw::ln_bwd_stream_kernel<__nv_bfloat16>,
