@@ -192,7 +192,8 @@ sky_status attention_fwd_tc(const void* qkv, const int32_t* lens, int B, int S, 
 
 sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse, const float* delta,
                             const int32_t* lens, int B, int S, int H, int A, void* dqkv,
-                            int32_t* status, uint64_t timeout_ns, cudaStream_t stream);
+                            int32_t* status, uint64_t timeout_ns, cudaStream_t stream,
+                            float* colpart);
 
 sky_status attention_fwd(const void* qkv, const int32_t* lens, int B, int S, int H, int A,
                          sky_dtype dt, void* ctx, float* lse, int32_t* status,
@@ -220,7 +221,7 @@ size_t attention_bwd_ws(int B, int S, int A) { return (size_t)B * A * S * sizeof
 
 sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, const float* lse,
                          const int32_t* lens, int B, int S, int H, int A, sky_dtype dt, void* dqkv,
-                         float* delta, int32_t* status, cudaStream_t stream) {
+                         float* delta, int32_t* status, cudaStream_t stream, float* colpart) {
   const int D = H / A;
   const int64_t rows = (int64_t)B * S;
   const int dblocks = ceil_div(rows * A * 32, 256);
@@ -232,7 +233,7 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
     count_launches(1);
     if (le != cudaSuccess) return cuda_fail(le, "attention delta launch");
     return attention_bwd_tc(qkv, dctx, lse, delta, lens, B, S, H, A, dqkv, status, 2000000000ull,
-                            stream);
+                            stream, colpart);
   } else {
     SKY_CHECK(D <= 128, SKY_ERR_UNSUPPORTED, "fp32 attention needs head dim <= 128");
     attn::attn_delta<float><<<dblocks, 256, 0, stream>>>(static_cast<const float*>(ctx),

@@ -343,9 +343,36 @@ struct BwdParams {
   const float* lse;
   const float* delta;
   __nv_bfloat16* dqkv;
+  // optional: column sums of the stored dQKV, one row per 128-row tile of a
+  // sequence: colpart[b * ceil(S/128) + tile][3H]
+  float* colpart;
   int32_t* status;
   uint64_t timeout_ns;
 };
+
+// v[j] of lane l -> after the call, v[0] of lane l holds the sum over the
+// warp's 32 lanes of v[l]: a butterfly in which every lane keeps the half of
+// its columns given by its lane bit and receives the partner's half (31
+// shuffles for 32 columns).
+__device__ __forceinline__ void lanes_column_sum(float (&v)[32], int lane) {
+#pragma unroll
+  for (int k = 16; k >= 1; k >>= 1) {
+    const bool upper = (lane & k) != 0;
+#pragma unroll
+    for (int j = 0; j < k; ++j) {
+      const float send = upper ? v[j] : v[j + k];
+      const float keep = upper ? v[j + k] : v[j];
+      v[j] = keep + __shfl_xor_sync(0xffffffffu, send, k);
+    }
+  }
+}
+__device__ __forceinline__ float bf16_round(float x) {
+  return __bfloat162float(__float2bfloat16_rn(x));
+}
+// The 8 softmax warps of a backward kernel (256 threads) meet here.
+__device__ __forceinline__ void softmax_warps_sync() {
+  asm volatile("bar.sync 1, 256;" ::: "memory");
+}
 
 __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorMap tmQ,
                                                           const __grid_constant__ CUtensorMap tmKV,
@@ -548,6 +575,7 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
       ptx::mbar_arrive(ds_full);
     }
     // epilogue: each half writes 32 of the 64 dQ columns
+    float* red = reinterpret_cast<float*>(smem + DQ_KV_OFF);  // [4 row quarters][64]: ring is idle
     if (ok && wait_all(dq_done, (n_kt - 1) & 1)) {
       ptx::tc_fence_after();
       __nv_bfloat16* out = p.dqkv + (static_cast<int64_t>(row0) + q) * (3 * H) + a * HD + hf * 32;
@@ -564,6 +592,23 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
                                   __uint_as_float(o[8 * u + 2 * t + 1]) * 0.125f);
           *reinterpret_cast<uint4*>(out + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
         }
+      }
+      if (p.colpart) {  // column sums of the stored values over this warp's 32 rows
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = q < S ? bf16_round(__uint_as_float(o[j]) * 0.125f) : 0.f;
+        lanes_column_sum(v, lane);
+        red[q4 * 64 + hf * 32 + lane] = v[0];
+      }
+    } else if (p.colpart) {
+      red[q4 * 64 + hf * 32 + lane] = 0.f;
+    }
+    if (p.colpart) {  // the four row quarters, added in order, by the quarter-0 warps
+      softmax_warps_sync();
+      if (q4 == 0) {
+        const int c = hf * 32 + lane;
+        const float sum = ((red[c] + red[64 + c]) + red[128 + c]) + red[192 + c];
+        p.colpart[(static_cast<int64_t>(b) * gridDim.x + qt) * (3 * H) + a * HD + c] = sum;
       }
     }
   }
@@ -626,6 +671,10 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
         *reinterpret_cast<uint4*>(base + H) = make_uint4(0, 0, 0, 0);
         *reinterpret_cast<uint4*>(base + 2 * H) = make_uint4(0, 0, 0, 0);
       }
+    }
+    if (p.colpart && threadIdx.x < 2 * HD) {  // and zero column sums
+      const int hf = threadIdx.x / HD, c = threadIdx.x % HD;
+      p.colpart[(static_cast<int64_t>(b) * gridDim.x + kt) * rs + (1 + hf) * H + a * HD + c] = 0.f;
     }
     return;
   }
@@ -854,6 +903,7 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
       ptx::mbar_arrive(pds_full);
     }
     // epilogue: the low-half warps write dK / sqrt(D), the high-half warps dV
+    float* red = reinterpret_cast<float*>(smem + KV_P_OFF);  // [2 halves][4 quarters][64]: P^T is idle
     if (ok && wait_all(mm_done, (n_qt - 1) & 1)) {
       ptx::tc_fence_after();
       const uint32_t tacc = hf == 0 ? tdK : tdV;
@@ -875,6 +925,29 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
                                     __uint_as_float(o[c][8 * u + 2 * t + 1]) * sc);
             *reinterpret_cast<uint4*>(out + c * 32 + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
           }
+      }
+      if (p.colpart) {  // column sums of the stored values over this warp's 32 rows
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          float v[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = key < S ? bf16_round(__uint_as_float(o[c][j]) * sc) : 0.f;
+          lanes_column_sum(v, lane);
+          red[(hf * 4 + q4) * 64 + c * 32 + lane] = v[0];
+        }
+      }
+    } else if (p.colpart) {
+      red[(hf * 4 + q4) * 64 + lane] = 0.f;
+      red[(hf * 4 + q4) * 64 + 32 + lane] = 0.f;
+    }
+    if (p.colpart) {  // the four row quarters, added in order, by the quarter-0 warps
+      softmax_warps_sync();
+      if (q4 == 0) {
+        const float* rh = red + hf * 4 * 64;
+        float* dst = p.colpart + (static_cast<int64_t>(b) * gridDim.x + kt) * rs + (1 + hf) * H + a * HD;
+#pragma unroll
+        for (int c = lane; c < 64; c += 32)
+          dst[c] = ((rh[c] + rh[64 + c]) + rh[128 + c]) + rh[192 + c];
       }
     }
   }
@@ -942,7 +1015,8 @@ sky_status attention_fwd_tc(const void* qkv, const int32_t* lens, int B, int S, 
 // Backward launchers (bf16, D = 64): delta must already hold rowsum(dO * O).
 sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse, const float* delta,
                             const int32_t* lens, int B, int S, int H, int A, void* dqkv,
-                            int32_t* status, uint64_t timeout_ns, cudaStream_t stream) {
+                            int32_t* status, uint64_t timeout_ns, cudaStream_t stream,
+                            float* colpart) {
   using namespace attn_tc;
   SKY_CHECK(H == A * HD, SKY_ERR_UNSUPPORTED, "tensor-core attention needs head dim 64");
   const int64_t T = static_cast<int64_t>(B) * S;
@@ -957,7 +1031,8 @@ sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse,
   if (a2 != cudaSuccess) return cuda_fail(a2, "attention dK/dV smem attribute");
   const int bulk = (S % 4 == 0) && (reinterpret_cast<uintptr_t>(lse) & 15) == 0 &&
                    (reinterpret_cast<uintptr_t>(delta) & 15) == 0;
-  BwdParams p{S, H, A, bulk, lens, lse, delta, static_cast<__nv_bfloat16*>(dqkv), status, timeout_ns};
+  BwdParams p{S, H, A, bulk, lens, lse, delta, static_cast<__nv_bfloat16*>(dqkv), colpart, status,
+              timeout_ns};
   cudaError_t e = launch_pdl(attn_bwd_dkdv_tc, dim3(ceil_div(S, BK2), A, B), dim3(NTHR_B), KV_SMEM,
                              stream, 1, tk128, tq64, to64, p);
   if (e == cudaSuccess)

@@ -9,9 +9,11 @@ namespace sky {
 sky_status attention_fwd(const void* qkv, const int32_t* lens, int B, int S, int H, int A,
                          sky_dtype dt, void* ctx, float* lse, int32_t* status, cudaStream_t st);
 size_t attention_bwd_ws(int B, int S, int A);
+// colpart (bf16 only, optional): column sums of the stored dqkv, one row per
+// 128-row tile of each sequence: colpart[b * ceil(S/128) + tile][3H].
 sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, const float* lse,
                          const int32_t* lens, int B, int S, int H, int A, sky_dtype dt, void* dqkv,
-                         float* delta, int32_t* status, cudaStream_t st);
+                         float* delta, int32_t* status, cudaStream_t st, float* colpart = nullptr);
 
 sky_status layernorm_fwd(const float* a, const float* r, const void* gamma, const void* beta,
                          int rows, int H, float eps, sky_dtype dt, float* u_out, float* y32,

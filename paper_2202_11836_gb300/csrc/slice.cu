@@ -130,6 +130,11 @@ struct sky_slice {
   size_t lnp_bytes = 0;
   float* db1p = nullptr;
   size_t db1p_bytes = 0;
+  // column partials of dQKV written by the attention backward kernels (one
+  // row per 128-row tile of every sequence), summed into dbqkv on the side
+  // stream
+  float* qkvp = nullptr;
+  size_t qkvp_bytes = 0;
   // local parameter update (Sec. III): fp32 master weights and state in one
   // allocation, the tensor and chunk tables the update kernel walks
   bool opt_ready = false;
@@ -414,13 +419,16 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   {
     Timed t(s, st, P_ATTN_BWD, 8.0 * H * S * (double)T, e * T * 8.0 * H);
     SKY_TRY(attention_bwd(Lb.QKV, Lb.ctx, s->dctx, Lb.lse, s->d_len, B, S, H, A, dt, s->dqkv,
-                          s->delta, s->d_status, st));
+                          s->delta, s->d_status, st, bf ? s->qkvp : nullptr));
   }
   SKY_TRY(fork(3));
-  {  // dbqkv = column sums of dQKV (on sw for bf16, with sw's scratch)
+  if (bf) {  // dbqkv = the attention kernels' column partials, added in order (on sw)
+    const int rows = B * ceil_div(S, 128);
+    Timed t(s, sw, P_COLSUM, 0, 4.0 * rows * 3.0 * H);
+    SKY_CUDA(gemm::reduce_rows_f32(s->qkvp, rows, 3 * H, Lb.g[1], sw));
+  } else {  // dbqkv = column sums of dQKV
     Timed t(s, sw, P_COLSUM, 0, e * T * 3.0 * H);
-    SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], bf ? s->ws2 : s->ws,
-                       bf ? s->ws2_bytes : s->ws_bytes, sw));
+    SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], s->ws, s->ws_bytes, sw));
   }
   // a16: dX = dQKV Wqkv + dU1;  dWqkv = dQKV^T X.  bf16: dU1 is added by the
   // GEMM epilogue (straight into dx for the slice's first layer with fp32
@@ -600,11 +608,12 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   s->ws2_bytes = bf ? align_up(side_workspace_need(s, T)) : 0;
   s->lnp_bytes = bf ? align_up(layernorm_bwd_ws((int)T, s->H)) : 0;
   s->db1p_bytes = bf ? align_up((size_t)gemm::colpart_rows_max((int)T) * s->F * 4) : 0;
+  s->qkvp_bytes = bf ? align_up((size_t)c.max_batch * ceil_div(c.max_seq, 128) * 3 * s->H * 4) : 0;
   // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | ws2 | lnp[2] |
-  // db1p | status
+  // db1p | qkvp | status
   const size_t wk = 6 * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
                     align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes +
-                    s->ws2_bytes + 2 * s->lnp_bytes + s->db1p_bytes + 256;
+                    s->ws2_bytes + 2 * s->lnp_bytes + s->db1p_bytes + s->qkvp_bytes + 256;
   s->ws_bytes_total = wk;
   *total = s->param_bytes + s->grad_bytes + s->stash_bytes + wk;
   return SKY_OK;
@@ -716,6 +725,7 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
     s->lnp[1] = take(s->lnp_bytes);
   }
   if (s->db1p_bytes) s->db1p = static_cast<float*>(take(s->db1p_bytes));
+  if (s->qkvp_bytes) s->qkvp = static_cast<float*>(take(s->qkvp_bytes));
   s->d_status = static_cast<int32_t*>(take(4));
   if (bf) {
     // the weight-gradient side stream and its events
