@@ -61,20 +61,19 @@ __device__ __forceinline__ float gelu_grad_f(float h) {
 
 // GELU(h) and GELU'(h) together, for the tensor-core epilogues: Phi from the
 // erf approximation of Abramowitz & Stegun, Handbook of Mathematical
-// Functions, formula 7.1.26 (|erf error| <= 1.5e-7 for all x), written for
+// Functions, formula 7.1.25 (|erf error| <= 2.5e-5 for all x: well below the
+// bf16 rounding of GELU and the fp16 rounding of GELU'), written for
 // x = |h| / sqrt 2 so that Phi and phi share one exponential exp(-h^2 / 2):
-//   t = 1 / (1 + p x),  Phi(-|h|) = (1/2)(a1 t + ... + a5 t^5) exp(-h^2/2).
+//   t = 1 / (1 + p x),  Phi(-|h|) = (1/2)(a1 t + a2 t^2 + a3 t^3) exp(-h^2/2).
 // The 1/2 is folded into the coefficients and 1/sqrt 2 into p; the
 // reciprocal and the exponential use the hardware approximations (relative
-// error of a few ulp, far below the bf16 / fp16 rounding of the results).
+// error of a few ulp).  The epilogue is bound by this arithmetic, so the
+// three-term formula (two FMAs fewer than the five-term 7.1.26) pays.
 __device__ __forceinline__ void gelu_and_grad_as(float h, float& g, float& gp) {
   float t, E;
-  const float den = fmaf(fabsf(h), 0.3275911f * 0.70710678118654752f, 1.f);
+  const float den = fmaf(fabsf(h), 0.47047f * 0.70710678118654752f, 1.f);
   asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(t) : "f"(den));
-  const float q_poly =
-      t * (0.5f * 0.254829592f +
-           t * (0.5f * -0.284496736f +
-                t * (0.5f * 1.421413741f + t * (0.5f * -1.453152027f + t * (0.5f * 1.061405429f)))));
+  const float q_poly = t * (0.5f * 0.3480242f + t * (0.5f * -0.0958798f + t * (0.5f * 0.7478556f)));
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(E) : "f"((h * -0.72134752044448170f) * h));  // exp(-h^2/2)
   const float q = q_poly * E;  // Phi(-|h|)
   const float Phi = h >= 0.f ? 1.f - q : q;
