@@ -134,8 +134,10 @@ sky_status sky_slice_get_grads(sky_slice* s, int32_t layer, void* const* tensors
  * x, y: device [B,S,H] in the boundary dtype (the slice dtype, or fp32 with
  * io_fp32; may not alias); d_len: device
  * int32[B], each in [1,S] (checked on the device: a bad length is clamped,
- * and reported as INVALID_ARG by the next synchronising call).  x is copied
- * into the stash, so the caller may reuse it once the stream has passed it.
+ * and reported as INVALID_ARG by the next synchronising call).  The stash
+ * keeps everything the backward needs, so x may be reused once the forward's
+ * work on `stream` is done (a bf16 slice with fp32 boundary tensors reads a
+ * 16-byte aligned x in place as the first layer's residual until then).
  * Enqueues work on `stream`; no host synchronisation.
  * Errors: INVALID_ARG (B > max_batch, S > max_seq, B or S < 1, null). */
 sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,

@@ -15,12 +15,23 @@ namespace gemm {
 // possibly on another stream ordered after this launch).
 // resid (optional, fp32 output of the STORE epilogue, no split): C = acc +
 // bias + resid[m, n], added in that order (the residual branch of Sec. II-C).
+// With `ln`, resid holds the pre-LayerNorm sum u of the previous sub-layer and
+// the residual added is its LayerNorm output, recomputed in the epilogue from
+// the row statistics: gamma[n] * ((u[m, n] - mean[m]) * rstd[m]) + beta[n]
+// (Eq. 3; the same expression the LayerNorm forward evaluates, so the sum is
+// the one an fp32 copy of the LayerNorm output would give).
+struct LnResid {
+  const float* mean;  // [M]
+  const float* rstd;  // [M]
+  const void* gamma;  // [N] bf16
+  const void* beta;   // [N] bf16
+};
 sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, const void* B,
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
                        cudaStream_t stream, float* colsum = nullptr, float* colpart = nullptr,
                        size_t colpart_bytes = 0, int* deferred_rows = nullptr,
-                       const float* resid = nullptr);
+                       const float* resid = nullptr, const LnResid* ln = nullptr);
 // Rows of column partials a bf16 GEMM with M rows writes (upper bound).
 int colpart_rows_max(int M);
 // out[n] = sum over r of part[r][n] in order r = 0, 1, ... (rowwise.cu).

@@ -86,6 +86,10 @@ struct Params {
   __half* aux_out;                // [M,N] GELU'(z) (BIAS_GELU) or null
   float* colpart;                 // [m_tiles * 4][N] per-warp column sums of C, or null
   const float* resid;             // [M,N] fp32 added after the bias (fp32 outputs), or null
+  const float* ln_mean;           // [M] with ln_rstd, ln_gamma, ln_beta: resid is the
+  const float* ln_rstd;           //   pre-LayerNorm sum u and LN(u) is added, or null
+  const __nv_bfloat16* ln_gamma;  // [N]
+  const __nv_bfloat16* ln_beta;   // [N]
   int32_t* status;
   uint64_t timeout_ns;
   int skip_loads;                 // fault injection: producer never issues TMA
@@ -326,6 +330,20 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
       if constexpr (OUT_F32) {
         if (rp) load_res(0, res);
       }
+      // LayerNorm residual: this lane's 8 rows' statistics (the same rows in
+      // every chunk)
+      const bool ln = OUT_F32 && rp && p.ln_mean;
+      float mu[OUT_F32 ? 8 : 1], rs[OUT_F32 ? 8 : 1];
+      if constexpr (OUT_F32) {
+        if (ln) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int row = m0 + q * 32 + 4 * i + rsub;
+            mu[i] = row < p.M ? __ldg(p.ln_mean + row) : 0.f;
+            rs[i] = row < p.M ? __ldg(p.ln_rstd + row) : 0.f;
+          }
+        }
+      }
       if (!ptx::mbar_wait(&tfull[acc], aphase, lim, p.status, kSleepNs)) break;
       ptx::tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN + hf * HALF;
@@ -414,7 +432,26 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
           v[i][0] = t4.x + b4[0]; v[i][1] = t4.y + b4[1]; v[i][2] = t4.z + b4[2]; v[i][3] = t4.w + b4[3];
         }
         if constexpr (OUT_F32) {
-          if (rp) {
+          if (ln) {
+            float g4[4] = {0.f, 0.f, 0.f, 0.f}, e4[4] = {0.f, 0.f, 0.f, 0.f};
+            if (col_ok) {
+              const uint2 gr = *reinterpret_cast<const uint2*>(p.ln_gamma + col);
+              const uint2 er = *reinterpret_cast<const uint2*>(p.ln_beta + col);
+              const __nv_bfloat162* gh = reinterpret_cast<const __nv_bfloat162*>(&gr);
+              const __nv_bfloat162* eh = reinterpret_cast<const __nv_bfloat162*>(&er);
+              const float2 g0 = __bfloat1622float2(gh[0]), g1 = __bfloat1622float2(gh[1]);
+              const float2 e0 = __bfloat1622float2(eh[0]), e1 = __bfloat1622float2(eh[1]);
+              g4[0] = g0.x; g4[1] = g0.y; g4[2] = g1.x; g4[3] = g1.y;
+              e4[0] = e0.x; e4[1] = e0.y; e4[2] = e1.x; e4[3] = e1.y;
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const float u4[4] = {res[i].x, res[i].y, res[i].z, res[i].w};
+#pragma unroll
+              for (int j = 0; j < 4; ++j) v[i][j] += g4[j] * ((u4[j] - mu[i]) * rs[i]) + e4[j];
+              res[i] = nxt[i];
+            }
+          } else if (rp) {
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
               v[i][0] += res[i].x; v[i][1] += res[i].y; v[i][2] += res[i].z; v[i][3] += res[i].w;
@@ -653,7 +690,7 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
                        void* C, bool out_f32, int epi, const void* bias, const void* aux,
                        void* aux_out, void* ws, size_t ws_bytes, int32_t* status,
                        cudaStream_t stream, float* colsum, float* colpart, size_t colpart_bytes,
-                       int* deferred_rows, const float* resid) {
+                       int* deferred_rows, const float* resid, const LnResid* ln) {
   // TMA row pitches and the 16-byte epilogue stores need the contiguous
   // dimensions to be multiples of 8 elements; the token dimension is free.
   const bool dims_ok = N % 8 == 0 && (form == SKY_GEMM_XTW ? M % 8 == 0 : K % 8 == 0);
@@ -675,6 +712,10 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   SKY_CHECK(!resid || (out_f32 && epi == SKY_EPI_STORE && !colsum && !deferred_rows &&
                        (reinterpret_cast<uintptr_t>(resid) & 15) == 0),
             SKY_ERR_UNSUPPORTED, "a residual needs a 16-byte aligned fp32 output of the STORE epilogue");
+  SKY_CHECK(!ln || (resid && ln->mean && ln->rstd && ln->gamma && ln->beta &&
+                    (reinterpret_cast<uintptr_t>(ln->gamma) & 7) == 0 &&
+                    (reinterpret_cast<uintptr_t>(ln->beta) & 7) == 0),
+            SKY_ERR_INVALID_ARG, "a LayerNorm residual needs u, mean, rstd and 8-byte aligned gamma, beta");
   const int sms = sm_count();
   SKY_CHECK(sms > 0, SKY_ERR_CUDA, "no CUDA device");
 
@@ -717,6 +758,12 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   }
   p.bias = static_cast<const __nv_bfloat16*>(bias);
   p.resid = resid;
+  if (ln) {
+    p.ln_mean = ln->mean;
+    p.ln_rstd = ln->rstd;
+    p.ln_gamma = static_cast<const __nv_bfloat16*>(ln->gamma);
+    p.ln_beta = static_cast<const __nv_bfloat16*>(ln->beta);
+  }
   p.aux = epi == SKY_EPI_GELU_BWD ? static_cast<const __half*>(aux) : nullptr;
   p.aux_out = static_cast<__half*>(aux_out);
   p.status = status;

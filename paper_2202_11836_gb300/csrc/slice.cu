@@ -82,14 +82,15 @@ static const char* kCatNames[P_NCAT] = {"gemm_fwd", "gemm_dgrad", "gemm_wgrad", 
                                         "attn_bwd", "ln_fwd", "ln_bwd", "colsum", "copy"};
 
 // Per-layer parameters, gradients and the activation stash.  The residual
-// stream (layer input X, the residual sums U1 and U2, the LayerNorm output X1)
-// is kept in fp32; tensors that feed a bf16 contraction have a copy in the
-// slice dtype (for fp32 slices the two are the same buffer).
+// sums U1 and U2 are kept in fp32.  bf16 slices keep the LayerNorm outputs
+// (X1 and the next layer's X) only as the bf16 copies the contractions read:
+// the residual branch that adds them in fp32 recomputes them from U and the
+// row statistics in the GEMM epilogue.  fp32 slices keep X and X1 in fp32.
 struct LayerBufs {
   void* p[SKY_NUM_PARAMS];
   float* g[SKY_NUM_PARAMS];
   void *Xb, *QKV, *ctx, *X1b, *Gp, *G;  // Gp = GELU'(Z) (fp16 in bf16 slices)
-  float *X32, *U1, *X1_32, *U2;
+  float *U1, *U2;
   float *lse, *mean1, *rstd1, *mean2, *rstd2;
 };
 
@@ -114,6 +115,11 @@ struct sky_slice {
   void* ws;
   size_t ws_bytes;
   int32_t* d_status;
+  // bf16 slices: the first layer's fp32 residual input (the caller's x when it
+  // is fp32 and 16-byte aligned, else the fp32 copy x32 made at the start of
+  // the forward)
+  float* x32 = nullptr;
+  const float* res0 = nullptr;
   // Weight-gradient GEMMs of a bf16 backward run on a second stream, so they
   // fill the SMs that the data-gradient chain leaves idle.  ev_in[j]: input j
   // of the side stream (dU2, dZ, dU1, dQKV) is ready on the caller's stream;
@@ -237,7 +243,8 @@ struct Timed {
 sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, int M, int N,
                     int K, const void* A, const void* Bm, void* C, bool out_f32, int epi,
                     const void* bias, const void* aux, void* aux_out, float* colsum = nullptr,
-                    void* ws = nullptr, size_t ws_bytes = 0, const float* resid = nullptr) {
+                    void* ws = nullptr, size_t ws_bytes = 0, const float* resid = nullptr,
+                    const gemm::LnResid* ln = nullptr) {
   Timed t(s, st, cat, 2.0 * M * N * K, 0);
   if (!ws) {
     ws = s->ws;
@@ -245,7 +252,7 @@ sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, 
   }
   if (s->cfg.dtype == SKY_DTYPE_BF16)
     return gemm::launch_bf16(form, M, N, K, A, Bm, C, out_f32, epi, bias, aux, aux_out, ws,
-                             ws_bytes, s->d_status, st, colsum, nullptr, 0, nullptr, resid);
+                             ws_bytes, s->d_status, st, colsum, nullptr, 0, nullptr, resid, ln);
   return gemm::launch_f32(form, M, N, K, static_cast<const float*>(A),
                           static_cast<const float*>(Bm), static_cast<float*>(C), epi,
                           static_cast<const float*>(bias), static_cast<const float*>(aux),
@@ -259,7 +266,7 @@ sky_status run_gemm(sky_slice* s, cudaStream_t st, int cat, sky_gemm_form form, 
   } while (0)
 
 // ------------------------------------------------------------------ forward
-// One layer, steps a1..a8.  y_out == nullptr: write the next layer's Xb/X32.
+// One layer, steps a1..a8.  y_out == nullptr: write the next layer's Xb.
 sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
   LayerBufs& Lb = s->layers[i];
   const int B = s->B, S = s->S, H = s->H, A = s->A, F = s->F;
@@ -275,38 +282,54 @@ sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
     SKY_TRY(attention_fwd(Lb.QKV, s->d_len, B, S, H, A, dt, Lb.ctx, Lb.lse, s->d_status, st));
   }
   // a3 + a4: U1 = ctx Wo^T + bo + X (fp32).  bf16: the residual X is added
-  // by the GEMM epilogue; fp32: by the LayerNorm.  X1 = LN(U1)
+  // by the GEMM epilogue (for layers after the first, as LN2 of the previous
+  // layer's U2, recomputed there); fp32: by the LayerNorm.  X1 = LN(U1)
   const bool bf = dt == SKY_DTYPE_BF16;
-  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, H, Lb.ctx, Lb.p[2], Lb.U1, true,
-                   SKY_EPI_STORE, Lb.p[3], nullptr, nullptr, nullptr, nullptr, 0,
-                   bf ? Lb.X32 : nullptr));
   {
-    Timed t(s, st, P_LN_FWD, 0, (bf ? 4.0 : 12.0) * T * H + (4.0 + e) * T * H + 8.0 * T);
-    SKY_TRY(layernorm_fwd(Lb.U1, bf ? nullptr : Lb.X32, Lb.p[4], Lb.p[5], T, H, s->cfg.ln_eps,
-                          dt, bf ? nullptr : Lb.U1, bf ? Lb.X1_32 : nullptr, Lb.X1b, Lb.mean1,
-                          Lb.rstd1, st));
+    const gemm::LnResid* ln = nullptr;
+    gemm::LnResid prev{};
+    const float* r = s->res0;
+    if (bf && i > 0) {
+      const LayerBufs& Pv = s->layers[i - 1];
+      prev = gemm::LnResid{Pv.mean2, Pv.rstd2, Pv.p[10], Pv.p[11]};
+      ln = &prev;
+      r = Pv.U2;
+    }
+    SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, H, Lb.ctx, Lb.p[2], Lb.U1, true,
+                     SKY_EPI_STORE, Lb.p[3], nullptr, nullptr, nullptr, nullptr, 0,
+                     bf ? r : nullptr, ln));
+  }
+  {
+    Timed t(s, st, P_LN_FWD, 0, (bf ? 4.0 + e : 16.0) * T * H + 8.0 * T);
+    SKY_TRY(layernorm_fwd(Lb.U1, bf ? nullptr : static_cast<const float*>(Lb.Xb), Lb.p[4],
+                          Lb.p[5], T, H, s->cfg.ln_eps, dt, bf ? nullptr : Lb.U1, nullptr,
+                          Lb.X1b, Lb.mean1, Lb.rstd1, st));
   }
   // a5 + a6: Z = X1 W1^T + b1; G = GELU(Z) and GELU'(Z) for the backward (fused epilogue)
   SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, F, H, Lb.X1b, Lb.p[6], Lb.G, false,
                    SKY_EPI_BIAS_GELU, Lb.p[7], nullptr, Lb.Gp));
-  // a7 + a8: U2 = G W2^T + b2 + X1 (fp32; the residual as in a3).  Y = LN(U2)
-  // -> next layer's input (fp32 + dtype copy) or the caller's y
-  SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, F, Lb.G, Lb.p[8], Lb.U2, true,
-                   SKY_EPI_STORE, Lb.p[9], nullptr, nullptr, nullptr, nullptr, 0,
-                   bf ? Lb.X1_32 : nullptr));
+  // a7 + a8: U2 = G W2^T + b2 + X1 (fp32; the residual as in a3, X1 = LN1(U1)
+  // recomputed in the bf16 epilogue).  Y = LN(U2) -> next layer's input (its
+  // dtype copy) or the caller's y
   {
-    Timed t(s, st, P_LN_FWD, 0, (bf ? 4.0 : 12.0) * T * H + (4.0 + e) * T * H + 8.0 * T);
-    const float* r2 = bf ? nullptr : Lb.X1_32;
+    const gemm::LnResid ln1{Lb.mean1, Lb.rstd1, Lb.p[4], Lb.p[5]};
+    SKY_TRY(run_gemm(s, st, P_GEMM_FWD, SKY_GEMM_XWT, T, H, F, Lb.G, Lb.p[8], Lb.U2, true,
+                     SKY_EPI_STORE, Lb.p[9], nullptr, nullptr, nullptr, nullptr, 0,
+                     bf ? Lb.U1 : nullptr, bf ? &ln1 : nullptr));
+  }
+  {
+    const bool f32 = bf && y_out && s->cfg.io_fp32;
+    Timed t(s, st, P_LN_FWD, 0, (bf ? 4.0 + (f32 ? 4.0 : e) : 16.0) * T * H + 8.0 * T);
+    const float* r2 = bf ? nullptr : static_cast<const float*>(Lb.X1b);
     float* u2 = bf ? nullptr : Lb.U2;
     if (y_out) {
-      const bool f32 = bf && s->cfg.io_fp32;
       SKY_TRY(layernorm_fwd(Lb.U2, r2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, u2,
                             f32 ? static_cast<float*>(y_out) : nullptr, f32 ? nullptr : y_out,
                             Lb.mean2, Lb.rstd2, st));
     } else {
       LayerBufs& Nx = s->layers[i + 1];
       SKY_TRY(layernorm_fwd(Lb.U2, r2, Lb.p[10], Lb.p[11], T, H, s->cfg.ln_eps, dt, u2,
-                            bf ? Nx.X32 : nullptr, Nx.Xb, Lb.mean2, Lb.rstd2, st));
+                            nullptr, Nx.Xb, Lb.mean2, Lb.rstd2, st));
     }
   }
   return SKY_OK;
@@ -457,14 +480,24 @@ sky_status forward_all(sky_slice* s, const void* x, void* y, cudaStream_t st,
                        std::vector<cudaEvent_t>* marks) {
   const int64_t n = (int64_t)s->B * s->S * s->H;
   {
-    Timed t(s, st, P_COPY, 0, (2.0 * s->esz + (s->esz == 2 ? 6.0 : 0.0)) * n);
     LayerBufs& L0 = s->layers[0];
+    s->res0 = nullptr;
     if (s->cfg.dtype == SKY_DTYPE_BF16 && s->cfg.io_fp32) {
-      SKY_CUDA(cudaMemcpyAsync(L0.X32, x, n * 4, cudaMemcpyDeviceToDevice, st));
-      SKY_TRY(f32_to_bf16(L0.X32, n, L0.Xb, st));
+      // the first layer's residual branch reads x in place; its bf16 copy
+      // feeds the QKV projection
+      const bool in_place = (reinterpret_cast<uintptr_t>(x) & 15) == 0;
+      Timed t(s, st, P_COPY, 0, (in_place ? 6.0 : 14.0) * n);
+      if (!in_place)
+        SKY_CUDA(cudaMemcpyAsync(s->x32, x, n * 4, cudaMemcpyDeviceToDevice, st));
+      s->res0 = in_place ? static_cast<const float*>(x) : s->x32;
+      SKY_TRY(f32_to_bf16(s->res0, n, L0.Xb, st));
     } else {
+      Timed t(s, st, P_COPY, 0, (2.0 * s->esz + (s->esz == 2 ? 6.0 : 0.0)) * n);
       SKY_CUDA(cudaMemcpyAsync(L0.Xb, x, n * s->esz, cudaMemcpyDeviceToDevice, st));
-      if (s->cfg.dtype == SKY_DTYPE_BF16) SKY_TRY(to_f32(x, n, s->cfg.dtype, L0.X32, st));
+      if (s->cfg.dtype == SKY_DTYPE_BF16) {
+        SKY_TRY(to_f32(x, n, s->cfg.dtype, s->x32, st));
+        s->res0 = s->x32;
+      }
     }
   }
   for (int i = 0; i < s->L; ++i) {
@@ -597,9 +630,9 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   const size_t t32 = align_up((size_t)T * s->H * 4);
   const bool bf = c.dtype == SKY_DTYPE_BF16;
   const size_t lse = align_up((size_t)c.max_batch * s->A * c.max_seq * 4);
-  // Xb ctx X1b | QKV | Gp G | U1 U2 (+ X32 X1_32 for bf16) | lse | 4 stats
+  // Xb ctx X1b | QKV | Gp G | U1 U2 | lse | 4 stats
   const size_t stash = 3 * th + align_up((size_t)T * 3 * s->H * s->esz) +
-                       2 * align_up((size_t)T * s->F * s->esz) + (bf ? 4 : 2) * t32 + lse +
+                       2 * align_up((size_t)T * s->F * s->esz) + 2 * t32 + lse +
                        4 * align_up((size_t)T * 4);
   s->param_bytes = pb * s->L;
   s->grad_bytes = gb * s->L;
@@ -610,8 +643,8 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   s->db1p_bytes = bf ? align_up((size_t)gemm::colpart_rows_max((int)T) * s->F * 4) : 0;
   s->qkvp_bytes = bf ? align_up((size_t)c.max_batch * ceil_div(c.max_seq, 128) * 3 * s->H * 4) : 0;
   // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | ws2 | lnp[2] |
-  // db1p | qkvp | status
-  const size_t wk = 6 * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
+  // db1p | qkvp | status | x32 (bf16)
+  const size_t wk = (bf ? 7 : 6) * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
                     align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes +
                     s->ws2_bytes + 2 * s->lnp_bytes + s->db1p_bytes + s->qkvp_bytes + 256;
   s->ws_bytes_total = wk;
@@ -698,8 +731,6 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
     Lb.G = take((size_t)T * s->F * s->esz);
     Lb.U1 = static_cast<float*>(take(t32));
     Lb.U2 = static_cast<float*>(take(t32));
-    Lb.X32 = bf ? static_cast<float*>(take(t32)) : static_cast<float*>(Lb.Xb);
-    Lb.X1_32 = bf ? static_cast<float*>(take(t32)) : static_cast<float*>(Lb.X1b);
     Lb.lse = static_cast<float*>(take(lse_b));
     Lb.mean1 = static_cast<float*>(take((size_t)T * 4));
     Lb.rstd1 = static_cast<float*>(take((size_t)T * 4));
@@ -727,6 +758,7 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   if (s->db1p_bytes) s->db1p = static_cast<float*>(take(s->db1p_bytes));
   if (s->qkvp_bytes) s->qkvp = static_cast<float*>(take(s->qkvp_bytes));
   s->d_status = static_cast<int32_t*>(take(4));
+  if (bf) s->x32 = static_cast<float*>(take(t32));
   if (bf) {
     // the weight-gradient side stream and its events
     bool ok = cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) == cudaSuccess;

@@ -159,6 +159,31 @@ def test_deterministic_and_status():
         assert e.value.status == L.SKY_ERR_INVALID_ARG
 
 
+def test_fp32_input_read_in_place_or_copied():
+    """A bf16 slice with fp32 boundary tensors reads an aligned x in place as
+    the first layer's residual and copies a misaligned one first.  Both give
+    the same bits (forward, input gradient, every weight gradient), and x is
+    left unchanged."""
+    w = synth.custom("x-align", layers=2, hidden=256, heads=4, ffn=512, seq=64, batch=4,
+                     len_lo=1, len_hi=64, dy_std=1e-2)
+    params = synth.slice_params(w, affine="random")
+    X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    xa = to_device(X, "fp32")
+    n = xa.numel()
+    buf = torch.empty(n + 1, dtype=torch.float32, device="cuda")
+    xm = buf[1:].view(xa.shape)  # 4 bytes past a 16-byte boundary
+    xm.copy_(xa)
+    assert xm.data_ptr() % 16 == 4
+    ya, dxa, ga = _slice_run(w, 0, 2, xa, lens, dY, params, io_fp32=True)
+    ym, dxm, gm = _slice_run(w, 0, 2, xm, lens, dY, params, io_fp32=True)
+    assert torch.equal(ya, ym) and torch.equal(dxa, dxm)
+    for a, b in zip(ga, gm):
+        for k in a:
+            assert np.array_equal(a[k], b[k]), k
+    assert torch.equal(xa.cpu(), torch.from_numpy(np.asarray(X, np.float32)))
+    assert torch.equal(xm, xa)
+
+
 def test_side_stream_backward_matches_in_line():
     """The bf16 backward runs its weight-gradient GEMMs on a second stream that
     overlaps the data-gradient chain and reuses shared gradient buffers across
