@@ -96,7 +96,8 @@ sky_status sky_attention_bwd(const void* qkv, const void* ctx, const void* dctx,
  * y = gamma * (u - mean) * rstd + beta, rstd = 1/sqrt(var + eps), biased
  * variance.  Writes u to u_out (may alias a, or NULL), y to y32 (fp32) and/or
  * y (dtype) -- either may be NULL but not both; gamma, beta: [H] (dtype);
- * mean, rstd: fp32 [T].  H % 8 == 0, H <= 2048 (bf16) or 1024 (fp32). */
+ * mean, rstd: fp32 [T].  H % 8 == 0, H <= 2048 (bf16) or 1024 (fp32).  The
+ * [T, H] tensors and gamma, beta must be 16-byte aligned (else UNSUPPORTED). */
 sky_status sky_layernorm_fwd(const float* a, const float* r, const void* gamma,
                              const void* beta, int32_t T, int32_t H, float eps, sky_dtype dtype,
                              float* u_out, float* y32, void* y, float* mean, float* rstd,
@@ -112,7 +113,8 @@ size_t sky_layernorm_bwd_workspace_bytes(int32_t T, int32_t H);
  * writes du = rstd * (g - mean(g) - xhat * mean(g * xhat)) to du32 (fp32)
  * and/or du (dtype), and the fp32 column sums dgamma = sum dy*xhat,
  * dbeta = sum dy, dbias = sum du (each [H]; any may be NULL), which are
- * deterministic (fixed-order partials in `workspace`). */
+ * deterministic (fixed-order partials in `workspace`).  The [T, H] tensors
+ * and gamma must be 16-byte aligned (else UNSUPPORTED). */
 sky_status sky_layernorm_bwd(const void* dy, sky_dtype dy_dtype, const float* dy2,
                              const float* u, const void* gamma, const float* mean,
                              const float* rstd, int32_t T, int32_t H, sky_dtype dtype,

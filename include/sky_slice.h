@@ -139,7 +139,8 @@ sky_status sky_slice_get_grads(sky_slice* s, int32_t layer, void* const* tensors
  * work on `stream` is done (a bf16 slice with fp32 boundary tensors reads a
  * 16-byte aligned x in place as the first layer's residual until then).
  * Enqueues work on `stream`; no host synchronisation.
- * Errors: INVALID_ARG (B > max_batch, S > max_seq, B or S < 1, null). */
+ * Errors: INVALID_ARG (B > max_batch, S > max_seq, B or S < 1, null),
+ * UNSUPPORTED (y not 16-byte aligned). */
 sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,
                              int32_t S, void* y, void* stream);
 
@@ -147,7 +148,8 @@ sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, 
  * (device [B,S,H], boundary dtype) writes dx = dL/dx and overwrites the fp32
  * gradients of every layer.  Must follow a forward on the same handle (the
  * forward's d_len must still be valid).  Enqueues on `stream`.
- * Errors: STATE (no forward since create), INVALID_ARG (null). */
+ * Errors: STATE (no forward since create), INVALID_ARG (null), UNSUPPORTED
+ * (dy not 16-byte aligned). */
 sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stream);
 
 /* Measures every layer of the slice: runs `iters` forward+backward passes at

@@ -557,9 +557,18 @@ int lane_vectors(int H) { return ceil_div(H, 32 * rw::V); }
     default: CALL(8); break;       \
   }
 
+namespace {
+// the row kernels move 16-byte vectors (and bulk-copy rows), so every [rows, H]
+// tensor and gamma, beta must start on a 16-byte boundary (null is accepted)
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+}  // namespace
+
 sky_status layernorm_fwd(const float* a, const float* r, const void* gamma, const void* beta,
                          int rows, int H, float eps, sky_dtype dt, float* u_out, float* y32,
                          void* y, float* mean, float* rstd, cudaStream_t st) {
+  SKY_CHECK(aligned16(a) && aligned16(r) && aligned16(gamma) && aligned16(beta) &&
+                aligned16(u_out) && aligned16(y32) && aligned16(y),
+            SKY_ERR_UNSUPPORTED, "LayerNorm tensors must be 16-byte aligned");
   SKY_CHECK(H % rw::V == 0 && lane_vectors(H) <= kMaxNV && (dt == SKY_DTYPE_BF16 || H <= 1024),
             SKY_ERR_UNSUPPORTED, "LayerNorm width %d unsupported", H);
   SKY_CHECK(y32 || y, SKY_ERR_INVALID_ARG, "LayerNorm forward needs an output");
@@ -590,7 +599,10 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
                          const void* gamma, const float* mean, const float* rstd, int rows, int H,
                          sky_dtype dt, float* du32, void* du, float* dgamma, float* dbeta,
                          float* dbias, void* ws, size_t ws_bytes, cudaStream_t st,
-                         int* deferred_parts) {
+                         int* deferred_parts, int32_t* status) {
+  SKY_CHECK(aligned16(dy) && aligned16(dy2) && aligned16(u) && aligned16(gamma) &&
+                aligned16(du32) && aligned16(du),
+            SKY_ERR_UNSUPPORTED, "LayerNorm tensors must be 16-byte aligned");
   SKY_CHECK(H % rw::V == 0 && lane_vectors(H) <= kMaxNV && (dt == SKY_DTYPE_BF16 || H <= 1024),
             SKY_ERR_UNSUPPORTED, "LayerNorm width %d unsupported", H);
   SKY_CHECK(du32 || du, SKY_ERR_INVALID_ARG, "LayerNorm backward needs an output");
@@ -614,14 +626,14 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
       if (a != cudaSuccess) return cuda_fail(a, "LayerNorm backward smem attribute");
       launch_pdl(rw::ln_bwd_stream_kernel<__nv_bfloat16>, dim3(sb), dim3(threads), smem, st, 1, 
           static_cast<const __nv_bfloat16*>(dy), dy2, u, static_cast<const __nv_bfloat16*>(gamma),
-          mean, rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, nullptr);
+          mean, rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, status);
     } else {
       static cudaError_t a = cudaFuncSetAttribute(rw::ln_bwd_stream_kernel<float>,
                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
       if (a != cudaSuccess) return cuda_fail(a, "LayerNorm backward smem attribute");
       launch_pdl(rw::ln_bwd_stream_kernel<float>, dim3(sb), dim3(threads), smem, st, 1, 
           static_cast<const float*>(dy), dy2, u, static_cast<const __nv_bfloat16*>(gamma), mean,
-          rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, nullptr);
+          rstd, rows, H, du32, static_cast<__nv_bfloat16*>(du), part, status);
     }
     count_launches(1);
     const cudaError_t e = cudaGetLastError();

@@ -15,6 +15,9 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
                          const int32_t* lens, int B, int S, int H, int A, sky_dtype dt, void* dqkv,
                          float* delta, int32_t* status, cudaStream_t st, float* colpart = nullptr);
 
+// LayerNorm launchers: [rows, H] tensors and gamma, beta 16-byte aligned;
+// `status` (optional) receives the timeout bit of the streamed backward's
+// bounded waits.
 sky_status layernorm_fwd(const float* a, const float* r, const void* gamma, const void* beta,
                          int rows, int H, float eps, sky_dtype dt, float* u_out, float* y32,
                          void* y, float* mean, float* rstd, cudaStream_t st);
@@ -23,7 +26,7 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
                          const void* gamma, const float* mean, const float* rstd, int rows, int H,
                          sky_dtype dt, float* du32, void* du, float* dgamma, float* dbeta,
                          float* dbias, void* ws, size_t ws_bytes, cudaStream_t st,
-                         int* deferred_parts = nullptr);
+                         int* deferred_parts = nullptr, int32_t* status = nullptr);
 // With `deferred_parts`, layernorm_bwd leaves dgamma / dbeta / dbias as
 // per-CTA partials in `ws` (*deferred_parts rows each) and this call, possibly
 // on another stream ordered after it, adds them in a fixed order.

@@ -385,7 +385,7 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     SKY_TRY(layernorm_bwd(dY, dy_dt, dY2, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
                           bf ? s->dU2_32 : nullptr, s->dU2b, Lb.g[10], Lb.g[11], Lb.g[9],
                           bf ? s->lnp[0] : s->ws, bf ? s->lnp_bytes : s->ws_bytes, st,
-                          bf ? &ln_parts : nullptr));
+                          bf ? &ln_parts : nullptr, s->d_status));
   }
   SKY_TRY(fork(0));
   if (bf) SKY_TRY(ln_reduce(0, Lb.g[10], Lb.g[11], Lb.g[9]));
@@ -427,7 +427,8 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? nullptr : static_cast<float*>(s->dU2b),
                           Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H, dt, bf ? s->dR[k] : nullptr,
                           dU1b, Lb.g[4], Lb.g[5], Lb.g[3], bf ? s->lnp[1] : s->ws,
-                          bf ? s->lnp_bytes : s->ws_bytes, st, bf ? &ln_parts : nullptr));
+                          bf ? s->lnp_bytes : s->ws_bytes, st, bf ? &ln_parts : nullptr,
+                          s->d_status));
   }
   SKY_TRY(fork(2));
   if (bf) SKY_TRY(ln_reduce(1, Lb.g[4], Lb.g[5], Lb.g[3]));
@@ -869,6 +870,8 @@ sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, 
   SKY_CHECK(B <= s->cfg.max_batch && S <= s->cfg.max_seq, SKY_ERR_INVALID_ARG,
             "B=%d S=%d exceed max_batch=%d max_seq=%d", B, S, s->cfg.max_batch, s->cfg.max_seq);
   SKY_CHECK(x != y, SKY_ERR_INVALID_ARG, "x and y must not alias");
+  SKY_CHECK((reinterpret_cast<uintptr_t>(y) & 15) == 0, SKY_ERR_UNSUPPORTED,
+            "y must be 16-byte aligned");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   s->B = B; s->S = S; s->d_len = d_len; s->last_stream = st;
   s->have_fwd = false;
@@ -882,6 +885,8 @@ sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stre
   ABI_GUARD_BEGIN
   SKY_CHECK(s && dy && dx, SKY_ERR_INVALID_ARG, "null argument");
   SKY_CHECK(s->have_fwd, SKY_ERR_STATE, "backward needs a forward on this slice first");
+  SKY_CHECK((reinterpret_cast<uintptr_t>(dy) & 15) == 0, SKY_ERR_UNSUPPORTED,
+            "dy must be 16-byte aligned");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   s->last_stream = st;
   return backward_all(s, dy, dx, st, nullptr);

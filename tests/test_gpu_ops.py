@@ -258,6 +258,61 @@ def test_layernorm(dt, TH):
     assert_close("add", to_host(s_out), rv.astype(np.float64) + dy2, dt)
 
 
+@pytest.mark.parametrize("TH", [(1000, 1024), (300, 768), (200, 2048), (100, 512)],
+                         ids=lambda t: f"T{t[0]}H{t[1]}")
+def test_layernorm_fwd_of_u_only(TH):
+    """bf16 LayerNorm of u alone (no residual operand, no u output), the form
+    the slice uses: against the oracle, and bit for bit against the same rows
+    with a zero residual added (which changes no sum).  Also with an fp32
+    output only, whose bf16 rounding is the bf16 output."""
+    T, H = TH
+    g = np.random.default_rng(T * H)
+    av = g.normal(0.5, 1.0, (T, H)).astype(np.float32)
+    gam, bet = round_bf16(1 + g.normal(0, 0.1, H)), round_bf16(g.normal(0, 0.1, H))
+    A_ = torch.from_numpy(av).cuda()
+    Z_ = torch.zeros_like(A_)
+    G_, B_ = to_device(gam, "bf16"), to_device(bet, "bf16")
+    eps = 1e-12
+    outs = []
+    for r in (None, Z_):
+        y = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
+        mean = torch.empty(T, dtype=torch.float32, device="cuda")
+        rstd = torch.empty(T, dtype=torch.float32, device="cuda")
+        L.call("sky_layernorm_fwd", P(A_), P(r) if r is not None else None, P(G_), P(B_), T, H,
+               C.c_float(eps), dt_code("bf16"), None, None, P(y), P(mean), P(rstd), stream())
+        outs.append((y, mean, rstd))
+    y32 = torch.empty((T, H), dtype=torch.float32, device="cuda")
+    m2, r2 = (torch.empty(T, dtype=torch.float32, device="cuda") for _ in range(2))
+    L.call("sky_layernorm_fwd", P(A_), None, P(G_), P(B_), T, H, C.c_float(eps), dt_code("bf16"),
+           None, P(y32), None, P(m2), P(r2), stream())
+    torch.cuda.synchronize()
+    (ys, ms, rs), (yw, mw, rw) = outs
+    assert torch.equal(ys, yw) and torch.equal(ms, mw) and torch.equal(rs, rw)
+    assert torch.equal(m2, ms) and torch.equal(r2, rs)
+    assert torch.equal(y32.bfloat16(), ys)
+    Yo, _, rso = ORC.layer_norm(av.astype(np.float64), gam.astype(np.float64),
+                                bet.astype(np.float64), eps)
+    assert l2rel(to_host(y32), Yo) <= 1e-5
+    assert_close("y", to_host(ys), Yo, "bf16")
+    assert l2rel(rs.cpu().numpy().astype(np.float64), rso.reshape(-1)) <= 1e-5
+
+
+def test_layernorm_rejects_misaligned_tensors():
+    """The row kernels move 16-byte vectors: a tensor off a 16-byte boundary
+    is refused on the host (UNSUPPORTED), before any launch."""
+    T, H = 200, 256
+    buf = torch.zeros(T * H + 1, dtype=torch.float32, device="cuda")
+    a = buf[1:]
+    G_ = torch.ones(H, dtype=torch.bfloat16, device="cuda")
+    B_ = torch.zeros(H, dtype=torch.bfloat16, device="cuda")
+    y = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
+    mean, rstd = (torch.empty(T, dtype=torch.float32, device="cuda") for _ in range(2))
+    with pytest.raises(L.SkyError) as e:
+        L.call("sky_layernorm_fwd", P(a), None, P(G_), P(B_), T, H, C.c_float(1e-12),
+               dt_code("bf16"), None, None, P(y), P(mean), P(rstd), stream())
+    assert e.value.status == L.SKY_ERR_UNSUPPORTED
+
+
 @pytest.mark.parametrize("dt", ["bf16", "fp32"])
 def test_gelu_and_column_sum(dt):
     T, N = 333, 1000
