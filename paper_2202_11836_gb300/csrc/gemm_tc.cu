@@ -52,11 +52,12 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;           // two fp32 accumulators of 128 x 256
 constexpr int NUM_EPI_WARPS = 8;            // two per TMEM lane quarter (default)
 constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
-// CTA-pair variant: per CTA and stage A 128 x 64 + B 128 x 64 (32 KiB), six
-// stages in the same 192 KiB
-constexpr int PAIR_STAGES = 6;
+// CTA-pair variant: per CTA and stage A 128 x 64 + B 128 x 64 (32 KiB), five
+// stages (160 KiB).  Six stages (192 KiB) made most kernels timed alone
+// 1-2 us faster, but the GELU' data-gradient kernel 5 us slower and the
+// whole training step 30-40 us slower; four stages were slower everywhere.
+constexpr int PAIR_STAGES = 5;
 constexpr int PAIR_STAGE_BYTES = A_BYTES + (BN / 2) * BK * 2;
-static_assert(PAIR_STAGES * PAIR_STAGE_BYTES == STAGES * STAGE_BYTES, "same ring size");
 
 // Launch shape per instantiation: epilogue warps (a multiple of 4, one group
 // per TMEM lane quarter), epilogue chunk width, ring stages and shared memory.
