@@ -389,8 +389,11 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
               const __half2 h0 = __floats2half2_rn(gp[0], gp[1]), h1 = __floats2half2_rn(gp[2], gp[3]);
               *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.C) + off) =
                   make_uint2(ptx::pack_bf16(z[0], z[1]), ptx::pack_bf16(z[2], z[3]));
-              *reinterpret_cast<uint2*>(p.aux_out + off) =
-                  make_uint2(*reinterpret_cast<const uint32_t*>(&h0), *reinterpret_cast<const uint32_t*>(&h1));
+              // GELU'(z) is read again only by the backward pass: a streaming
+              // store keeps it from displacing G, which FFN2 reads next, in L2
+              __stcs(reinterpret_cast<uint2*>(p.aux_out + off),
+                     make_uint2(*reinterpret_cast<const uint32_t*>(&h0),
+                                *reinterpret_cast<const uint32_t*>(&h1)));
             }
           }
         }
@@ -510,7 +513,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
               *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.C) + off) =
                   make_uint2(ptx::pack_bf16(v[i][0], v[i][1]), ptx::pack_bf16(v[i][2], v[i][3]));
               if constexpr (EPI == SKY_EPI_BIAS_GELU)
-                *reinterpret_cast<uint2*>(p.aux_out + off) = gq[i];
+                __stcs(reinterpret_cast<uint2*>(p.aux_out + off), gq[i]);
             }
           }
         }
