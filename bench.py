@@ -5,7 +5,9 @@ every layer of the slice, then the backward pass in reverse order with all
 weight and input gradients (the per-device unit of work of the paper's
 layer-partitioned training, Sec. III / IV-D).  Default workload: BERT-large
 width, 8 layers, S=512, B=16 (bf16, seeded synthetic inputs standing in for
-the paper's MNLI batches).
+the paper's MNLI batches).  The timed step is the slice's forward + backward
+captured once as a CUDA graph (sky_slice_step_graph_create) and replayed;
+direct forward / backward calls are timed beside it.
 
 Prints one JSON line (rank 0).  `--impl reference` times the float64 CPU
 oracle instead (the reference arm).  With torchrun (N > 1) every rank runs an
@@ -290,6 +292,13 @@ def run_gpu(args, w):
         s.forward(x, ln, y, stream)
         s.backward(dy, dx, stream)
 
+    # the same step captured once as a CUDA graph held by the slice
+    # (sky_slice_step_graph_create); replays launch the same kernels
+    s.step_graph(x, ln, y, dy, dx, stream)
+
+    def step_graph():
+        s.launch_step_graph(stream)
+
     def barrier():
         if world > 1:
             dist.barrier()
@@ -319,9 +328,13 @@ def run_gpu(args, w):
     props = torch.cuda.get_device_properties(local)
     gpu_id = ("GPU-" + str(props.uuid)) if getattr(props, "uuid", None) else str(local)
     with ClockSampler(gpu_id) as clk:
-        ms = timed_region(step, args.steps, args.warmup, sync, barrier, reduce_max, start, stop)
+        ms = timed_region(step_graph, args.steps, args.warmup, sync, barrier, reduce_max, start,
+                          stop)
     launches = (_lib.lib().sky_launch_count() - launches0)
     launches_timed = launches * args.steps // (args.steps + args.warmup)
+    s.sync()
+    # the same steps as direct sky_slice_forward / sky_slice_backward calls
+    ms_direct = timed_region(step, args.steps, args.warmup, sync, barrier, reduce_max, start, stop)
     s.sync()
     ms_step = ms / args.steps
     tokens = w.tokens
@@ -382,8 +395,7 @@ def run_gpu(args, w):
         x.copy_(xh, non_blocking=True)
         dy.copy_(dyh, non_blocking=True)
         ln.copy_(lh, non_blocking=True)
-        s.forward(x, ln, y, stream)
-        s.backward(dy, dx, stream)
+        s.launch_step_graph(stream)
         yh.copy_(y, non_blocking=True)
         dxh.copy_(dx, non_blocking=True)
 
@@ -410,6 +422,10 @@ def run_gpu(args, w):
             "allocation": allocation_plan(rec),
             "optimizer": optimizer,
             "valid_tokens_per_s": world * int(np.sum(lens)) * args.steps / (ms / 1e3),
+            "step": "one CUDA graph of the slice's forward + backward (sky_slice_step_graph_launch)",
+            "direct_calls": {"value": world * tokens * args.steps / (ms_direct / 1e3),
+                             "ms_per_step": ms_direct / args.steps,
+                             "how": "sky_slice_forward + sky_slice_backward each step"},
             "roofline": {"kernel": "gemm_tc_kernel (all GEMM launches of the step)",
                          "bound": "tensor", "achieved": round(achieved, 1),
                          "peak": pk["bf16_sus"], "unit": "TFLOP/s",

@@ -152,6 +152,29 @@ sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, 
  * (dy not 16-byte aligned). */
 sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stream);
 
+/* A device's training step over its slice (Sec. III: forward through its
+ * layers, then backward in reverse order) as one CUDA graph.
+ * sky_slice_step_graph_create runs sky_slice_forward(x, d_len, B, S, y) and
+ * sky_slice_backward(dy, dx) once on `stream` (checking every argument as
+ * those calls do, and synchronising `stream`), then captures the same two
+ * calls on a private stream into an executable graph that the slice owns,
+ * replacing any earlier one.  sky_slice_step_graph_launch enqueues that graph
+ * on `stream`: the same kernels, in the same order, on the same buffers, so
+ * its results equal the two calls' bit for bit.  The graph keeps the pointers
+ * and B, S it was created with: the caller refills x, d_len and dy in place
+ * between launches and keeps all five buffers alive while the graph exists.
+ * Replays on one slice must not overlap each other or direct calls on that
+ * slice (they share its stash and workspace).  Launches are counted in
+ * sky_launch_count at every replay; per-kernel timing does not see them.
+ * The graph is freed by the next create and by sky_slice_destroy.
+ * Errors: those of sky_slice_forward / sky_slice_backward; STATE if
+ * per-kernel timing is on (create) or no graph exists (launch); CUDA if the
+ * capture or instantiation fails. */
+sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_t* d_len,
+                                       int32_t B, int32_t S, void* y, const void* dy, void* dx,
+                                       void* stream);
+sky_status sky_slice_step_graph_launch(sky_slice* s, void* stream);
+
 /* Measures every layer of the slice: runs `iters` forward+backward passes at
  * [B,S] with full-length sequences and synthetic data already on the device
  * (parameters as set), records CUDA events around each layer, and writes the

@@ -124,9 +124,14 @@ struct sky_slice {
   // fill the SMs that the data-gradient chain leaves idle.  ev_in[j]: input j
   // of the side stream (dU2, dZ, dU1, dQKV) is ready on the caller's stream;
   // ev_out[j]: the side GEMM reading input j is done, so the next layer may
-  // overwrite that buffer.  ws2: the side GEMMs' split-K scratch.
+  // overwrite that buffer; ev_out_live[j]: ev_out[j] was recorded by the
+  // current backward call (earlier records are already ordered by that
+  // call's final join, and waiting on them would tie a captured backward
+  // pass to work outside its CUDA graph).  ws2: the side GEMMs' split-K
+  // scratch.
   cudaStream_t side = nullptr;
   cudaEvent_t ev_in[4] = {}, ev_out[4] = {}, ev_join = nullptr;
+  bool ev_out_live[4] = {};
   void* ws2 = nullptr;
   size_t ws2_bytes = 0;
   // Column partials whose fixed-order reduction (a bias / LayerNorm-parameter
@@ -156,6 +161,14 @@ struct sky_slice {
   int B = 0, S = 0;
   const int32_t* d_len = nullptr;
   cudaStream_t last_stream = nullptr;
+  // one captured training step (forward + backward) as an executable CUDA
+  // graph, the private stream it was captured on, the kernel launches it
+  // holds and the batch shape and lengths it was captured with
+  cudaGraphExec_t step_exec = nullptr;
+  cudaStream_t cap_stream = nullptr;
+  int64_t step_launches = 0;
+  int step_B = 0, step_S = 0;
+  const int32_t* step_len = nullptr;
   // profiling
   bool prof = false;
   std::vector<sky::ProfRecord> recs;
@@ -362,11 +375,14 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     return SKY_OK;
   };
   auto reuse = [&](int j) -> sky_status {
-    if (two) SKY_CUDA(cudaStreamWaitEvent(st, s->ev_out[j], 0));
+    if (two && s->ev_out_live[j]) SKY_CUDA(cudaStreamWaitEvent(st, s->ev_out[j], 0));
     return SKY_OK;
   };
   auto done = [&](int j) -> sky_status {
-    if (two) SKY_CUDA(cudaEventRecord(s->ev_out[j], sw));
+    if (two) {
+      SKY_CUDA(cudaEventRecord(s->ev_out[j], sw));
+      s->ev_out_live[j] = true;
+    }
     return SKY_OK;
   };
   void* ws2 = bf ? s->ws2 : nullptr;
@@ -525,6 +541,7 @@ sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
     SKY_CUDA(cudaStreamWaitEvent(st, s->ev_join, 0));
     return SKY_OK;
   };
+  for (bool& live : s->ev_out_live) live = false;
   if (sw != st) {  // the side stream starts after everything before this call
     SKY_CUDA(cudaEventRecord(s->ev_join, st));
     SKY_CUDA(cudaStreamWaitEvent(sw, s->ev_join, 0));
@@ -788,6 +805,8 @@ sky_status sky_slice_destroy(sky_slice* s) {
     if (s->ev_out[j]) cudaEventDestroy(s->ev_out[j]);
   }
   if (s->ev_join) cudaEventDestroy(s->ev_join);
+  if (s->step_exec) cudaGraphExecDestroy(s->step_exec);
+  if (s->cap_stream) cudaStreamDestroy(s->cap_stream);
   if (s->side) cudaStreamDestroy(s->side);
   if (s->opt_mem) cudaFree(s->opt_mem);
   if (s->arena) cudaFree(s->arena);
@@ -890,6 +909,66 @@ sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stre
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   s->last_stream = st;
   return backward_all(s, dy, dx, st, nullptr);
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_t* d_len,
+                                       int32_t B, int32_t S, void* y, const void* dy, void* dx,
+                                       void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s, SKY_ERR_INVALID_ARG, "null handle");
+  SKY_CHECK(!s->prof, SKY_ERR_STATE, "per-kernel timing is on; a step graph holds no timers");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // One step in the ordinary way first: it checks every argument, and any
+  // one-time set-up (kernel attributes, occupancy queries) happens outside
+  // the capture.
+  SKY_TRY(sky_slice_forward(s, x, d_len, B, S, y, stream));
+  SKY_TRY(sky_slice_backward(s, dy, dx, stream));
+  SKY_CUDA(cudaStreamSynchronize(st));
+  if (s->step_exec) {
+    SKY_CUDA(cudaGraphExecDestroy(s->step_exec));
+    s->step_exec = nullptr;
+  }
+  if (!s->cap_stream) SKY_CUDA(cudaStreamCreateWithFlags(&s->cap_stream, cudaStreamNonBlocking));
+  cudaStream_t cs = s->cap_stream;
+  const int64_t n0 = sky_launch_count();
+  SKY_CUDA(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
+  s->B = B; s->S = S; s->d_len = d_len;
+  sky_status rc = forward_all(s, x, y, cs, nullptr);
+  if (rc == SKY_OK) rc = backward_all(s, dy, dx, cs, nullptr);
+  cudaGraph_t graph = nullptr;
+  const cudaError_t ec = cudaStreamEndCapture(cs, &graph);
+  if (rc != SKY_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return rc;
+  }
+  if (ec != cudaSuccess) return cuda_fail(ec, "cudaStreamEndCapture");
+  const cudaError_t ei = cudaGraphInstantiate(&s->step_exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (ei != cudaSuccess) {
+    s->step_exec = nullptr;
+    return cuda_fail(ei, "cudaGraphInstantiate");
+  }
+  // the captured launches ran nothing yet: they are counted at every replay
+  s->step_launches = sky_launch_count() - n0;
+  count_launches(-static_cast<int>(s->step_launches));
+  s->step_B = B; s->step_S = S; s->step_len = d_len;
+  SKY_CUDA(cudaGraphUpload(s->step_exec, st));
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_step_graph_launch(sky_slice* s, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s, SKY_ERR_INVALID_ARG, "null handle");
+  SKY_CHECK(s->step_exec, SKY_ERR_STATE, "no step graph: call sky_slice_step_graph_create");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SKY_CUDA(cudaGraphLaunch(s->step_exec, st));
+  count_launches(static_cast<int>(s->step_launches));
+  s->B = s->step_B; s->S = s->step_S; s->d_len = s->step_len;
+  s->last_stream = st;
+  s->have_fwd = true;
+  return SKY_OK;
   ABI_GUARD_END
 }
 

@@ -119,6 +119,20 @@ class EncoderSlice:
         L.call("sky_slice_backward", self.h, _ptr(dy), _ptr(dx), _stream_ptr(stream))
         return dx
 
+    def step_graph(self, x, lens, y, dy, dx, stream=None) -> None:
+        """Captures forward(x, lens, y) + backward(dy, dx) as one CUDA graph held
+        by the slice (after running the step once); replay it with
+        ``launch_step_graph``.  The five tensors stay bound to the graph."""
+        import torch
+        B, S, H = x.shape
+        assert H == self.H and x.is_contiguous() and lens.dtype == torch.int32
+        L.call("sky_slice_step_graph_create", self.h, _ptr(x), _ptr(lens), B, S, _ptr(y),
+               _ptr(dy), _ptr(dx), _stream_ptr(stream))
+        self._graph_keep = (x, lens, y, dy, dx)
+
+    def launch_step_graph(self, stream=None) -> None:
+        L.call("sky_slice_step_graph_launch", self.h, _stream_ptr(stream))
+
     def sync(self) -> None:
         L.call("sky_slice_sync", self.h)
 

@@ -81,6 +81,9 @@ def test_null_arguments(lib):
     assert lib.sky_slice_destroy(None) == L.SKY_OK
     assert lib.sky_slice_forward(None, None, None, 1, 1, None, None) == L.SKY_ERR_INVALID_ARG
     assert lib.sky_slice_backward(None, None, None, None) == L.SKY_ERR_INVALID_ARG
+    assert lib.sky_slice_step_graph_create(None, None, None, 1, 1, None, None, None,
+                                           None) == L.SKY_ERR_INVALID_ARG
+    assert lib.sky_slice_step_graph_launch(None, None) == L.SKY_ERR_INVALID_ARG
     assert lib.sky_gemm(0, 8, 8, 8, 0, None, None, None, 0, 0, None, None, None, None, 0, None,
                         None) == L.SKY_ERR_INVALID_ARG
     assert lib.sky_column_sum_workspace_bytes(0, 5) == 0

@@ -247,3 +247,58 @@ def test_layer_cost_feeds_allocator():
     assert pi[0] == 0 and pi[-1] == le - lb and min(counts) >= 1
     assert counts[1] <= min(counts[0], counts[2])
     assert P.makespan(pi) <= P.makespan(allocator.even(le - lb, 3))
+
+
+@pytest.mark.parametrize("wname", ["base-s128", "tiny-fp32"])
+def test_step_graph_replays_direct_step_bitwise(wname):
+    """The captured training step (sky_slice_step_graph_create / _launch)
+    reproduces a direct forward + backward bit for bit (output, input
+    gradient, every layer's gradients) on inputs refilled in place after the
+    capture, over two replays, and counts the same kernel launches."""
+    from paper_2202_11836_gb300 import _lib as L
+    from paper_2202_11836_gb300.slice import EncoderSlice
+    w = synth.WORKLOADS[wname]
+    params = synth.slice_params(w, affine="random")
+    X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    X2 = synth.activations(w, seed=synth.SEED + 1)
+    dY2 = synth.upstream_grad(w, seed=synth.SEED + 1)
+    lens2 = synth.lengths(w, seed=synth.SEED + 1)
+    lib = L.lib()
+    with EncoderSlice(w.hidden, w.heads, w.ffn, 0, w.layers, w.batch, w.seq, w.dtype) as s:
+        for i, p in enumerate(params):
+            s.set_params(i, p)
+        # direct step on the second inputs: the reference
+        n0 = lib.sky_launch_count()
+        y_ref = s.forward(to_device(X2, w.dtype), torch.from_numpy(lens2).cuda())
+        dx_ref = s.backward(to_device(dY2, w.dtype))
+        s.sync()
+        per_step = lib.sky_launch_count() - n0
+        g_ref = [s.get_grads(i) for i in range(w.layers)]
+        # capture on the first inputs, then refill them in place
+        x = to_device(X, w.dtype)
+        ln = torch.from_numpy(lens).cuda()
+        dy = to_device(dY, w.dtype)
+        y, dx = torch.empty_like(x), torch.empty_like(x)
+        s.step_graph(x, ln, y, dy, dx)
+        s.sync()
+        x.copy_(to_device(X2, w.dtype))
+        dy.copy_(to_device(dY2, w.dtype))
+        ln.copy_(torch.from_numpy(lens2))
+        for _ in range(2):
+            y.zero_()
+            dx.zero_()
+            n1 = lib.sky_launch_count()
+            s.launch_step_graph()
+            s.sync()
+            assert lib.sky_launch_count() - n1 == per_step
+            assert torch.equal(y, y_ref) and torch.equal(dx, dx_ref)
+            for i in range(w.layers):
+                g = s.get_grads(i)
+                for k in g:
+                    assert np.array_equal(g[k], g_ref[i][k]), (i, k)
+        # per-kernel timing cannot be captured
+        s.set_profiling(True)
+        with pytest.raises(L.SkyError) as e:
+            s.step_graph(x, ln, y, dy, dx)
+        assert e.value.status == L.SKY_ERR_STATE
+        s.set_profiling(False)
