@@ -448,6 +448,95 @@ def run_gpu(args, w):
     return 0
 
 
+def gemm_shapes(w):
+    """The 13 GEMMs of one encoder layer of workload ``w`` as sky_gemm calls:
+    (name, form, M, N, K, epilogue, bias, fp32 output, aux in, aux out)."""
+    T, H, F = w.tokens, w.hidden, w.ffn
+    return [
+        ("fwd QKV", "XWT", T, 3 * H, H, "STORE", True, False, None, None),
+        ("fwd attn-out", "XWT", T, H, H, "STORE", True, True, None, None),
+        ("fwd FFN1", "XWT", T, F, H, "BIAS_GELU", True, False, None, "f16"),
+        ("fwd FFN2", "XWT", T, H, F, "STORE", True, True, None, None),
+        ("dgrad FFN2", "XW", T, F, H, "GELU_BWD", False, False, "f16", None),
+        ("dgrad FFN1", "XW", T, H, F, "STORE", False, True, None, None),
+        ("dgrad attn-out", "XW", T, H, H, "STORE", False, False, None, None),
+        ("dgrad QKV", "XW", T, H, 3 * H, "STORE", False, True, None, None),
+        ("wgrad W2", "XTW", H, F, T, "STORE", False, True, None, None),
+        ("wgrad W1", "XTW", F, H, T, "STORE", False, True, None, None),
+        ("wgrad Wo", "XTW", H, H, T, "STORE", False, True, None, None),
+        ("wgrad Wqkv", "XTW", 3 * H, H, T, "STORE", False, True, None, None),
+        ("plain FFN1 shape", "XWT", T, F, H, "STORE", False, False, None, None),
+    ]
+
+
+def run_gemm_shapes(args, w):
+    """Times every GEMM shape of one layer alone through sky_gemm (bf16 in,
+    fp32 accumulation): L2 flushed by a 256 MB write before each launch,
+    ``--warmup`` untimed and ``--steps`` timed launches per shape (CUDA events
+    around each), median.  sky_gemm has no residual operand, so the two
+    residual-branch forward GEMMs and two data gradients run without it.
+    ``--only`` picks shapes by name (comma-separated substrings)."""
+    import ctypes as C
+
+    import torch
+    from paper_2202_11836_gb300 import _lib as L
+
+    def ptr(t):
+        return C.c_void_p(0 if t is None else int(t.data_ptr()))
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    st = torch.cuda.current_stream(dev)
+    sp = C.c_void_p(int(st.cuda_stream))
+    gen = torch.Generator(device=dev).manual_seed(synth.SEED)
+    flush = torch.empty(256 * 2 ** 20, dtype=torch.uint8, device=dev)
+    forms = {"XWT": L.SKY_GEMM_XWT, "XW": L.SKY_GEMM_XW, "XTW": L.SKY_GEMM_XTW}
+    epis = {"STORE": L.SKY_EPI_STORE, "BIAS_GELU": L.SKY_EPI_BIAS_GELU,
+            "GELU_BWD": L.SKY_EPI_GELU_BWD}
+    bf = L.SKY_DTYPE_BF16
+    picks = [p for p in (args.only or "").split(",") if p]
+    total_us, total_f, rows = 0.0, 0.0, []
+    for name, form, M, N, K, epi, bias, f32, aux_in, aux_out in gemm_shapes(w):
+        if picks and not any(p in name for p in picks):
+            continue
+        a_shape = (K, M) if form == "XTW" else (M, K)
+        b_shape = (N, K) if form == "XWT" else (K, N)
+        A = torch.randn(a_shape, device=dev, generator=gen).bfloat16()
+        Bm = (0.02 * torch.randn(b_shape, device=dev, generator=gen)).bfloat16()
+        Cm = torch.empty((M, N), device=dev, dtype=torch.float32 if f32 else torch.bfloat16)
+        bv = torch.zeros(N, device=dev, dtype=torch.bfloat16) if bias else None
+        ai = torch.rand((M, N), device=dev, generator=gen).half() if aux_in else None
+        ao = torch.empty((M, N), device=dev, dtype=torch.float16) if aux_out else None
+        odt = L.SKY_DTYPE_FP32 if f32 else bf
+        wsb = L.lib().sky_gemm_workspace_bytes(forms[form], M, N, K, bf, odt)
+        ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device=dev)
+        times = []
+        for it in range(args.warmup + args.steps):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            L.call("sky_gemm", forms[form], M, N, K, bf, ptr(A), ptr(Bm), ptr(Cm), odt, epis[epi],
+                   ptr(bv), ptr(ai), ptr(ao), ptr(ws), wsb, None, sp)
+            e1.record(st)
+            e1.synchronize()
+            if it >= args.warmup:
+                times.append(e0.elapsed_time(e1) * 1e3)
+        us = statistics.median(times)
+        f = 2.0 * M * N * K
+        total_us += us
+        total_f += f
+        rows.append({"gemm": name, "M": M, "N": N, "K": K, "epilogue": epi, "fp32_out": f32,
+                     "us": round(us, 2), "tflops": round(f / us / 1e6, 1)})
+        print(f"{name:18s} M={M:6d} N={N:6d} K={K:6d} {epi:9s} f32={int(f32)} "
+              f"{us:8.1f} us {f / us / 1e6:8.1f} TF/s", flush=True)
+    if rows:
+        print(f"TOTAL {total_us:.1f} us  {total_f / total_us / 1e6:.1f} TF/s", flush=True)
+    print(json.dumps({"gemm_shapes": rows, "workload": w.name, "launches_timed": args.steps,
+                      "l2": "flushed before each launch"}), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__)
     ap.add_argument("--gpus", type=int, default=1)
@@ -457,11 +546,17 @@ def main(argv=None):
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--gemm-shapes", action="store_true",
+                    help="time each GEMM shape of one layer alone through sky_gemm")
+    ap.add_argument("--only", default="", help="with --gemm-shapes: shapes whose name "
+                    "contains one of these comma-separated strings")
     args = ap.parse_args(argv)
     assert args.warmup >= 0 and args.steps >= 1
     w = synth.WORKLOADS[args.workload]
     if args.impl == "reference":
         return run_reference(args, w)
+    if args.gemm_shapes:
+        return run_gemm_shapes(args, w)
     return run_gpu(args, w)
 
 

@@ -78,3 +78,15 @@ def test_flop_accounting_matches_closed_form():
     # 80.2 M flop per token per layer at the mean valid length 384 of U{256..512}
     mean_len = (g + 8 * 12 * H * 512 * 16 * 384) / 8 / T
     assert abs(mean_len / 1e6 - 80.2) < 0.1
+
+
+def test_gemm_shapes_cover_one_layer():
+    """The per-shape GEMM table holds the 12 GEMMs of one layer (forward, data
+    and weight gradients), whose FLOPs add up to 6 T (4 H^2 + 2 H F)."""
+    import bench
+    from paper_2202_11836_gb300 import synth
+    w = synth.WORKLOADS["large-s512"]
+    shapes = [s for s in bench.gemm_shapes(w) if not s[0].startswith("plain")]
+    assert len(shapes) == 12
+    T, H, F = w.tokens, w.hidden, w.ffn
+    assert sum(2 * M * N * K for _, _, M, N, K, *_ in shapes) == 6 * T * (4 * H * H + 2 * H * F)
