@@ -537,6 +537,61 @@ def run_gemm_shapes(args, w):
     return 0
 
 
+def run_uneven(args, w):
+    """The load-balanced uneven slices of the 160-layer base-width model
+    (lengths 1, 3, 7, 17; Sec. IV-D partitions), each run on its own: the
+    per-slice step time (graph replays, CUDA events, ``--steps`` after
+    ``--warmup``), the per-layer cost records of sky_slice_layer_cost, and a
+    least-squares fit t(n) = alpha + beta n of slice time over layer count."""
+    import torch
+    from paper_2202_11836_gb300.slice import EncoderSlice
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    st = torch.cuda.current_stream(dev)
+    lens = synth.lengths(w)
+    x = torch.from_numpy(synth.activations(w)).to(dev).to(torch.bfloat16)
+    dy = torch.from_numpy(synth.upstream_grad(w)).to(dev).to(torch.bfloat16)
+    ln = torch.from_numpy(lens).to(dev)
+    y, dx = torch.empty_like(x), torch.empty_like(x)
+    rows = []
+    for lb, le in synth.UNEVEN_SLICES:
+        with EncoderSlice(w.hidden, w.heads, w.ffn, lb, le, w.batch, w.seq, "bf16") as s:
+            for l in range(lb, le):
+                s.set_params(l, synth.layer_params(l, w.hidden, w.ffn, "bf16"))
+            s.step_graph(x, ln, y, dy, dx, st)
+            for _ in range(args.warmup):
+                s.launch_step_graph(st)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record(st)
+            for _ in range(args.steps):
+                s.launch_step_graph(st)
+            e1.record(st)
+            e1.synchronize()
+            ms = e0.elapsed_time(e1) / args.steps
+            s.sync()
+            rec = s.layer_cost(w.batch, w.seq, iters=5)
+        layer_ms = [r["fwd_ms"] + r["bwd_ms"] for r in rec]
+        rows.append({"layers": [lb, le], "n": le - lb, "ms_per_step": round(ms, 4),
+                     "tokens_per_s": round(w.tokens / (ms / 1e3), 1),
+                     "sum_layer_cost_ms": round(sum(layer_ms), 4),
+                     "median_layer_cost_ms": round(statistics.median(layer_ms), 4)})
+    n = np.array([r["n"] for r in rows], float)
+    fits = {}
+    for key in ("ms_per_step", "sum_layer_cost_ms"):
+        t = np.array([r[key] for r in rows])
+        beta, alpha = np.polyfit(n, t, 1)
+        pred = alpha + beta * n
+        r2 = 1.0 - float(((t - pred) ** 2).sum() / ((t - t.mean()) ** 2).sum())
+        fits[key] = {"alpha_ms": round(float(alpha), 4), "beta_ms_per_layer": round(float(beta), 4),
+                     "r2": round(r2, 6)}
+    print(json.dumps({"workload": w.name, "slices": rows, "fit": fits,
+                      "config": config_of(w)}), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__)
     ap.add_argument("--gpus", type=int, default=1)
@@ -548,6 +603,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--gemm-shapes", action="store_true",
                     help="time each GEMM shape of one layer alone through sky_gemm")
+    ap.add_argument("--uneven", action="store_true",
+                    help="time the uneven slices {1,3,7,17} of the 160-layer base-width model")
     ap.add_argument("--only", default="", help="with --gemm-shapes: shapes whose name "
                     "contains one of these comma-separated strings")
     args = ap.parse_args(argv)
@@ -557,6 +614,8 @@ def main(argv=None):
         return run_reference(args, w)
     if args.gemm_shapes:
         return run_gemm_shapes(args, w)
+    if args.uneven:
+        return run_uneven(args, synth.WORKLOADS["base-s128-b16"])
     return run_gpu(args, w)
 
 
