@@ -45,12 +45,15 @@ def to_host(t):
     return t.float().cpu().numpy().astype(np.float64)
 
 
-def run_gpu_slice(w, X, lens, dY, params, affine_layers, eps=1e-12, steps=1, profiling=False):
+def run_gpu_slice(w, X, lens, dY, params, affine_layers, eps=1e-12, steps=1, profiling=False,
+                  graph=False):
     """Runs forward+backward of workload ``w`` on the GPU; returns (Y, dX, grads).
 
     ``steps`` > 1 repeats the step back to back on one stream (results of the
     last one are returned); ``profiling`` runs every kernel in line on the
-    caller's stream (per-kernel timing mode)."""
+    caller's stream (per-kernel timing mode); ``graph`` captures the step as
+    the benchmark runs it (sky_slice_step_graph_create) and returns the
+    results of a replay into zeroed outputs."""
     import torch
     from paper_2202_11836_gb300.slice import EncoderSlice
     B = X.shape[0]
@@ -62,9 +65,18 @@ def run_gpu_slice(w, X, lens, dY, params, affine_layers, eps=1e-12, steps=1, pro
         x = to_device(X, w.dtype)
         ln = torch.from_numpy(np.asarray(lens, np.int32)).cuda()
         dy = to_device(dY, w.dtype)
-        for _ in range(steps):
-            y = s.forward(x, ln)
-            dx = s.backward(dy)
+        if graph:
+            y, dx = torch.empty_like(x), torch.empty_like(x)
+            s.step_graph(x, ln, y, dy, dx)
+            s.sync()
+            for _ in range(steps):
+                y.zero_()
+                dx.zero_()
+                s.launch_step_graph()
+        else:
+            for _ in range(steps):
+                y = s.forward(x, ln)
+                dx = s.backward(dy)
         s.sync()
         grads = [s.get_grads(w.layer_begin + i) for i in range(len(params))]
         return to_host(y), to_host(dx), grads

@@ -51,13 +51,15 @@ def test_base_width_slice_full():
 
 
 def sampled_case(w, sample):
-    """GPU on the whole batch, oracle on the sampled sequences."""
+    """GPU on the whole batch, oracle on the sampled sequences.  The GPU side
+    runs the step as the benchmark times it: captured once as a CUDA graph
+    and replayed."""
     params = synth.slice_params(w, affine="bert")
     X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
     mask = np.zeros(w.batch, bool)
     mask[list(sample)] = True
     dY = dY * mask[:, None, None]
-    Y, dX, grads = run_gpu_slice(w, X, lens, dY, params, None)
+    Y, dX, grads = run_gpu_slice(w, X, lens, dY, params, None, graph=True)
     idx = np.array(sample)
     Yo, dXo, go = oracle_slice(w, X[idx], lens[idx], dY[idx], params)
     rep = compare_slice(w, Y, dX, grads, Yo, dXo, go, rows=idx)
