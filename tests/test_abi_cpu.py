@@ -118,3 +118,55 @@ def test_bf16_rounding_matches_torch():
     x = x.astype(np.float32)
     ref = torch.from_numpy(x).to(torch.bfloat16).float().numpy()
     assert np.array_equal(synth.round_bf16(x), ref)
+
+
+def _kind_c(t, enums):
+    """Storage class of a C type as written in include/*.h."""
+    t = " ".join(t.replace("const", " ").split())
+    if "*" in t:
+        return ("ptr",)
+    table = {"int32_t": ("i", 4), "int": ("i", 4), "int64_t": ("i", 8), "uint64_t": ("u", 8),
+             "size_t": ("u", 8), "float": ("f", 4), "double": ("f", 8), "sky_status": ("i", 4),
+             "void": None}
+    if t in enums:
+        return ("i", 4)
+    assert t in table, f"unmapped C type {t!r}"
+    return table[t]
+
+
+def _kind_ctypes(ct):
+    if ct is None:
+        return None
+    if ct in (C.c_void_p, C.c_char_p) or issubclass(ct, C._Pointer):
+        return ("ptr",)
+    if ct in (C.c_float, C.c_double):
+        return ("f", C.sizeof(ct))
+    signed = ct(-1).value < 0
+    return ("i" if signed else "u", C.sizeof(ct))
+
+
+def test_binding_signatures_match_headers():
+    """Every declared function has the same parameter count, parameter
+    storage classes and return class in the ctypes table as in its header."""
+    decls, enums = {}, set()
+    for h in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if not h.endswith(".h"):
+            continue
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", "", src)
+        enums |= set(re.findall(r"typedef\s+enum\s*\{[^}]*\}\s*(\w+)\s*;", src))
+        for ret, name, params in re.findall(r"([\w\s\*]+?)\b(sky_\w+)\s*\(([^)]*)\)\s*;", src):
+            ret = ret.split("\n")[-1].strip()
+            ps = [p.strip() for p in params.split(",") if p.strip() and p.strip() != "void"]
+            # drop the parameter name: the last identifier of each declarator
+            types = [re.sub(r"\b\w+\s*$", "", p) if re.search(r"[\s\*]\w+\s*$", p) else p
+                     for p in ps]
+            decls[name] = (ret, types)
+    assert set(decls) == set(L._SIGNATURES)
+    for name, (ret, types) in decls.items():
+        restype, argtypes = L._SIGNATURES[name]
+        assert len(argtypes) == len(types), (name, types)
+        assert _kind_ctypes(restype) == _kind_c(ret, enums), (name, ret, restype)
+        for i, (ct, t) in enumerate(zip(argtypes, types)):
+            assert _kind_ctypes(ct) == _kind_c(t, enums), (name, i, t, ct)
