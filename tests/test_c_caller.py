@@ -1,6 +1,9 @@
 """The public headers are plain C: a C99 program that includes all of them
 compiles with warnings as errors, links against libsky_slice.so and runs
-without a GPU (argument rejection and the host-side layer allocator)."""
+without a GPU (argument rejection and the host-side layer allocator).  The
+sizes and field offsets it prints for every public struct must equal those of
+the ctypes structures of the Python binding."""
+import ctypes as C
 import os
 import shutil
 import subprocess
@@ -28,7 +31,17 @@ def test_c99_program_builds_and_runs(tmp_path):
     assert r.returncode == 0, r.stderr
     r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
     assert r.returncode == 0, r.stderr
-    lines = dict(line.split(" ", 1) for line in r.stdout.strip().splitlines())
+    out = r.stdout.strip().splitlines()
+    lines = dict(line.split(" ", 1) for line in out if not line.startswith("layout "))
+    layouts = {ln.split()[1]: list(map(int, ln.split()[2:])) for ln in out
+               if ln.startswith("layout ")}
+    structs = {"sky_slice_config": L.SkySliceConfig, "sky_layer_cost": L.SkyLayerCost,
+               "sky_kernel_stat": L.SkyKernelStat, "sky_optimizer_config": L.SkyOptimizerConfig,
+               "sky_alloc_problem": L.SkyAllocProblem}
+    assert set(layouts) == set(structs)
+    for cname, py in structs.items():
+        want = [C.sizeof(py)] + [getattr(py, f).offset for f, _ in py._fields_]
+        assert layouts[cname] == want, (cname, layouts[cname], want)
     assert lines["create"] == "SKY_ERR_INVALID_ARG 1"
     # Sec. IV-A even split of 9 layers on 3 devices
     assert lines["even"] == "SKY_OK 0 3 6 9"
