@@ -90,3 +90,18 @@ def test_gemm_shapes_cover_one_layer():
     assert len(shapes) == 12
     T, H, F = w.tokens, w.hidden, w.ffn
     assert sum(2 * M * N * K for _, _, M, N, K, *_ in shapes) == 6 * T * (4 * H * H + 2 * H * F)
+
+
+def test_allocation_plan_on_synthetic_layer_costs():
+    """The bench's allocation object runs the host allocator (no GPU) on a
+    160-layer table built from per-layer records: the exact ordered optimum
+    is no worse than the heuristic, and the heuristic no worse than the even
+    split, for devices whose speeds differ as the paper's slow-down factors."""
+    rec = [{"fwd_ms": 0.25, "bwd_ms": 0.45, "param_bytes": 14_000_000,
+            "grad_bytes": 28_000_000, "stash_bytes": 300_000_000} for _ in range(8)]
+    plan = bench.allocation_plan(rec)
+    m = plan["makespan_ms"]
+    assert plan["layers"] == 160 and plan["devices"] == 64
+    assert plan["layer_ms"] == 0.7
+    assert m["best_in_device_order"] <= m["heuristic"] + 1e-9 <= m["even"] + 2e-9
+    assert m["heuristic"] < m["even"]
