@@ -48,8 +48,9 @@ typedef enum { SKY_GEMM_XWT = 0, SKY_GEMM_XW = 1, SKY_GEMM_XTW = 2 } sky_gemm_fo
  *               bf16 inputs (finer than bf16 on its range [-0.17, 1.13]) and
  *               as fp32 for fp32 inputs
  *   GELU_BWD  : C = acc * aux[m,n], aux = GELU'(z) as stored by BIAS_GELU
- * Residual additions are not fused here: the LayerNorm kernels that follow
- * every residual branch point read the fp32 residual themselves. */
+ * sky_gemm takes no residual operand: with the ops of this header the
+ * residual is added by sky_layernorm_fwd (its r operand).  The slice
+ * (sky_slice.h) adds its residuals inside its own GEMM epilogues. */
 typedef enum { SKY_EPI_STORE = 0, SKY_EPI_BIAS_GELU = 1, SKY_EPI_GELU_BWD = 2 } sky_epilogue;
 
 /* Scratch bytes sky_gemm needs for (form, M, N, K) with an fp32 output
