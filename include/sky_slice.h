@@ -109,9 +109,12 @@ typedef struct sky_slice sky_slice;  /* opaque, owned by the library */
 
 /* Creates a slice and allocates its parameters, gradients, stash and
  * workspace on the current CUDA device.  Parameters start at zero.
- * Errors: INVALID_ARG (non-positive sizes, width % heads, l0 >= l1),
- * UNSUPPORTED (bf16 with head dim != 64, or width % 8), OOM (the arena does
- * not fit, or exceeds the cap of sky_debug_set_alloc_cap), CUDA. */
+ * Errors: INVALID_ARG (non-positive sizes, width % heads, l0 >= l1, an
+ * unknown dtype, ln_eps < 0, io_fp32 not 0 or 1, max_batch * max_seq above
+ * 2^30), UNSUPPORTED (bf16: head dim != 64, width or ffn not a multiple of
+ * 8, width above 2048; fp32: head dim above 128, width above 1024 or not a
+ * multiple of 4), OOM (the arena does not fit, or exceeds the cap of
+ * sky_debug_set_alloc_cap), CUDA. */
 sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out);
 
 /* Frees everything the slice owns.  NULL is accepted.  Synchronises the device. */
