@@ -178,11 +178,16 @@ sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_
                                        void* stream);
 sky_status sky_slice_step_graph_launch(sky_slice* s, void* stream);
 
-/* Measures every layer of the slice: runs `iters` forward+backward passes at
- * [B,S] with full-length sequences and synthetic data already on the device
- * (parameters as set), records CUDA events around each layer, and writes the
- * median per-layer times with the analytic FLOPs and the byte counts.
- * n_out must equal layer_end - layer_begin.  Synchronous; overwrites grads. */
+/* Measures every layer of the slice: runs 2 warm-up and `iters` timed
+ * forward+backward passes at [B,S] with full-length sequences on a fixed
+ * pattern written on the device (parameters as set), records CUDA events
+ * around each layer on a stream of its own, and writes the median per-layer
+ * times with the analytic FLOPs and the byte counts.  The weight-gradient
+ * stream joins after every layer, so a layer's time includes its own weight
+ * gradients.  It allocates its input, output and length buffers for the
+ * measurement (cudaMalloc) and frees them before returning.
+ * n_out must equal layer_end - layer_begin.  Synchronous; overwrites grads,
+ * and a following sky_slice_backward needs a new forward (STATE). */
 sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, int32_t iters,
                                 sky_layer_cost* out, int32_t n_out);
 
