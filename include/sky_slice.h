@@ -259,7 +259,13 @@ void sky_debug_set_alloc_cap(uint64_t bytes);
  * handles and threads), for accounting of GPU work. */
 int64_t sky_launch_count(void);
 
+/* Name of a status code ("SKY_OK", "SKY_ERR_INVALID_ARG", ...), a static
+ * string owned by the library; an unknown code gives "SKY_ERR_UNKNOWN". */
 const char* sky_status_string(sky_status st);
+
+/* Message of the calling thread's most recent failed call (empty before the
+ * first failure; a successful call leaves it unchanged).  The string belongs
+ * to the library and stays valid until that thread's next failing call. */
 const char* sky_last_error(void);
 
 #ifdef __cplusplus
