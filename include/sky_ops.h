@@ -155,9 +155,12 @@ sky_status sky_column_sum(const void* x, int32_t T, int32_t N, sky_dtype dtype, 
  * Same arguments and result as sky_column_sum minus the workspace: the
  * partial sums live in a 1 MiB device array inside the library, which every
  * device that loads the library holds until the process exits.
- *   - The first call on a device looks up that array's device address
- *     (cudaGetSymbolAddress) with the device current; make that first call
- *     before capturing the stream into a CUDA graph.
+ *   - Every call looks up that array's device address on the current
+ *     device (cudaGetSymbolAddress, which enqueues no work); the first call
+ *     on a device also loads the library's module there, so make that first
+ *     call before capturing the stream into a CUDA graph.  A device reset
+ *     discards the array's contents with the module; the next call finds
+ *     the new address.
  *   - All calls share the array and it keeps the previous call's contents;
  *     nothing in it needs to start at zero, but calls that may overlap on
  *     the GPU (different streams, or different host threads, same device)

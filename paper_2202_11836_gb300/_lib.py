@@ -79,7 +79,8 @@ _SIGNATURES = {
     "sky_slice_backward": (C.c_int, [_VP, _VP, _VP, _VP]),
     "sky_slice_step_graph_create": (C.c_int, [_VP, _VP, _VP, _I32, _I32, _VP, _VP, _VP, _VP]),
     "sky_slice_step_graph_launch": (C.c_int, [_VP, _VP]),
-    "sky_slice_layer_cost": (C.c_int, [_VP, _I32, _I32, _I32, C.POINTER(SkyLayerCost), _I32]),
+    "sky_slice_layer_cost": (C.c_int, [_VP, _I32, _I32, C.POINTER(_I32), _I32,
+                                        C.POINTER(SkyLayerCost), _I32]),
     "sky_slice_sync": (C.c_int, [_VP]),
     "sky_slice_set_profiling": (C.c_int, [_VP, C.c_int]),
     "sky_slice_kernel_stats": (C.c_int, [_VP, C.POINTER(SkyKernelStat), _I32, C.POINTER(_I32)]),

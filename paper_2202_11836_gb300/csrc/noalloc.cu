@@ -9,8 +9,6 @@
 // entry point serves them: its scratch is a file-scope device array that
 // exists from the moment the library is loaded on a device until the process
 // exits, so nothing is allocated or freed per call.
-#include <mutex>
-
 #include "common.cuh"
 #include "rowwise.h"
 
@@ -20,25 +18,16 @@ namespace {
 constexpr size_t kScratchBytes = size_t(1) << 20;  // 1 MiB per device
 static __device__ __align__(256) unsigned char g_colsum_scratch[kScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-void* g_scratch_ptr[kMaxDevices] = {nullptr};
-
 // Device address of the scratch array on the current device.  Host code only
 // sees a host-side stand-in under the array's name, so the address is looked
-// up once per device (with that device current) and cached.
+// up with the device current.  The lookup is repeated on every call (it is
+// cheap and enqueues nothing): an address cached across calls would dangle
+// after a device reset unloads the module.
 sky_status scratch_on_current_device(void** out) {
-  int dev = 0;
-  SKY_CUDA(cudaGetDevice(&dev));
-  SKY_CHECK(dev >= 0 && dev < kMaxDevices, SKY_ERR_UNSUPPORTED, "device index %d too large", dev);
-  std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_colsum_scratch);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(column-sum scratch)");
-    g_scratch_ptr[dev] = p;
-  }
-  *out = g_scratch_ptr[dev];
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_colsum_scratch);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(column-sum scratch)");
+  *out = p;
   return SKY_OK;
 }
 

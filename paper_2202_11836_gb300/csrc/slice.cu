@@ -580,10 +580,6 @@ __global__ void fill_pattern(void* p, int64_t n, int bf16, float scale, uint32_t
     else static_cast<float*>(p)[i] = v;
   }
 }
-__global__ void fill_int(int32_t* p, int n, int v) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < n) p[i] = v;
-}
 
 }  // namespace
 }  // namespace sky
@@ -972,42 +968,75 @@ sky_status sky_slice_step_graph_launch(sky_slice* s, void* stream) {
   ABI_GUARD_END
 }
 
-sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, int32_t iters,
-                                sky_layer_cost* out, int32_t n_out) {
+// Buffers, stream and events of one layer-cost measurement, released on every
+// return path.
+struct CostScratch {
+  void *x = nullptr, *y = nullptr, *dy = nullptr, *dx = nullptr;
+  int32_t* len = nullptr;
+  cudaStream_t st = nullptr;
+  std::vector<cudaEvent_t> ev;
+  ~CostScratch() {
+    if (st) cudaStreamSynchronize(st);
+    for (auto e : ev)
+      if (e) cudaEventDestroy(e);
+    if (st) cudaStreamDestroy(st);
+    cudaFree(x); cudaFree(y); cudaFree(dy); cudaFree(dx); cudaFree(len);
+  }
+};
+
+sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, const int32_t* lens,
+                                int32_t iters, sky_layer_cost* out, int32_t n_out) {
   ABI_GUARD_BEGIN
   SKY_CHECK(s && out, SKY_ERR_INVALID_ARG, "null argument");
   SKY_CHECK(n_out == s->L, SKY_ERR_INVALID_ARG, "n_out must be %d", s->L);
   SKY_CHECK(iters >= 1 && B >= 1 && S >= 1 && B <= s->cfg.max_batch && S <= s->cfg.max_seq,
             SKY_ERR_INVALID_ARG, "bad B/S/iters");
+  std::vector<int32_t> hlen(B, S);
+  double sum_len = (double)B * S;
+  if (lens) {
+    sum_len = 0;
+    for (int b = 0; b < B; ++b) {
+      SKY_CHECK(lens[b] >= 1 && lens[b] <= S, SKY_ERR_INVALID_ARG,
+                "lens[%d] = %d outside [1, %d]", b, lens[b], S);
+      hlen[b] = lens[b];
+      sum_len += lens[b];
+    }
+  }
+  // The measurement reuses the stash, workspace, gradients and status word:
+  // wait for every step already enqueued on this slice (the caller's stream
+  // of its last call, and the weight-gradient stream) before touching them.
+  if (s->last_stream) SKY_CUDA(cudaStreamSynchronize(s->last_stream));
+  if (s->side) SKY_CUDA(cudaStreamSynchronize(s->side));
+  SKY_CUDA(cudaDeviceSynchronize());
   const bool io32 = s->cfg.io_fp32 && s->cfg.dtype == SKY_DTYPE_BF16;
   const size_t xb = (size_t)B * S * s->H * (io32 ? 4 : s->esz);
-  void *x = nullptr, *y = nullptr, *dy = nullptr, *dx = nullptr;
-  int32_t* len = nullptr;
-  SKY_CUDA(cudaMalloc(&x, xb));
-  SKY_CUDA(cudaMalloc(&y, xb));
-  SKY_CUDA(cudaMalloc(&dy, xb));
-  SKY_CUDA(cudaMalloc(&dx, xb));
-  SKY_CUDA(cudaMalloc(&len, B * sizeof(int32_t)));
-  cudaStream_t st;
-  SKY_CUDA(cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking));
+  CostScratch cs;
+  SKY_CUDA(cudaMalloc(&cs.x, xb));
+  SKY_CUDA(cudaMalloc(&cs.y, xb));
+  SKY_CUDA(cudaMalloc(&cs.dy, xb));
+  SKY_CUDA(cudaMalloc(&cs.dx, xb));
+  SKY_CUDA(cudaMalloc(&cs.len, B * sizeof(int32_t)));
+  SKY_CUDA(cudaStreamCreateWithFlags(&cs.st, cudaStreamNonBlocking));
+  cudaStream_t st = cs.st;
+  SKY_CUDA(cudaMemcpyAsync(cs.len, hlen.data(), B * sizeof(int32_t), cudaMemcpyHostToDevice, st));
   const int64_t n = (int64_t)B * S * s->H;
   const int bf = s->cfg.dtype == SKY_DTYPE_BF16 && !io32;
-  fill_pattern<<<256, 256, 0, st>>>(x, n, bf, 1.0f, 1u);
-  fill_pattern<<<256, 256, 0, st>>>(dy, n, bf, 1e-3f, 2u);
-  fill_int<<<ceil_div(B, 256), 256, 0, st>>>(len, B, S);
-  count_launches(3);
-  std::vector<cudaEvent_t> fm(2 * s->L), bm(2 * s->L);
-  for (auto& e : fm) SKY_CUDA(cudaEventCreate(&e));
-  for (auto& e : bm) SKY_CUDA(cudaEventCreate(&e));
+  fill_pattern<<<256, 256, 0, st>>>(cs.x, n, bf, 1.0f, 1u);
+  fill_pattern<<<256, 256, 0, st>>>(cs.dy, n, bf, 1e-3f, 2u);
+  count_launches(2);
+  cs.ev.assign(4 * s->L, nullptr);
+  for (auto& e : cs.ev) SKY_CUDA(cudaEventCreate(&e));
+  std::vector<cudaEvent_t> fm(cs.ev.begin(), cs.ev.begin() + 2 * s->L);
+  std::vector<cudaEvent_t> bm(cs.ev.begin() + 2 * s->L, cs.ev.end());
   std::vector<std::vector<double>> ft(s->L), bt(s->L);
-  s->B = B; s->S = S; s->d_len = len; s->last_stream = st;
+  s->B = B; s->S = S; s->d_len = cs.len; s->last_stream = st;
   const bool prof = s->prof;
   s->prof = false;
   sky_status rc = SKY_OK;
   const int warm = 2;
   for (int it = 0; it < warm + iters && rc == SKY_OK; ++it) {
-    rc = forward_all(s, x, y, st, &fm);
-    if (rc == SKY_OK) rc = backward_all(s, dy, dx, st, &bm);
+    rc = forward_all(s, cs.x, cs.y, st, &fm);
+    if (rc == SKY_OK) rc = backward_all(s, cs.dy, cs.dx, st, &bm);
     if (rc != SKY_OK) break;
     if (cudaStreamSynchronize(st) != cudaSuccess) { rc = cuda_fail(cudaGetLastError(), "sync"); break; }
     if (it < warm) continue;
@@ -1021,15 +1050,11 @@ sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, int32_t iter
   }
   s->prof = prof;
   s->have_fwd = false;
-  s->last_stream = nullptr;  // the measuring stream is destroyed below
-  for (auto& e : fm) cudaEventDestroy(e);
-  for (auto& e : bm) cudaEventDestroy(e);
-  cudaStreamDestroy(st);
-  cudaFree(x); cudaFree(y); cudaFree(dy); cudaFree(dx); cudaFree(len);
+  s->last_stream = nullptr;  // the measuring stream is destroyed with cs
   if (rc != SKY_OK) return rc;
   const double T = (double)B * S, H = s->H, F = s->F;
   const double gemm_fwd = 2.0 * T * (4.0 * H * H + 2.0 * H * F);
-  const double attn_fwd = 4.0 * H * S * T;  // all query rows against all (valid) keys
+  const double attn_fwd = 4.0 * H * S * sum_len;  // all S query rows against the valid keys
   size_t per_param = 0, per_grad = 0;
   for (int k = 0; k < SKY_NUM_PARAMS; ++k) {
     per_param += param_elems(s, k) * s->esz;

@@ -136,10 +136,17 @@ class EncoderSlice:
     def sync(self) -> None:
         L.call("sky_slice_sync", self.h)
 
-    def layer_cost(self, B: int, S: int, iters: int = 5) -> list:
+    def layer_cost(self, B: int, S: int, iters: int = 5, lens=None) -> list:
+        """Per-layer cost records (sky_slice_layer_cost).  ``lens``: the valid
+        length of each of the B sequences (host ints); None = full length."""
         n = self.layer_end - self.layer_begin
         out = (L.SkyLayerCost * n)()
-        L.call("sky_slice_layer_cost", self.h, B, S, iters, out, n)
+        lp = None
+        if lens is not None:
+            la = np.ascontiguousarray(lens, dtype=np.int32)
+            assert la.shape == (B,)
+            lp = la.ctypes.data_as(C.POINTER(C.c_int32))
+        L.call("sky_slice_layer_cost", self.h, B, S, lp, iters, out, n)
         return [{f: getattr(o, f) for f, _ in L.SkyLayerCost._fields_ if f != "_pad"} for o in out]
 
     def set_profiling(self, on: bool) -> None:

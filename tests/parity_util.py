@@ -98,3 +98,27 @@ def oracle_slice(w, X, lens, dY, params, eps=1e-12):
     return ORC.slice_step(np.asarray(X, np.float64), np.asarray(lens), np.asarray(dY, np.float64),
                           [{k: np.asarray(v, np.float64) for k, v in p.items()} for p in params],
                           w.heads, eps)
+
+
+def oracle_slice_by_sequence(w, X, lens, dY, params, eps=1e-12):
+    """The oracle's slice step on the whole batch, one sequence at a time.
+
+    Each sequence's output and input gradient depend on that sequence alone
+    (attention mixes only within a sequence; every other step acts row by
+    row), and every weight gradient is a sum over the batch's rows, so the
+    per-sequence weight gradients are added here in sequence order.  This
+    keeps only one sequence's activation caches in host memory at a time."""
+    B = X.shape[0]
+    Y = np.empty(X.shape, np.float64)
+    dX = np.empty(X.shape, np.float64)
+    total = None
+    for b in range(B):
+        Yb, dXb, gb = oracle_slice(w, X[b:b + 1], lens[b:b + 1], dY[b:b + 1], params, eps)
+        Y[b], dX[b] = Yb[0], dXb[0]
+        if total is None:
+            total = gb
+        else:
+            for acc, g in zip(total, gb):
+                for k in acc:
+                    acc[k] = acc[k] + g[k]
+    return Y, dX, total

@@ -36,7 +36,7 @@ def test_pipeline_composes_and_heuristic_beats_even():
         y_ref = s.forward(x, ln).cpu().numpy()
         dx_ref = s.backward(dy).cpu().numpy()
         g_ref = [s.get_grads(l) for l in range(L)]
-        costs = s.layer_cost(B, w.seq, iters=3)
+        costs = s.layer_cost(B, w.seq, iters=3, lens=lens)
 
     slow = [1.0, 2.0, 4.0, 7.0]
     t_layer = [r["fwd_ms"] + r["bwd_ms"] for r in costs]

@@ -2,18 +2,17 @@
 GPU (through sky_slice.h) against the float64 oracle on the same seeded
 inputs, every output tensor (Y, dX and the 12 gradients of every layer).
 
-Small cases run in full; the full-size workloads are checked on sampled
-sequences: each sequence's forward and input gradient depend on that sequence
-alone, and with the upstream gradient zero on every other sequence the weight
-gradients equal those of the sampled sequences alone, so the oracle runs on
-the sample while the GPU runs the whole batch in the benchmark's launch
-configuration.
+Every case compares the whole batch.  At the full-size workloads the oracle
+runs one sequence at a time (a sequence's forward and input gradient depend
+on it alone, and weight gradients are sums over sequences), while the GPU runs
+the whole batch in the benchmark's launch configuration.
 """
 import numpy as np
 import pytest
 
 from paper_2202_11836_gb300 import synth
-from parity_util import compare_slice, oracle_slice, run_gpu_slice, to_device, to_host
+from parity_util import (compare_slice, oracle_slice, oracle_slice_by_sequence, run_gpu_slice,
+                         to_device, to_host)
 
 pytestmark = pytest.mark.gpu
 torch = pytest.importorskip("torch")
@@ -50,36 +49,53 @@ def test_base_width_slice_full():
     full_case(synth.WORKLOADS["base-s128"], affine="bert")
 
 
-def sampled_case(w, sample):
-    """GPU on the whole batch, oracle on the sampled sequences.  The GPU side
-    runs the step as the benchmark times it: captured once as a CUDA graph
-    and replayed."""
+def full_batch_case(w):
+    """The whole batch on both sides, with the workload's upstream gradient on
+    every sequence: the GPU runs the step as the benchmark times it (captured
+    once as a CUDA graph and replayed into zeroed outputs); the oracle runs
+    sequence by sequence.  Every row of Y and dX and every gradient of every
+    layer is compared."""
     params = synth.slice_params(w, affine="bert")
     X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    Y, dX, grads = run_gpu_slice(w, X, lens, dY, params, None, graph=True)
+    Yo, dXo, go = oracle_slice_by_sequence(w, X, lens, dY, params)
+    rep = compare_slice(w, Y, dX, grads, Yo, dXo, go)
+    worst = max(rep.items(), key=lambda kv: kv[1][1])
+    print(f"\n{w.name}: worst l2rel {worst[1][1]:.2e} ({worst[0]}), "
+          f"worst maxrel {max(v[0] for v in rep.values()):.2e}")
+    return rep
+
+
+def test_large_width_slice_full_batch():
+    """BERT-large width, 8 layers, S=512, B=16 (the benchmark workload): all
+    16 sequences, every output tensor."""
+    full_batch_case(synth.WORKLOADS["large-s512"])
+
+
+def test_long_sequence_slice_full_batch():
+    """S=2048, B=4, 4 layers (two full-length sequences, two ragged): all 4
+    sequences, every output tensor."""
+    full_batch_case(synth.WORKLOADS["large-s2048"])
+
+
+def test_padding_gradient_isolation_at_full_size():
+    """Full-size batch with the upstream gradient zeroed on all but two
+    sequences: those two match the oracle run on them alone, and the other
+    sequences receive an input gradient of exactly zero."""
+    w = synth.WORKLOADS["large-s512"]
+    lens = synth.lengths(w)
+    sample = (int(np.argmin(lens)), int(np.argmax(lens)))
+    params = synth.slice_params(w, affine="bert")
+    X, dY = synth.activations(w), synth.upstream_grad(w)
     mask = np.zeros(w.batch, bool)
     mask[list(sample)] = True
     dY = dY * mask[:, None, None]
     Y, dX, grads = run_gpu_slice(w, X, lens, dY, params, None, graph=True)
     idx = np.array(sample)
     Yo, dXo, go = oracle_slice(w, X[idx], lens[idx], dY[idx], params)
-    rep = compare_slice(w, Y, dX, grads, Yo, dXo, go, rows=idx)
-    # rows outside the sample receive exactly zero input gradient
+    compare_slice(w, Y, dX, grads, Yo, dXo, go, rows=idx)
     rest = np.where(~mask)[0]
     assert np.all(dX[rest] == 0.0)
-    return rep
-
-
-def test_large_width_slice_sampled():
-    """BERT-large width, 8 layers, S=512, B=16 (full size), 2 sequences sampled."""
-    w = synth.WORKLOADS["large-s512"]
-    lens = synth.lengths(w)
-    sampled_case(w, (int(np.argmin(lens)), int(np.argmax(lens))))
-
-
-def test_long_sequence_slice_sampled():
-    """S=2048, B=4, 4 layers (full size): one full-length and one partial sequence."""
-    w = synth.WORKLOADS["large-s2048"]
-    sampled_case(w, (0, 3))
 
 
 def _slice_run(w, lb, le, X, lens, dY, params, io_fp32=False):
@@ -213,7 +229,7 @@ def test_layer_cost_and_linearity():
         with EncoderSlice(w.hidden, w.heads, w.ffn, lb, le, w.batch, w.seq) as s:
             for l in range(lb, le):
                 s.set_params(l, synth.layer_params(l, w.hidden, w.ffn, "bf16"))
-            rec = s.layer_cost(w.batch, w.seq, iters=3)
+            rec = s.layer_cost(w.batch, w.seq, iters=3, lens=synth.lengths(w))
             assert len(rec) == le - lb
             for r in rec:
                 assert r["fwd_ms"] > 0 and r["bwd_ms"] > 0
@@ -227,6 +243,46 @@ def test_layer_cost_and_linearity():
     assert r2 >= 0.99, (times, r2)
 
 
+def test_layer_cost_counts_the_mask_and_waits_for_queued_work():
+    """sky_slice_layer_cost measures the workload's own lengths (its attention
+    FLOPs count the valid keys) and rejects a length outside [1, S].  Called
+    right after a step that is still queued on the caller's stream, it first
+    waits for that step: the step's y and dx equal those of the same step run
+    alone."""
+    from paper_2202_11836_gb300 import _lib as L
+    from paper_2202_11836_gb300.slice import EncoderSlice
+    w = synth.custom("cost", layers=2, hidden=1024, heads=16, ffn=4096, seq=512, batch=8,
+                     len_lo=100, len_hi=512)
+    params = synth.slice_params(w, affine="random")
+    X, lens, dY = synth.activations(w), synth.lengths(w), synth.upstream_grad(w)
+    T, H, F, S = w.batch * w.seq, w.hidden, w.ffn, w.seq
+    with EncoderSlice(H, w.heads, F, 0, w.layers, w.batch, S) as s:
+        for i, p in enumerate(params):
+            s.set_params(i, p)
+        x, dy = to_device(X, "bf16"), to_device(dY, "bf16")
+        ln = torch.from_numpy(lens).cuda()
+        y_ref = s.forward(x, ln).clone()
+        dx_ref = s.backward(dy).clone()
+        s.sync()
+        y, dx = torch.empty_like(x), torch.empty_like(x)
+        s.forward(x, ln, y)
+        s.backward(dy, dx)
+        rec = s.layer_cost(w.batch, S, iters=2, lens=lens)  # no sync before it
+        torch.cuda.synchronize()
+        assert torch.equal(y, y_ref) and torch.equal(dx, dx_ref)
+        gemm = 2.0 * T * (4 * H * H + 2 * H * F)
+        for r in rec:
+            assert r["fwd_flops"] == pytest.approx(gemm + 4.0 * H * S * lens.sum(), rel=1e-12)
+            assert r["bwd_flops"] == pytest.approx(2 * r["fwd_flops"], rel=1e-12)
+        full = s.layer_cost(w.batch, S, iters=2)
+        assert full[0]["fwd_flops"] == pytest.approx(gemm + 4.0 * H * S * S * w.batch, rel=1e-12)
+        bad = lens.copy()
+        bad[1] = S + 1
+        with pytest.raises(L.SkyError) as e:
+            s.layer_cost(w.batch, S, iters=1, lens=bad)
+        assert e.value.status == L.SKY_ERR_INVALID_ARG
+
+
 def test_layer_cost_feeds_allocator():
     """The per-layer records of sky_slice_layer_cost are the model benchmark
     of Sec. IV-B: their time and bytes form the allocator's layer table, and
@@ -238,7 +294,7 @@ def test_layer_cost_feeds_allocator():
     with EncoderSlice(w.hidden, w.heads, w.ffn, lb, le, w.batch, w.seq) as s:
         for l in range(lb, le):
             s.set_params(l, synth.layer_params(l, w.hidden, w.ffn, "bf16"))
-        rec = s.layer_cost(w.batch, w.seq, iters=3)
+        rec = s.layer_cost(w.batch, w.seq, iters=3, lens=synth.lengths(w))
     lf, lm = allocator.layer_table(rec)
     assert all(f > 0 for f in lf) and all(m > 0 for m in lm)
     t = [r["fwd_ms"] + r["bwd_ms"] for r in rec]
