@@ -75,7 +75,9 @@ sky_status sky_gemm(sky_gemm_form form, int32_t M, int32_t N, int32_t K, sky_dty
 /* Masked scaled dot-product attention, forward (Eq. 1).
  * qkv: [B*S, 3H] (Q | K | V blocks, head a at columns a*D..a*D+D-1 in each);
  * d_len: int32[B] valid lengths; ctx: [B*S, H] out; lse: fp32 [B, A, S] out,
- * the natural-log softmax normaliser of each query row (kept for backward).
+ * the softmax normaliser of each query row in base-2 units,
+ * log2 sum_{j < len} exp2(log2(e) q.k_j / sqrt(D)) (kept for the backward,
+ * which takes it in the same units).
  * bf16 needs D = H/A = 64. */
 sky_status sky_attention_fwd(const void* qkv, const int32_t* d_len, int32_t B, int32_t S,
                              int32_t H, int32_t A, sky_dtype dtype, void* ctx, float* lse,

@@ -116,7 +116,7 @@ __global__ void attn_fwd_f32(const float* __restrict__ qkv, const int32_t* __res
       acc = fmaf(p[j], qkv[((int64_t)b * S + j) * rs + 2 * H + a * D + d], acc);
     ctx[((int64_t)b * S + i) * H + a * D + d] = acc * inv;
   }
-  if (l == 0) lse[((int64_t)b * A + a) * S + i] = mx + logf(sum);
+  if (l == 0) lse[((int64_t)b * A + a) * S + i] = (mx + logf(sum)) * 1.4426950408889634f;  // base 2
 }
 
 // dQ rows (mode 0) or dK/dV rows (mode 1), one warp per row.
@@ -151,7 +151,7 @@ __global__ void attn_bwd_f32(const float* __restrict__ qkv, const float* __restr
       }
       s = warp_sum(s);
       dp = warp_sum(dp);
-      const float p = expf(s * sc - lse_b[i]);
+      const float p = exp2f(fmaf(s, sc * 1.4426950408889634f, -lse_b[i]));
       const float ds = p * (dp - del_b[i]);
       for (int d = l, c = 0; d < D; d += 32, ++c) acc0[c] = fmaf(ds, K(j, d), acc0[c]);
     }
@@ -168,7 +168,7 @@ __global__ void attn_bwd_f32(const float* __restrict__ qkv, const float* __restr
         }
         s = warp_sum(s);
         dp = warp_sum(dp);
-        const float p = expf(s * sc - lse_b[i]);
+        const float p = exp2f(fmaf(s, sc * 1.4426950408889634f, -lse_b[i]));
         const float ds = p * (dp - del_b[i]);
         for (int d = l, c = 0; d < D; d += 32, ++c) {
           acc0[c] = fmaf(ds, Q(i, d), acc0[c]);   // dK

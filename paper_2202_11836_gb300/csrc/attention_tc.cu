@@ -5,23 +5,26 @@
 // 64-key tile j (only tiles below len[b] are visited):
 //   S_j = Q K_j^T                  tcgen05.mma M=128 N=64 K=64 -> TMEM
 //   softmax (4 warps, thread = query row = TMEM lane): row max over the
-//     valid keys, P_j = exp2(S_j log2(e)/sqrt(D) - m) written as bf16 to
-//     shared memory in the 128-byte-swizzled K-major operand layout
-//   O += P_j V_j                   tcgen05.mma M=128 N=64 K=64 -> TMEM
+//     valid keys, P_j = exp2(S_j log2(e)/sqrt(D) - m) written as bf16 pairs
+//     back to tensor memory (tcgen05.st), where the next product reads it
+//   O += P_j V_j                   tcgen05.mma M=128 N=64 K=64, A = P_j from
+//                                  TMEM, B = V_j from shared memory -> TMEM
 // Q, K and V come straight out of the packed QKV activations by TMA (one
 // tensor map, per-head column offsets).  Because a thread owns a whole query
 // row, the row max and row sum need no shuffles.
 //
-// The steps are pipelined inside the CTA: S has two TMEM buffers and P two
-// shared-memory buffers, so the MMA warp computes S_{j+1} (issued one tile
+// The steps are pipelined inside the CTA: S and P have two TMEM buffers each,
+// so the MMA warp computes S_{j+1} (issued one tile
 // ahead) and P_{j-1} V_{j-1} while the softmax warps work on tile j, and K/V
 // tiles stream through a 3-stage TMA ring.  The exponent offset m of a row
 // is only raised when the tile's max exceeds it by more than 2^8 (a factor
 // 256 in P): then O and the row sum are rescaled in TMEM once the pending
 // P V product has landed.  Otherwise P may exceed 1 by at most that factor,
 // which bf16 and the fp32 sums carry with the same relative precision; the
-// final O / l and the log-sum-exp do not depend on m.  All mbarrier waits
-// are time-bounded.
+// final O / l and the log-sum-exp do not depend on m.  The log-sum-exp is
+// kept in base-2 units, lse2 = log2 sum_j exp2(S_ij log2(e)/sqrt(D)), which
+// is what the backward kernels subtract in the exponent.  All mbarrier
+// waits are time-bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -36,14 +39,18 @@ namespace attn_tc {
 constexpr int BQ = 128, BKV = 64, HD = 64;
 constexpr int Q_BYTES = BQ * HD * 2;    // 16 KiB
 constexpr int KV_BYTES = BKV * HD * 2;  // 8 KiB per K or V tile
-constexpr int STAGES = 2;               // backward operand rings
 constexpr int NTHR = 192;               // warp 0 TMA, warp 1 MMA, warps 2..5 softmax
+constexpr int STAGES = 2;               // dK/dV operand ring
 // The backward kernels run eight softmax warps: warps w and w + 4 share TMEM
 // lane quarter w % 4 and take the low / high 32 columns of each 64-wide tile.
-constexpr int NTHR_B = 320;             // warp 0 TMA, warp 1 MMA, warps 2..9 softmax
 constexpr int NSM_B = 256;              // softmax threads in the backward kernels
+// Backward CTAs: warp 0 TMA, warp 1 issues the score products (S and dP),
+// warps 2..9 softmax, warp 10 issues the accumulating products (dQ, or dV
+// and dK).  One thread issues a tcgen05.mma only about every 100 cycles,
+// while an M=128, N=64, K=16 product keeps the tensor pipe busy for about
+// 32, so the two kinds of product are issued side by side by two warps.
+constexpr int NTHR_B = 352;
 constexpr float LOG2E = 1.4426950408889634f;
-constexpr float LN2 = 0.6931471805599453f;
 // Suspend-time hint (ns) of every mbarrier wait: a waiting thread sleeps
 // until the phase completes instead of spinning on issue slots that the
 // softmax warps (the critical path) share with the producer and MMA threads.
@@ -310,7 +317,7 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
           }
         }
       }
-      if (q < S) p.lse[(static_cast<int64_t>(b) * p.A + a) * S + q] = (m + log2f(l)) * LN2;
+      if (q < S) p.lse[(static_cast<int64_t>(b) * p.A + a) * S + q] = m + log2f(l);
     }
   }
   ptx::tc_fence_before();
@@ -394,8 +401,8 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
   uint64_t* s_free = s_full + 1;
   uint64_t* ds_full = s_free + 1;
   uint64_t* dq_done = ds_full + 1;
-  uint64_t* done = dq_done + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* done = dq_done + 1;  // [2], one per issuing warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 2);
 
   const int qt = blockIdx.x, a = blockIdx.y, b = blockIdx.z;
   const int S = p.S, H = p.H;
@@ -413,13 +420,14 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
     ptx::mbar_init(qd_full, 1);
     for (int s = 0; s < DQ_STAGES; ++s) {
       ptx::mbar_init(&kv_full[s], 1);
-      ptx::mbar_init(&kv_empty[s], 1);
+      ptx::mbar_init(&kv_empty[s], 2);  // the tile's S / dP products and its dQ product
     }
     ptx::mbar_init(s_full, 1);
     ptx::mbar_init(s_free, NSM_B);
     ptx::mbar_init(ds_full, NSM_B);
     ptx::mbar_init(dq_done, 1);
-    ptx::mbar_init(done, 1);
+    ptx::mbar_init(&done[0], 1);
+    ptx::mbar_init(&done[1], 1);
     ptx::fence_mbar_init();
     ptx::fence_proxy_async_smem();
   }
@@ -461,11 +469,16 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idS = ptx::idesc_bf16_f32(BQ, BKV, false, false);
-      constexpr uint32_t idQ = ptx::idesc_bf16_f32(BQ, HD, false, true);
       const uint32_t sq = ptx::smem_u32(smem + DQ_Q_OFF), so = ptx::smem_u32(smem + DQ_DO_OFF);
       const uint32_t skv = ptx::smem_u32(smem + DQ_KV_OFF);
-      // S_j = Q K_j^T and dP_j = dO V_j^T (operands already landed)
-      auto mma_sdp = [&](int j) {
+      // S_j = Q K_j^T and dP_j = dO V_j^T, as soon as the softmax warps hold
+      // S_{j-1} / dP_{j-1} in registers (s_free) and K_j / V_j have landed
+      bool ok = ptx::mbar_wait(qd_full, 0, lim, p.status, kWaitHint);
+      for (int j = 0; j < n_kt && ok; ++j) {
+        if (j >= 1 && !ptx::mbar_wait(s_free, (j - 1) & 1, lim, p.status, kWaitHint)) break;
+        if (!ptx::mbar_wait(&kv_full[j % DQ_STAGES], (j / DQ_STAGES) & 1, lim, p.status, kWaitHint))
+          break;
+        ptx::tc_fence_after();
         const uint32_t sk = skv + (j % DQ_STAGES) * 2 * KV_BYTES, sv = sk + KV_BYTES;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
@@ -476,30 +489,21 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
           ptx::tc_mma_f16(tdP, ptx::smem_desc_sw128(so + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(sv + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
         ptx::tc_commit(s_full);
-      };
-      bool ok = ptx::mbar_wait(qd_full, 0, lim, p.status, kWaitHint) &&
-                ptx::mbar_wait(&kv_full[0], 0, lim, p.status, kWaitHint);
-      if (ok) {
-        ptx::tc_fence_after();
-        mma_sdp(0);
+        ptx::tc_commit(&kv_empty[j % DQ_STAGES]);
       }
-      for (int j = 0; j < n_kt && ok; ++j) {
-        // While dS_j is being formed, issue S_{j+1} / dP_{j+1} as soon as the
-        // softmax warps hold S_j / dP_j in registers (s_free) and K_{j+1} /
-        // V_{j+1} have landed; the dQ product of tile j is never held up by
-        // that tile's loads.
-        const int jn = j + 1;
-        bool next_done = jn >= n_kt;
-        auto next_ready = [&] {
-          return ptx::mbar_try_wait(s_free, j & 1) &&
-                 ptx::mbar_try_wait(&kv_full[jn % DQ_STAGES], (jn / DQ_STAGES) & 1);
-        };
-        auto next_issue = [&] {
-          ptx::tc_fence_after();
-          mma_sdp(jn);
-        };
-        if (!ptx::mbar_wait_with(ds_full, j & 1, lim, p.status, kWaitHint, next_done, next_ready,
-                                 next_issue))
+      ptx::tc_commit(&done[0]);
+      ptx::mbar_wait(&done[0], 0, lim, p.status, kWaitHint);
+    }
+  } else if (warp == 10) {
+    // dQ += dS_j K_j, in tile order, from a warp of its own: one thread
+    // issues a tcgen05.mma only about every 100 cycles, so the dQ products
+    // and the score products of the next tile go in side by side
+    if (lane == 0) {
+      constexpr uint32_t idQ = ptx::idesc_bf16_f32(BQ, HD, false, true);
+      const uint32_t skv = ptx::smem_u32(smem + DQ_KV_OFF);
+      for (int j = 0; j < n_kt; ++j) {
+        if (!ptx::mbar_wait(ds_full, j & 1, lim, p.status, kWaitHint)) break;
+        if (!ptx::mbar_wait(&kv_full[j % DQ_STAGES], (j / DQ_STAGES) & 1, lim, p.status, kWaitHint))
           break;
         ptx::tc_fence_after();
         const uint32_t sk = skv + (j % DQ_STAGES) * 2 * KV_BYTES;
@@ -509,16 +513,9 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
                                  idQ, (j > 0 || kk > 0) ? 1u : 0u);
         ptx::tc_commit(dq_done);
         ptx::tc_commit(&kv_empty[j % DQ_STAGES]);
-        if (!next_done) {
-          if (!ptx::mbar_wait(s_free, j & 1, lim, p.status, kWaitHint) ||
-              !ptx::mbar_wait(&kv_full[jn % DQ_STAGES], (jn / DQ_STAGES) & 1, lim, p.status,
-                              kWaitHint))
-            break;
-          next_issue();
-        }
       }
-      ptx::tc_commit(done);
-      ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
+      ptx::tc_commit(&done[1]);
+      ptx::mbar_wait(&done[1], 0, lim, p.status, kWaitHint);
     }
   } else {
     const int q4 = warp & 3;
@@ -528,7 +525,7 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
     const float sl2 = LOG2E * 0.125f;
     const int64_t sidx = (static_cast<int64_t>(b) * p.A + a) * S + (q < S ? q : 0);
-    const float nlse2 = q < S ? -p.lse[sidx] * LOG2E : -INFINITY;  // P = 0 on rows past S
+    const float nlse2 = q < S ? -p.lse[sidx] : -INFINITY;  // P = 0 on rows past S
     const float dl = q < S ? p.delta[sidx] : 0.f;
     bool ok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
@@ -688,8 +685,8 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
   uint64_t* s_free = s_full + 1;
   uint64_t* pds_full = s_free + 1;
   uint64_t* mm_done = pds_full + 1;
-  uint64_t* done = mm_done + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* done = mm_done + 1;  // [2], one per issuing warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 2);
   const int n_qt = (S + BQ2 - 1) / BQ2;
   const uint64_t lim = p.timeout_ns;
 
@@ -697,13 +694,14 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
     ptx::mbar_init(kv_full, 1);
     for (int s = 0; s < STAGES; ++s) {
       ptx::mbar_init(&q_full[s], 32);  // lane 0's expect_tx + 31 lanes' lse/delta stores
-      ptx::mbar_init(&q_empty[s], 1);
+      ptx::mbar_init(&q_empty[s], 2);  // the tile's S^T / dP^T and dV / dK products
     }
     ptx::mbar_init(s_full, 1);
     ptx::mbar_init(s_free, NSM_B);
     ptx::mbar_init(pds_full, NSM_B);
     ptx::mbar_init(mm_done, 1);
-    ptx::mbar_init(done, 1);
+    ptx::mbar_init(&done[0], 1);
+    ptx::mbar_init(&done[1], 1);
     ptx::fence_mbar_init();
     ptx::fence_proxy_async_smem();
   }
@@ -768,14 +766,17 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
         ptx::mbar_wait(&q_full[i & 1], (i >> 1) & 1, lim, p.status, kWaitHint);
     }
   } else if (warp == 1) {
+    // S^T_i = K Q_i^T and dP^T_i = V dO_i^T, as soon as the softmax warps
+    // hold S^T_{i-1} / dP^T_{i-1} in registers (s_free) and Q_i / dO_i have landed
     if (lane == 0) {
       constexpr uint32_t idS = ptx::idesc_bf16_f32(BK2, BQ2, false, false);
-      constexpr uint32_t idG = ptx::idesc_bf16_f32(BK2, HD, false, true);
       const uint32_t sk = ptx::smem_u32(smem + KV_K_OFF), sv = ptx::smem_u32(smem + KV_V_OFF);
-      const uint32_t sp = ptx::smem_u32(smem + KV_P_OFF), sds = ptx::smem_u32(smem + KV_DS_OFF);
-      // S^T_i = K Q_i^T and dP^T_i = V dO_i^T (operands already landed)
-      auto mma_st = [&](int i) {
+      bool ok = ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint);
+      for (int i = 0; i < n_qt && ok; ++i) {
         const int st = i & 1;
+        if (i >= 1 && !ptx::mbar_wait(s_free, (i - 1) & 1, lim, p.status, kWaitHint)) break;
+        if (!ptx::mbar_wait(&q_full[st], (i >> 1) & 1, lim, p.status, kWaitHint)) break;
+        ptx::tc_fence_after();
         const uint32_t sq = ptx::smem_u32(smem + KV_Q_OFF + st * QO2_BYTES);
         const uint32_t so = ptx::smem_u32(smem + KV_O_OFF + st * QO2_BYTES);
 #pragma unroll
@@ -787,30 +788,21 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
           ptx::tc_mma_f16(tdPT, ptx::smem_desc_sw128(sv + kk * 32, 16, 1024),
                           ptx::smem_desc_sw128(so + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
         ptx::tc_commit(s_full);
-      };
-      bool ok = ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint) &&
-                ptx::mbar_wait(&q_full[0], 0, lim, p.status, kWaitHint);
-      if (ok) {
-        ptx::tc_fence_after();
-        mma_st(0);
+        ptx::tc_commit(&q_empty[st]);
       }
-      for (int i = 0; i < n_qt && ok; ++i) {
+      ptx::tc_commit(&done[0]);
+      ptx::mbar_wait(&done[0], 0, lim, p.status, kWaitHint);
+    }
+  } else if (warp == 10) {
+    // dV += P^T_i dO_i and dK += dS^T_i Q_i, in tile order, from a warp of
+    // its own so that they go in beside the next tile's score products
+    if (lane == 0) {
+      constexpr uint32_t idG = ptx::idesc_bf16_f32(BK2, HD, false, true);
+      const uint32_t sp = ptx::smem_u32(smem + KV_P_OFF), sds = ptx::smem_u32(smem + KV_DS_OFF);
+      for (int i = 0; i < n_qt; ++i) {
         const int st = i & 1;
-        // as in the dQ kernel: tile i+1's S^T / dP^T go in as soon as tile i's
-        // are in registers and Q_{i+1} / dO_{i+1} have landed, without holding
-        // up tile i's dV / dK products
-        const int in = i + 1;
-        bool next_done = in >= n_qt;
-        auto next_ready = [&] {
-          return ptx::mbar_try_wait(s_free, i & 1) &&
-                 ptx::mbar_try_wait(&q_full[in & 1], (in >> 1) & 1);
-        };
-        auto next_issue = [&] {
-          ptx::tc_fence_after();
-          mma_st(in);
-        };
-        if (!ptx::mbar_wait_with(pds_full, i & 1, lim, p.status, kWaitHint, next_done, next_ready, next_issue))
-          break;
+        if (!ptx::mbar_wait(pds_full, i & 1, lim, p.status, kWaitHint)) break;
+        if (!ptx::mbar_wait(&q_full[st], (i >> 1) & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
         const uint32_t sq = ptx::smem_u32(smem + KV_Q_OFF + st * QO2_BYTES);
         const uint32_t so = ptx::smem_u32(smem + KV_O_OFF + st * QO2_BYTES);
@@ -825,15 +817,9 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
         }
         ptx::tc_commit(mm_done);
         ptx::tc_commit(&q_empty[st]);
-        if (!next_done) {
-          if (!ptx::mbar_wait(s_free, i & 1, lim, p.status, kWaitHint) ||
-              !ptx::mbar_wait(&q_full[in & 1], (in >> 1) & 1, lim, p.status, kWaitHint))
-            break;
-          next_issue();
-        }
       }
-      ptx::tc_commit(done);
-      ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
+      ptx::tc_commit(&done[1]);
+      ptx::mbar_wait(&done[1], 0, lim, p.status, kWaitHint);
     }
   } else {
     const int q4 = warp & 3;
@@ -865,10 +851,10 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
       uint32_t pp[16], dd[16];
 #pragma unroll
       for (int t = 0; t < 32; t += 4) {
-        // lse / delta of queries t .. t+3: one broadcast 16-byte load each
+        // base-2 log-sum-exp / delta of queries t .. t+3: one broadcast 16-byte load each
         const float4 lq = *reinterpret_cast<const float4*>(l2 + t);
         const float4 dq = *reinterpret_cast<const float4*>(l2 + BQ2 + t);
-        const float lv[4] = {lq.x * LOG2E, lq.y * LOG2E, lq.z * LOG2E, lq.w * LOG2E};
+        const float lv[4] = {lq.x, lq.y, lq.z, lq.w};
         const float dlv[4] = {dq.x, dq.y, dq.z, dq.w};
         float pt[4], ds[4];
 #pragma unroll
