@@ -389,8 +389,8 @@ def run_gpu(args, w):
     per_layer_flops = statistics.median([r["fwd_flops"] + r["bwd_flops"] for r in rec])
 
     # 3b. the local parameter update (Sec. III), timed on its own: AdamW over
-    # every parameter of the slice, an HBM stream of 30 bytes per parameter
-    s.optimizer_init("adamw", lr=2e-5, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01)
+    # every parameter of the slice, an HBM stream of 20-30 bytes per parameter
+    s.optimizer_init(args.optimizer, lr=2e-5, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01)
     n_params = sum(int(np.prod(v)) for v in s.shapes().values()) * w.layers
     for _ in range(3):
         s.optimizer_step(2e-5, stream)
@@ -404,9 +404,14 @@ def run_gpu(args, w):
     t1.record(stream)
     t1.synchronize()
     upd_ms = t0.elapsed_time(t1) / n_upd
-    upd_gbs = 30.0 * n_params / (upd_ms / 1e3) / 1e9
-    optimizer = {"kind": "adamw", "params": n_params, "ms": round(upd_ms, 4),
-                 "bytes_per_param": 30, "achieved_gbs": round(upd_gbs, 1),
+    # bytes per parameter: AdamW reads g, w, m, v and writes w, m, v (and, in a
+    # bf16 slice, the parameter rounded to bf16); SGD reads g, w, b and writes
+    # w, b (and the bf16 parameter).  An fp32 slice updates its parameters in place.
+    bpp = (30 if args.optimizer == "adamw" else 22) if w.dtype == "bf16" else \
+        (28 if args.optimizer == "adamw" else 20)
+    upd_gbs = bpp * n_params / (upd_ms / 1e3) / 1e9
+    optimizer = {"kind": args.optimizer, "params": n_params, "ms": round(upd_ms, 4),
+                 "bytes_per_param": bpp, "achieved_gbs": round(upd_gbs, 1),
                  "peak_gbs": pk["hbm"], "frac": round(upd_gbs / pk["hbm"], 4)}
 
     # 4. end to end through the public API with host buffers
@@ -635,6 +640,8 @@ def main(argv=None):
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--optimizer", default="adamw", choices=["adamw", "sgd"],
+                    help="local update rule timed after the step")
     ap.add_argument("--sustain-s", type=float, default=2.0,
                     help="length of the second, sustained timed region (seconds; 0 = skip)")
     ap.add_argument("--gemm-shapes", action="store_true",

@@ -76,6 +76,10 @@ typedef struct {
                            fp32 boundaries a chain of slices [a,b), [b,c) reproduces
                            slice [a,c) bit for bit; with slice-dtype boundaries
                            they agree up to one rounding of the boundary tensor. */
+  int32_t stash_slots;  /* activation stashes kept (0 or 1: one).  With M > 1, up to M
+                           forwards (sky_slice_forward_slot, slots 0..M-1) may precede
+                           their backwards, as the micro-batches of a pipelined step do
+                           (Sec. III); the stash memory grows M-fold. */
 } sky_slice_config;
 
 /* Per-layer cost record (Sec. IV-B: the model benchmark's per-layer FLOPs
@@ -110,8 +114,8 @@ typedef struct sky_slice sky_slice;  /* opaque, owned by the library */
 /* Creates a slice and allocates its parameters, gradients, stash and
  * workspace on the current CUDA device.  Parameters start at zero.
  * Errors: INVALID_ARG (non-positive sizes, width % heads, l0 >= l1, an
- * unknown dtype, ln_eps < 0, io_fp32 not 0 or 1, max_batch * max_seq above
- * 2^30), UNSUPPORTED (bf16: head dim != 64, width or ffn not a multiple of
+ * unknown dtype, ln_eps < 0, io_fp32 not 0 or 1, stash_slots outside
+ * [0, 64], max_batch * max_seq above 2^30), UNSUPPORTED (bf16: head dim != 64, width or ffn not a multiple of
  * 8, width above 2048; fp32: head dim above 128, width above 1024 or not a
  * multiple of 4), OOM (the arena does not fit, or exceeds the cap of
  * sky_debug_set_alloc_cap), CUDA. */
@@ -154,6 +158,33 @@ sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, 
  * Errors: STATE (no forward since create), INVALID_ARG (null), UNSUPPORTED
  * (dy not 16-byte aligned). */
 sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stream);
+
+/* Micro-batched use (Sec. III: a device runs the forward passes of several
+ * micro-batches before their backward passes, and its layers' gradients are
+ * the sum over the micro-batches).  sky_slice_forward_slot is
+ * sky_slice_forward keeping the activations in stash `slot`
+ * (0 <= slot < stash_slots); sky_slice_backward_slot is sky_slice_backward
+ * for the most recent forward into that slot (its x, d_len, B, S).  With
+ * accumulate == 0 the backward overwrites the gradients; with accumulate == 1
+ * it adds this micro-batch's gradients to them (each layer's gradients are
+ * formed in a scratch set and added on the device, in call order, so a
+ * fixed order of calls gives the same bits).  sky_slice_forward /
+ * sky_slice_backward are slot 0 without accumulation.  Slots are
+ * independent: a forward into slot m leaves the other slots' stashes as
+ * they were.  Errors: as the calls they extend; INVALID_ARG (slot out of
+ * range, accumulate not 0 or 1), STATE (no forward into the slot),
+ * UNSUPPORTED (accumulate == 1 on a slice with stash_slots < 2). */
+sky_status sky_slice_forward_slot(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,
+                                  int32_t S, void* y, int32_t slot, void* stream);
+sky_status sky_slice_backward_slot(sky_slice* s, const void* dy, void* dx, int32_t slot,
+                                   int32_t accumulate, void* stream);
+
+/* Emulates a slower device (the slow_down factor of Sec. V-B): enqueues on
+ * `stream` one single-thread kernel that returns after `ns` nanoseconds of
+ * wall time, so work enqueued behind it on that stream starts that much
+ * later while other streams keep the GPU's SMs.  ns <= 10^10, else
+ * INVALID_ARG; 0 enqueues nothing. */
+sky_status sky_device_delay(uint64_t ns, void* stream);
 
 /* A device's training step over its slice (Sec. III: forward through its
  * layers, then backward in reverse order) as one CUDA graph.

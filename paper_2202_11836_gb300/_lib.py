@@ -25,7 +25,8 @@ class SkySliceConfig(C.Structure):
     _fields_ = [("width", C.c_int32), ("heads", C.c_int32), ("ffn", C.c_int32),
                 ("layer_begin", C.c_int32), ("layer_end", C.c_int32),
                 ("max_batch", C.c_int32), ("max_seq", C.c_int32),
-                ("dtype", C.c_int), ("ln_eps", C.c_float), ("io_fp32", C.c_int32)]
+                ("dtype", C.c_int), ("ln_eps", C.c_float), ("io_fp32", C.c_int32),
+                ("stash_slots", C.c_int32)]
 
 
 class SkyLayerCost(C.Structure):
@@ -77,6 +78,9 @@ _SIGNATURES = {
     "sky_slice_get_grads": (C.c_int, [_VP, _I32, C.POINTER(_VP), C.c_int]),
     "sky_slice_forward": (C.c_int, [_VP, _VP, _VP, _I32, _I32, _VP, _VP]),
     "sky_slice_backward": (C.c_int, [_VP, _VP, _VP, _VP]),
+    "sky_slice_forward_slot": (C.c_int, [_VP, _VP, _VP, _I32, _I32, _VP, _I32, _VP]),
+    "sky_slice_backward_slot": (C.c_int, [_VP, _VP, _VP, _I32, _I32, _VP]),
+    "sky_device_delay": (C.c_int, [C.c_uint64, _VP]),
     "sky_slice_step_graph_create": (C.c_int, [_VP, _VP, _VP, _I32, _I32, _VP, _VP, _VP, _VP]),
     "sky_slice_step_graph_launch": (C.c_int, [_VP, _VP]),
     "sky_slice_layer_cost": (C.c_int, [_VP, _I32, _I32, C.POINTER(_I32), _I32,

@@ -27,6 +27,9 @@
 
 namespace sky {
 
+constexpr int kMaxStashSlots = 64;
+constexpr uint64_t kMaxDelayNs = 10ull * 1000 * 1000 * 1000;  // sky_device_delay: 10 s
+
 namespace {
 thread_local std::string g_last_error;
 uint64_t g_alloc_cap = 0;
@@ -156,8 +159,24 @@ struct sky_slice {
   sky::opt::Tensor* d_opt_tensors = nullptr;
   sky::opt::Chunk* d_opt_chunks = nullptr;
   int opt_chunks = 0;
-  // state of the most recent forward
-  bool have_fwd = false;
+  // Activation stashes: slot m holds everything the backward pass of the
+  // micro-batch whose forward used slot m needs (stash_slots of them, so
+  // that several forwards can precede their backwards, as in a micro-batched
+  // pipeline).  slot_layers[m][i] has layer i's parameter and gradient
+  // pointers (shared by all slots) and slot m's stash pointers; `layers` is
+  // the view of the slot the current call uses.
+  int n_slots = 1;
+  std::vector<std::vector<sky::LayerBufs>> slot_layers;
+  // per slot: the batch shape and lengths of its most recent forward
+  std::vector<char> slot_fwd;
+  std::vector<int> slot_B, slot_S;
+  std::vector<const int32_t*> slot_len;
+  // gradient accumulation: a backward with accumulate = 1 writes each
+  // layer's gradients into this scratch set and adds it into the layer's
+  // gradients on the weight-gradient stream (one layer's worth, reused)
+  float* gscr[SKY_NUM_PARAMS] = {};
+  bool accumulate = false;
+  // batch shape and lengths of the pass in progress (the slot in use)
   int B = 0, S = 0;
   const int32_t* d_len = nullptr;
   cudaStream_t last_stream = nullptr;
@@ -356,6 +375,9 @@ sky_status forward_layer(sky_slice* s, int i, void* y_out, cudaStream_t st) {
 sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, const float* dY2,
                           int k, void* dx, cudaStream_t st, cudaStream_t sw) {
   LayerBufs& Lb = s->layers[i];
+  // gradients go to the layer's buffers, or with accumulation to the scratch
+  // set that is added into them at the end of the layer
+  float* const* G = s->accumulate ? s->gscr : Lb.g;
   const int B = s->B, S = s->S, H = s->H, A = s->A, F = s->F;
   const int T = B * S;
   const sky_dtype dt = s->cfg.dtype;
@@ -399,16 +421,16 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   {
     Timed t(s, st, P_LN_BWD, 0, (dye + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(dY, dy_dt, dY2, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
-                          bf ? s->dU2_32 : nullptr, s->dU2b, Lb.g[10], Lb.g[11], Lb.g[9],
+                          bf ? s->dU2_32 : nullptr, s->dU2b, G[10], G[11], G[9],
                           bf ? s->lnp[0] : s->ws, bf ? s->lnp_bytes : s->ws_bytes, st,
                           bf ? &ln_parts : nullptr, s->d_status));
   }
   SKY_TRY(fork(0));
-  if (bf) SKY_TRY(ln_reduce(0, Lb.g[10], Lb.g[11], Lb.g[9]));
+  if (bf) SKY_TRY(ln_reduce(0, G[10], G[11], G[9]));
   // a10 + a11: dW2 = dU2^T G (on sw, beside the data gradient);
   //            dZ = (dU2 W2) * GELU'(Z);
   //            db1 = sum_rows dZ (fused into the bf16 epilogue; a column-sum pass for fp32)
-  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, Lb.g[8], true,
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, F, T, s->dU2b, Lb.G, G[8], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
   SKY_TRY(done(0));
   SKY_TRY(reuse(1));
@@ -421,19 +443,19 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
                      SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr));
     Timed t(s, st, P_COLSUM, 0, e * T * F);
-    SKY_TRY(column_sum(s->dH, T, F, dt, Lb.g[7], s->ws, s->ws_bytes, st));
+    SKY_TRY(column_sum(s->dH, T, F, dt, G[7], s->ws, s->ws_bytes, st));
   }
   SKY_TRY(fork(1));
   if (bf) {  // db1 = sum of the fused partials
     Timed t(s, sw, P_COLSUM, 0, 4.0 * db1_rows * F);
-    SKY_CUDA(gemm::reduce_rows_f32(s->db1p, db1_rows, F, Lb.g[7], sw));
+    SKY_CUDA(gemm::reduce_rows_f32(s->db1p, db1_rows, F, G[7], sw));
   }
   // a12: dX1 = dZ W1 + dU2 (fp32; bf16: dU2 added by the GEMM epilogue, fp32:
   // by the LN1 backward);  dW1 = dZ^T X1
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dP1, true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, nullptr, 0,
                    bf ? s->dU2_32 : nullptr));
-  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, F, H, T, s->dH, Lb.X1b, Lb.g[6], true,
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, F, H, T, s->dH, Lb.X1b, G[6], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
   SKY_TRY(done(1));
   // a13: LN1 backward of dX1 = P1 + dU2 -> dU1 (fp32 + dtype), dgamma1, dbeta1, dbo
@@ -442,16 +464,16 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, st, P_LN_BWD, 0, (bf ? 4.0 : 8.0) * T * H + (4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? nullptr : static_cast<float*>(s->dU2b),
                           Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H, dt, bf ? s->dR[k] : nullptr,
-                          dU1b, Lb.g[4], Lb.g[5], Lb.g[3], bf ? s->lnp[1] : s->ws,
+                          dU1b, G[4], G[5], G[3], bf ? s->lnp[1] : s->ws,
                           bf ? s->lnp_bytes : s->ws_bytes, st, bf ? &ln_parts : nullptr,
                           s->d_status));
   }
   SKY_TRY(fork(2));
-  if (bf) SKY_TRY(ln_reduce(1, Lb.g[4], Lb.g[5], Lb.g[3]));
+  if (bf) SKY_TRY(ln_reduce(1, G[4], G[5], G[3]));
   // a14: dctx = dU1 Wo;  dWo = dU1^T ctx
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, H, dU1b, Lb.p[2], s->dctx, false,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
-  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, H, T, dU1b, Lb.ctx, Lb.g[2], true,
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, H, H, T, dU1b, Lb.ctx, G[2], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
   SKY_TRY(done(2));
   // a15: attention backward -> dQKV
@@ -465,10 +487,10 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   if (bf) {  // dbqkv = the attention kernels' column partials, added in order (on sw)
     const int rows = B * ceil_div(S, 128);
     Timed t(s, sw, P_COLSUM, 0, 4.0 * rows * 3.0 * H);
-    SKY_CUDA(gemm::reduce_rows_f32(s->qkvp, rows, 3 * H, Lb.g[1], sw));
+    SKY_CUDA(gemm::reduce_rows_f32(s->qkvp, rows, 3 * H, G[1], sw));
   } else {  // dbqkv = column sums of dQKV
     Timed t(s, sw, P_COLSUM, 0, e * T * 3.0 * H);
-    SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, Lb.g[1], s->ws, s->ws_bytes, sw));
+    SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, G[1], s->ws, s->ws_bytes, sw));
   }
   // a16: dX = dQKV Wqkv + dU1;  dWqkv = dQKV^T X.  bf16: dU1 is added by the
   // GEMM epilogue (straight into dx for the slice's first layer with fp32
@@ -487,9 +509,14 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     else
       SKY_CUDA(cudaMemcpyAsync(dx, s->dP[k], (size_t)T * H * 4, cudaMemcpyDeviceToDevice, st));
   }
-  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, 3 * H, H, T, s->dqkv, Lb.Xb, Lb.g[0], true,
+  SKY_TRY(run_gemm(s, sw, P_GEMM_WGRAD, SKY_GEMM_XTW, 3 * H, H, T, s->dqkv, Lb.Xb, G[0], true,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr, nullptr, ws2, ws2b));
   SKY_TRY(done(3));
+  if (s->accumulate) {  // Lb.g += scratch: both are the 12 tensors laid out alike, contiguous
+    const int64_t n = (Lb.g[SKY_NUM_PARAMS - 1] + param_elems(s, SKY_NUM_PARAMS - 1)) - Lb.g[0];
+    Timed t(s, sw, P_COPY, 0, 12.0 * n);
+    SKY_TRY(add_f32(Lb.g[0], s->gscr[0], n, SKY_DTYPE_FP32, Lb.g[0], sw));
+  }
   return SKY_OK;
 }
 
@@ -581,6 +608,18 @@ __global__ void fill_pattern(void* p, int64_t n, int bf16, float scale, uint32_t
   }
 }
 
+// Occupies the stream for `ns` nanoseconds of wall time (one thread polling
+// the global timer, sleeping between polls), then returns.
+__global__ void delay_kernel(uint64_t ns) {
+  if (threadIdx.x != 0) return;
+  uint64_t t0, t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  do {
+    __nanosleep(2000);
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  } while (t - t0 < ns);
+}
+
 }  // namespace
 }  // namespace sky
 
@@ -650,7 +689,7 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
                        4 * align_up((size_t)T * 4);
   s->param_bytes = pb * s->L;
   s->grad_bytes = gb * s->L;
-  s->stash_bytes = stash * s->L;
+  s->stash_bytes = stash * s->L * s->n_slots;
   s->ws_bytes = align_up(workspace_need(s, T));
   s->ws2_bytes = bf ? align_up(side_workspace_need(s, T)) : 0;
   s->lnp_bytes = bf ? align_up(layernorm_bwd_ws((int)T, s->H)) : 0;
@@ -660,7 +699,8 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   // db1p | qkvp | status | x32 (bf16)
   const size_t wk = (bf ? 7 : 6) * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
                     align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes +
-                    s->ws2_bytes + 2 * s->lnp_bytes + s->db1p_bytes + s->qkvp_bytes + 256;
+                    s->ws2_bytes + 2 * s->lnp_bytes + s->db1p_bytes + s->qkvp_bytes + 256 +
+                    (s->n_slots > 1 ? gb : 0);  // gradient-accumulation scratch (one layer)
   s->ws_bytes_total = wk;
   *total = s->param_bytes + s->grad_bytes + s->stash_bytes + wk;
   return SKY_OK;
@@ -681,6 +721,8 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
             "unknown dtype");
   SKY_CHECK(c.ln_eps >= 0.f, SKY_ERR_INVALID_ARG, "ln_eps must be >= 0");
   SKY_CHECK(c.io_fp32 == 0 || c.io_fp32 == 1, SKY_ERR_INVALID_ARG, "io_fp32 must be 0 or 1");
+  SKY_CHECK(c.stash_slots >= 0 && c.stash_slots <= kMaxStashSlots, SKY_ERR_INVALID_ARG,
+            "stash_slots must be in [0, %d]", kMaxStashSlots);
   const int D = c.width / c.heads;
   if (c.dtype == SKY_DTYPE_BF16) {
     SKY_CHECK(D == 64, SKY_ERR_UNSUPPORTED, "bf16 slices need head dim 64 (got %d)", D);
@@ -698,6 +740,7 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   s->L = c.layer_end - c.layer_begin;
   s->H = c.width; s->A = c.heads; s->F = c.ffn; s->D = D;
   s->esz = c.dtype == SKY_DTYPE_BF16 ? 2 : 4;
+  s->n_slots = c.stash_slots > 1 ? c.stash_slots : 1;
   size_t total = 0;
   plan_slice(s, &total);
   if (g_alloc_cap && total > g_alloc_cap) {
@@ -735,10 +778,7 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   const size_t t32 = (size_t)T * s->H * 4;
   const bool bf = c.dtype == SKY_DTYPE_BF16;
   const size_t lse_b = (size_t)c.max_batch * s->A * c.max_seq * 4;
-  s->layers.resize(s->L);
-  for (auto& Lb : s->layers) {
-    for (int k = 0; k < SKY_NUM_PARAMS; ++k) Lb.p[k] = take(param_elems(s, k) * s->esz);
-    for (int k = 0; k < SKY_NUM_PARAMS; ++k) Lb.g[k] = static_cast<float*>(take(param_elems(s, k) * 4));
+  auto take_stash = [&](LayerBufs& Lb) {
     Lb.Xb = take(th); Lb.ctx = take(th); Lb.X1b = take(th);
     Lb.QKV = take((size_t)T * 3 * s->H * s->esz);
     Lb.Gp = take((size_t)T * s->F * s->esz);
@@ -750,6 +790,12 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
     Lb.rstd1 = static_cast<float*>(take((size_t)T * 4));
     Lb.mean2 = static_cast<float*>(take((size_t)T * 4));
     Lb.rstd2 = static_cast<float*>(take((size_t)T * 4));
+  };
+  s->layers.resize(s->L);
+  for (auto& Lb : s->layers) {
+    for (int k = 0; k < SKY_NUM_PARAMS; ++k) Lb.p[k] = take(param_elems(s, k) * s->esz);
+    for (int k = 0; k < SKY_NUM_PARAMS; ++k) Lb.g[k] = static_cast<float*>(take(param_elems(s, k) * 4));
+    take_stash(Lb);
   }
   for (int k = 0; k < 2; ++k) {
     s->dP[k] = static_cast<float*>(take(t32));
@@ -773,6 +819,17 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   if (s->qkvp_bytes) s->qkvp = static_cast<float*>(take(s->qkvp_bytes));
   s->d_status = static_cast<int32_t*>(take(4));
   if (bf) s->x32 = static_cast<float*>(take(t32));
+  // further stash slots (parameters and gradients are shared), and the
+  // gradient-accumulation scratch, laid out like one layer's gradients
+  s->slot_layers.assign(s->n_slots, s->layers);
+  for (int m = 1; m < s->n_slots; ++m)
+    for (auto& Lb : s->slot_layers[m]) take_stash(Lb);
+  if (s->n_slots > 1)
+    for (int k = 0; k < SKY_NUM_PARAMS; ++k) s->gscr[k] = static_cast<float*>(take(param_elems(s, k) * 4));
+  s->slot_fwd.assign(s->n_slots, 0);
+  s->slot_B.assign(s->n_slots, 0);
+  s->slot_S.assign(s->n_slots, 0);
+  s->slot_len.assign(s->n_slots, nullptr);
   if (bf) {
     // the weight-gradient side stream and its events
     bool ok = cudaStreamCreateWithFlags(&s->side, cudaStreamNonBlocking) == cudaSuccess;
@@ -877,10 +934,12 @@ sky_status sky_slice_get_grads(sky_slice* s, int32_t layer, void* const* tensors
   ABI_GUARD_END
 }
 
-sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,
-                             int32_t S, void* y, void* stream) {
+sky_status sky_slice_forward_slot(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,
+                                  int32_t S, void* y, int32_t slot, void* stream) {
   ABI_GUARD_BEGIN
   SKY_CHECK(s && x && d_len && y, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(slot >= 0 && slot < s->n_slots, SKY_ERR_INVALID_ARG, "slot %d outside [0, %d)", slot,
+            s->n_slots);
   SKY_CHECK(B >= 1 && S >= 1, SKY_ERR_INVALID_ARG, "B and S must be >= 1 (got %d, %d)", B, S);
   SKY_CHECK(B <= s->cfg.max_batch && S <= s->cfg.max_seq, SKY_ERR_INVALID_ARG,
             "B=%d S=%d exceed max_batch=%d max_seq=%d", B, S, s->cfg.max_batch, s->cfg.max_seq);
@@ -888,24 +947,58 @@ sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, 
   SKY_CHECK((reinterpret_cast<uintptr_t>(y) & 15) == 0, SKY_ERR_UNSUPPORTED,
             "y must be 16-byte aligned");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s->layers = s->slot_layers[slot];
   s->B = B; s->S = S; s->d_len = d_len; s->last_stream = st;
-  s->have_fwd = false;
+  s->slot_fwd[slot] = 0;
   SKY_TRY(forward_all(s, x, y, st, nullptr));
-  s->have_fwd = true;
+  s->slot_fwd[slot] = 1;
+  s->slot_B[slot] = B; s->slot_S[slot] = S; s->slot_len[slot] = d_len;
+  return SKY_OK;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_backward_slot(sky_slice* s, const void* dy, void* dx, int32_t slot,
+                                   int32_t accumulate, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(s && dy && dx, SKY_ERR_INVALID_ARG, "null argument");
+  SKY_CHECK(slot >= 0 && slot < s->n_slots, SKY_ERR_INVALID_ARG, "slot %d outside [0, %d)", slot,
+            s->n_slots);
+  SKY_CHECK(accumulate == 0 || accumulate == 1, SKY_ERR_INVALID_ARG, "accumulate must be 0 or 1");
+  SKY_CHECK(!accumulate || s->n_slots > 1, SKY_ERR_UNSUPPORTED,
+            "gradient accumulation needs a slice created with stash_slots >= 2");
+  SKY_CHECK(s->slot_fwd[slot], SKY_ERR_STATE, "backward needs a forward into slot %d first", slot);
+  SKY_CHECK((reinterpret_cast<uintptr_t>(dy) & 15) == 0, SKY_ERR_UNSUPPORTED,
+            "dy must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  s->layers = s->slot_layers[slot];
+  s->B = s->slot_B[slot]; s->S = s->slot_S[slot]; s->d_len = s->slot_len[slot];
+  s->last_stream = st;
+  s->accumulate = accumulate != 0;
+  const sky_status rc = backward_all(s, dy, dx, st, nullptr);
+  s->accumulate = false;
+  return rc;
+  ABI_GUARD_END
+}
+
+sky_status sky_slice_forward(sky_slice* s, const void* x, const int32_t* d_len, int32_t B,
+                             int32_t S, void* y, void* stream) {
+  return sky_slice_forward_slot(s, x, d_len, B, S, y, 0, stream);
+}
+
+sky_status sky_device_delay(uint64_t ns, void* stream) {
+  ABI_GUARD_BEGIN
+  SKY_CHECK(ns <= kMaxDelayNs, SKY_ERR_INVALID_ARG, "delay of %llu ns above the %llu ns limit",
+            (unsigned long long)ns, (unsigned long long)kMaxDelayNs);
+  if (ns == 0) return SKY_OK;
+  delay_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(ns);
+  count_launches(1);
+  SKY_CUDA(cudaGetLastError());
   return SKY_OK;
   ABI_GUARD_END
 }
 
 sky_status sky_slice_backward(sky_slice* s, const void* dy, void* dx, void* stream) {
-  ABI_GUARD_BEGIN
-  SKY_CHECK(s && dy && dx, SKY_ERR_INVALID_ARG, "null argument");
-  SKY_CHECK(s->have_fwd, SKY_ERR_STATE, "backward needs a forward on this slice first");
-  SKY_CHECK((reinterpret_cast<uintptr_t>(dy) & 15) == 0, SKY_ERR_UNSUPPORTED,
-            "dy must be 16-byte aligned");
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  s->last_stream = st;
-  return backward_all(s, dy, dx, st, nullptr);
-  ABI_GUARD_END
+  return sky_slice_backward_slot(s, dy, dx, 0, 0, stream);
 }
 
 sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_t* d_len,
@@ -929,6 +1022,7 @@ sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_
   cudaStream_t cs = s->cap_stream;
   const int64_t n0 = sky_launch_count();
   SKY_CUDA(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
+  s->layers = s->slot_layers[0];
   s->B = B; s->S = S; s->d_len = d_len;
   sky_status rc = forward_all(s, x, y, cs, nullptr);
   if (rc == SKY_OK) rc = backward_all(s, dy, dx, cs, nullptr);
@@ -963,7 +1057,8 @@ sky_status sky_slice_step_graph_launch(sky_slice* s, void* stream) {
   count_launches(static_cast<int>(s->step_launches));
   s->B = s->step_B; s->S = s->step_S; s->d_len = s->step_len;
   s->last_stream = st;
-  s->have_fwd = true;
+  s->slot_fwd[0] = 1;
+  s->slot_B[0] = s->step_B; s->slot_S[0] = s->step_S; s->slot_len[0] = s->step_len;
   return SKY_OK;
   ABI_GUARD_END
 }
@@ -1029,6 +1124,7 @@ sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, const int32_
   std::vector<cudaEvent_t> fm(cs.ev.begin(), cs.ev.begin() + 2 * s->L);
   std::vector<cudaEvent_t> bm(cs.ev.begin() + 2 * s->L, cs.ev.end());
   std::vector<std::vector<double>> ft(s->L), bt(s->L);
+  s->layers = s->slot_layers[0];
   s->B = B; s->S = S; s->d_len = cs.len; s->last_stream = st;
   const bool prof = s->prof;
   s->prof = false;
@@ -1049,7 +1145,7 @@ sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, const int32_
     }
   }
   s->prof = prof;
-  s->have_fwd = false;
+  s->slot_fwd[0] = 0;
   s->last_stream = nullptr;  // the measuring stream is destroyed with cs
   if (rc != SKY_OK) return rc;
   const double T = (double)B * S, H = s->H, F = s->F;

@@ -30,18 +30,18 @@ class EncoderSlice:
 
     def __init__(self, width: int, heads: int, ffn: int, layer_begin: int, layer_end: int,
                  max_batch: int, max_seq: int, dtype: str = "bf16", ln_eps: float = 1e-12,
-                 io_fp32: bool = False):
+                 io_fp32: bool = False, stash_slots: int = 1):
         self.H, self.A, self.F = width, heads, ffn
         self.layer_begin, self.layer_end = layer_begin, layer_end
         self.dtype = dtype
         self.io_fp32 = io_fp32
         cfg = L.SkySliceConfig(width, heads, ffn, layer_begin, layer_end, max_batch, max_seq,
                                L.SKY_DTYPE_BF16 if dtype == "bf16" else L.SKY_DTYPE_FP32,
-                               ln_eps, 1 if io_fp32 else 0)
+                               ln_eps, 1 if io_fp32 else 0, stash_slots)
         h = C.c_void_p()
         L.call("sky_slice_create", C.byref(cfg), C.byref(h))
         self.h = h
-        self._fwd_keep = None
+        self._fwd_keep = {}
 
     # ----------------------------------------------------------- parameters
     def shapes(self):
@@ -101,22 +101,29 @@ class EncoderSlice:
         return dict(zip(PARAM_NAMES, bufs))
 
     # -------------------------------------------------------------- compute
-    def forward(self, x, lens, y=None, stream=None):
-        """x: device [B, S, H] tensor (slice dtype); lens: device int32 [B]."""
+    def forward(self, x, lens, y=None, stream=None, slot: int = 0):
+        """x: device [B, S, H] tensor (slice dtype); lens: device int32 [B].
+        ``slot`` picks the activation stash (sky_slice_forward_slot)."""
         import torch
         B, S, H = x.shape
         assert H == self.H and x.is_contiguous() and lens.dtype == torch.int32
         if y is None:
             y = torch.empty_like(x)
-        L.call("sky_slice_forward", self.h, _ptr(x), _ptr(lens), B, S, _ptr(y), _stream_ptr(stream))
-        self._fwd_keep = (x, lens)
+        L.call("sky_slice_forward_slot", self.h, _ptr(x), _ptr(lens), B, S, _ptr(y), slot,
+               _stream_ptr(stream))
+        if not hasattr(self, "_fwd_keep") or not isinstance(self._fwd_keep, dict):
+            self._fwd_keep = {}
+        self._fwd_keep[slot] = (x, lens)
         return y
 
-    def backward(self, dy, dx=None, stream=None):
+    def backward(self, dy, dx=None, stream=None, slot: int = 0, accumulate: bool = False):
+        """Backward of the last forward into ``slot``; ``accumulate`` adds the
+        gradients to the current ones instead of overwriting them."""
         import torch
         if dx is None:
             dx = torch.empty_like(dy)
-        L.call("sky_slice_backward", self.h, _ptr(dy), _ptr(dx), _stream_ptr(stream))
+        L.call("sky_slice_backward_slot", self.h, _ptr(dy), _ptr(dx), slot, 1 if accumulate else 0,
+               _stream_ptr(stream))
         return dx
 
     def step_graph(self, x, lens, y, dy, dx, stream=None) -> None:

@@ -47,13 +47,13 @@ int main(void) {
   printf("launches %lld\n", (long long)sky_launch_count());
 
 #define OFF(T, f) (unsigned long)offsetof(T, f)
-  printf("layout sky_slice_config %lu %lu %lu %lu %lu %lu %lu %lu %lu %lu %lu\n",
+  printf("layout sky_slice_config %lu %lu %lu %lu %lu %lu %lu %lu %lu %lu %lu %lu\n",
          (unsigned long)sizeof(sky_slice_config), OFF(sky_slice_config, width),
          OFF(sky_slice_config, heads), OFF(sky_slice_config, ffn),
          OFF(sky_slice_config, layer_begin), OFF(sky_slice_config, layer_end),
          OFF(sky_slice_config, max_batch), OFF(sky_slice_config, max_seq),
          OFF(sky_slice_config, dtype), OFF(sky_slice_config, ln_eps),
-         OFF(sky_slice_config, io_fp32));
+         OFF(sky_slice_config, io_fp32), OFF(sky_slice_config, stash_slots));
   printf("layout sky_layer_cost %lu %lu %lu %lu %lu %lu %lu %lu %lu %lu %lu\n",
          (unsigned long)sizeof(sky_layer_cost), OFF(sky_layer_cost, layer),
          OFF(sky_layer_cost, _pad), OFF(sky_layer_cost, fwd_ms), OFF(sky_layer_cost, bwd_ms),
