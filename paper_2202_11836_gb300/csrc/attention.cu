@@ -20,8 +20,12 @@ using bf16 = __nv_bfloat16;
 
 // delta[b,a,s] = sum_d dctx[b,s,a,d] * ctx[b,s,a,d]  (equals sum_j P_sj dP_sj)
 // One warp per token row; each lane takes 8 consecutive elements (16 bytes
-// of bf16) per step, and the 8 lanes covering one 64-wide head reduce with
-// shuffles.  Requires D == 64.
+// of bf16) per 256-column group, and the 8 lanes covering one 64-wide head
+// reduce with shuffles.  NV > 0: the row has exactly NV groups, and every
+// load of the row is issued before the first product (more bytes in flight
+// per warp); NV == 0: any H that is a multiple of 64, one group at a time.
+// Requires D == 64.
+template <int NV>
 __global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __restrict__ dctx, int S,
                                 int H, int A, int64_t rows, float* __restrict__ delta) {
   pdl_trigger();
@@ -30,24 +34,41 @@ __global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __rest
   const int l = threadIdx.x & 31;
   if (row >= rows) return;
   const int64_t b = row / S, s = row % S;
-  for (int c0 = 0; c0 < H; c0 += 256) {
-    const int col = c0 + l * 8;
+  auto dot8 = [](const uint4& x, const uint4& y) {
+    const __nv_bfloat162* xs = reinterpret_cast<const __nv_bfloat162*>(&x);
+    const __nv_bfloat162* ys = reinterpret_cast<const __nv_bfloat162*>(&y);
     float acc = 0.f;
-    if (col < H) {
-      const uint4 x = *reinterpret_cast<const uint4*>(ctx + row * H + col);
-      const uint4 y = *reinterpret_cast<const uint4*>(dctx + row * H + col);
-      const __nv_bfloat162* xs = reinterpret_cast<const __nv_bfloat162*>(&x);
-      const __nv_bfloat162* ys = reinterpret_cast<const __nv_bfloat162*>(&y);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float2 p = __bfloat1622float2(xs[i]), q = __bfloat1622float2(ys[i]);
-        acc += p.x * q.x + p.y * q.y;
-      }
+    for (int i = 0; i < 4; ++i) {
+      const float2 p = __bfloat1622float2(xs[i]), q = __bfloat1622float2(ys[i]);
+      acc += p.x * q.x + p.y * q.y;
     }
+    return acc;
+  };
+  auto finish = [&](float acc, int col) {
     acc += __shfl_xor_sync(0xffffffffu, acc, 1);
     acc += __shfl_xor_sync(0xffffffffu, acc, 2);
     acc += __shfl_xor_sync(0xffffffffu, acc, 4);
     if ((l & 7) == 0 && col < H) delta[(b * A + col / HD) * S + s] = acc;
+  };
+  if constexpr (NV > 0) {
+    uint4 x[NV], y[NV];
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+      x[v] = *reinterpret_cast<const uint4*>(ctx + row * H + v * 256 + l * 8);
+      y[v] = *reinterpret_cast<const uint4*>(dctx + row * H + v * 256 + l * 8);
+    }
+#pragma unroll
+    for (int v = 0; v < NV; ++v) finish(dot8(x[v], y[v]), v * 256 + l * 8);
+  } else {
+    for (int c0 = 0; c0 < H; c0 += 256) {
+      const int col = c0 + l * 8;
+      float acc = 0.f;
+      if (col < H)
+        acc = dot8(*reinterpret_cast<const uint4*>(ctx + row * H + col),
+                   *reinterpret_cast<const uint4*>(dctx + row * H + col));
+      finish(acc, col);
+    }
   }
 }
 
@@ -227,9 +248,16 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
   const int dblocks = ceil_div(rows * A * 32, 256);
   if (dt == SKY_DTYPE_BF16) {
     SKY_CHECK(D == attn::HD, SKY_ERR_UNSUPPORTED, "bf16 attention needs head dim 64 (got %d)", D);
-    const cudaError_t le = launch_pdl(attn::attn_delta_bf16, dim3(ceil_div(rows * 32, 256)), dim3(256),
-                                      0, stream, 1, static_cast<const __nv_bfloat16*>(ctx),
-                                      static_cast<const __nv_bfloat16*>(dctx), S, H, A, rows, delta);
+    const auto* c = static_cast<const __nv_bfloat16*>(ctx);
+    const auto* dc = static_cast<const __nv_bfloat16*>(dctx);
+    const dim3 g(ceil_div(rows * 32, 256)), blk(256);
+    cudaError_t le;
+    switch (H % 256 == 0 ? H / 256 : 0) {
+      case 3: le = launch_pdl(attn::attn_delta_bf16<3>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
+      case 4: le = launch_pdl(attn::attn_delta_bf16<4>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
+      case 8: le = launch_pdl(attn::attn_delta_bf16<8>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
+      default: le = launch_pdl(attn::attn_delta_bf16<0>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
+    }
     count_launches(1);
     if (le != cudaSuccess) return cuda_fail(le, "attention delta launch");
     return attention_bwd_tc(qkv, dctx, lse, delta, lens, B, S, H, A, dqkv, status, 2000000000ull,

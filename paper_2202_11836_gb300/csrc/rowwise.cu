@@ -8,6 +8,8 @@
 // statistics are fp32, two-pass in registers, reduced with warp shuffles.
 // Column sums never use floating-point atomics: each CTA writes per-column
 // partials, and a second pass adds them in a fixed order.
+#include <algorithm>
+
 #include "common.cuh"
 #include "ptx.cuh"
 #include "gemm.h"
@@ -412,31 +414,82 @@ __global__ void __launch_bounds__(32 * (SB_WARPS + 1), 1) ln_bwd_stream_kernel(
 }
 
 // out_k[n] = sum_b part[k][b][n] for the non-null outputs, in a fixed order:
-// CTA (cx, k) owns 32 columns; its 8 warps each add every 8th partial row
-// (coalesced 128-byte reads), then the 8 warp sums are added in order.
-__global__ void __launch_bounds__(256) reduce_partials(const float* __restrict__ part, int nblk,
-                                                       int N, float* out0, float* out1,
-                                                       float* out2) {
+// CTA (cx, k) owns 32 columns; warp w of its RP_WARPS warps adds the partial
+// rows b = w + RP_WARPS * (4 i + j) into accumulator j (coalesced 128-byte
+// reads, four rows in flight per warp), the four accumulators are added as
+// (a0 + a1) + (a2 + a3), and the warp sums are added in warp order.
+constexpr int RP_WARPS = 16;
+__global__ void __launch_bounds__(RP_WARPS * 32) reduce_partials(const float* __restrict__ part,
+                                                                 int nblk, int N, float* out0,
+                                                                 float* out1, float* out2) {
   pdl_trigger();
   pdl_wait();
-  __shared__ float red[8][33];
+  __shared__ float red[RP_WARPS][33];
   const int k = blockIdx.y;
   float* out = k == 0 ? out0 : (k == 1 ? out1 : out2);
   if (out == nullptr) return;  // uniform over the CTA
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int n = blockIdx.x * 32 + lane;
-  float s = 0.f;
+  float a[4] = {0.f, 0.f, 0.f, 0.f};
   if (n < N) {
     const float* p = part + (int64_t)k * nblk * N + n;
-    for (int b = w; b < nblk; b += 8) s += p[(int64_t)b * N];
+    int b = w;
+    for (; b + 3 * RP_WARPS < nblk; b += 4 * RP_WARPS) {
+      float v[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) v[j] = p[(int64_t)(b + j * RP_WARPS) * N];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) a[j] += v[j];
+    }
+    // fewer than four rows left: at most three
+    if (b < nblk) a[0] += p[(int64_t)b * N];
+    if (b + RP_WARPS < nblk) a[1] += p[(int64_t)(b + RP_WARPS) * N];
+    if (b + 2 * RP_WARPS < nblk) a[2] += p[(int64_t)(b + 2 * RP_WARPS) * N];
   }
-  red[w][lane] = s;
+  red[w][lane] = (a[0] + a[1]) + (a[2] + a[3]);
   __syncthreads();
   if (w == 0 && n < N) {
     float t = 0.f;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) t += red[j][lane];
+    for (int j = 0; j < RP_WARPS; ++j) t += red[j][lane];
     out[n] = t;
+  }
+}
+
+// Several fixed-order column reductions in one launch: segment y = blockIdx.y
+// computes segs[y].out[n] = sum_b segs[y].part[b][n] over its rows, exactly
+// as reduce_partials does (so the same partials give the same bits).
+__global__ void __launch_bounds__(RP_WARPS * 32) reduce_segments(const ColSegments segs) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float red[RP_WARPS][33];
+  const ColSegment& sg = segs.seg[blockIdx.y];
+  const int N = sg.cols, nblk = sg.rows;
+  if (blockIdx.x * 32 >= N) return;  // uniform over the CTA
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int n = blockIdx.x * 32 + lane;
+  float a[4] = {0.f, 0.f, 0.f, 0.f};
+  if (n < N) {
+    const float* p = sg.part + n;
+    int b = w;
+    for (; b + 3 * RP_WARPS < nblk; b += 4 * RP_WARPS) {
+      float v[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) v[j] = p[(int64_t)(b + j * RP_WARPS) * N];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) a[j] += v[j];
+    }
+    if (b < nblk) a[0] += p[(int64_t)b * N];
+    if (b + RP_WARPS < nblk) a[1] += p[(int64_t)(b + RP_WARPS) * N];
+    if (b + 2 * RP_WARPS < nblk) a[2] += p[(int64_t)(b + 2 * RP_WARPS) * N];
+  }
+  red[w][lane] = (a[0] + a[1]) + (a[2] + a[3]);
+  __syncthreads();
+  if (w == 0 && n < N) {
+    float t = 0.f;
+#pragma unroll
+    for (int j = 0; j < RP_WARPS; ++j) t += red[j][lane];
+    sg.out[n] = t;
   }
 }
 
@@ -675,16 +728,27 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
 sky_status layernorm_bwd_reduce(const void* ws, int parts, int H, float* dgamma, float* dbeta,
                                 float* dbias, cudaStream_t st) {
   dim3 grid(ceil_div(H, 32), 3);
-  launch_pdl(rw::reduce_partials, dim3(grid), dim3(256), 0, st, 1, static_cast<const float*>(ws), parts, H, dgamma,
+  launch_pdl(rw::reduce_partials, dim3(grid), dim3(rw::RP_WARPS * 32), 0, st, 1, static_cast<const float*>(ws), parts, H, dgamma,
                                             dbeta, dbias);
   count_launches(1);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "layernorm backward reduce launch");
 }
 
+sky_status reduce_column_segments(const ColSegments& segs, cudaStream_t st) {
+  if (segs.n <= 0) return SKY_OK;
+  int max_cols = 0;
+  for (int i = 0; i < segs.n; ++i) max_cols = std::max(max_cols, segs.seg[i].cols);
+  launch_pdl(rw::reduce_segments, dim3(ceil_div(max_cols, 32), segs.n), dim3(rw::RP_WARPS * 32), 0,
+             st, 1, segs);
+  count_launches(1);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? SKY_OK : cuda_fail(e, "column-segment reduce launch");
+}
+
 namespace gemm {
 cudaError_t reduce_rows_f32(const float* part, int rows, int N, float* out, cudaStream_t stream) {
-  launch_pdl(rw::reduce_partials, dim3(dim3(ceil_div(N, 32), 1)), dim3(256), 0, stream, 1, part, rows, N, out, nullptr,
+  launch_pdl(rw::reduce_partials, dim3(dim3(ceil_div(N, 32), 1)), dim3(rw::RP_WARPS * 32), 0, stream, 1, part, rows, N, out, nullptr,
                                                                   nullptr);
   count_launches(1);
   return cudaGetLastError();
@@ -754,7 +818,7 @@ sky_status column_sum(const void* x, int rows, int N, sky_dtype dt, float* out, 
         static_cast<const __nv_bfloat16*>(x), rows, N, part);
   else
     launch_pdl(rw::colsum_partial<float>, dim3(grid), dim3(256), 0, st, 1, static_cast<const float*>(x), rows, N, part);
-  launch_pdl(rw::reduce_partials, dim3(dim3(ceil_div(N, 32), 1)), dim3(256), 0, st, 1, part, groups, N, out, nullptr,
+  launch_pdl(rw::reduce_partials, dim3(dim3(ceil_div(N, 32), 1)), dim3(rw::RP_WARPS * 32), 0, st, 1, part, groups, N, out, nullptr,
                                                                 nullptr);
   count_launches(2);
   const cudaError_t e = cudaGetLastError();

@@ -32,6 +32,21 @@ sky_status layernorm_bwd(const void* dy, sky_dtype dy_dt, const float* dy2, cons
 // on another stream ordered after it, adds them in a fixed order.
 sky_status layernorm_bwd_reduce(const void* ws, int parts, int H, float* dgamma, float* dbeta,
                                 float* dbias, cudaStream_t st);
+// Fixed-order column sums of several partial matrices in one launch:
+// seg[i].out[n] = sum over b < seg[i].rows of seg[i].part[b * cols + n].
+// The same partials give the same bits as layernorm_bwd_reduce and
+// gemm::reduce_rows_f32.
+struct ColSegment {
+  const float* part;
+  float* out;
+  int rows, cols;
+};
+constexpr int kMaxColSegments = 8;
+struct ColSegments {
+  ColSegment seg[kMaxColSegments];
+  int n;
+};
+sky_status reduce_column_segments(const ColSegments& segs, cudaStream_t st);
 sky_status add_f32(const float* a, const float* b, int64_t n, sky_dtype out_dt, void* out,
                    cudaStream_t st);
 sky_status f32_to_bf16(const float* x, int64_t n, void* out, cudaStream_t st);

@@ -139,15 +139,22 @@ struct sky_slice {
   size_t ws2_bytes = 0;
   // Column partials whose fixed-order reduction (a bias / LayerNorm-parameter
   // gradient, needed by nothing downstream) also runs on the side stream:
-  // lnp[0] / lnp[1] of the LN2 / LN1 backward, db1p of the fused db1.
-  void* lnp[2] = {nullptr, nullptr};
+  // lnp[k][0] / lnp[k][1] of the LN2 / LN1 backward, db1p[k] of the fused
+  // db1.  Two sets, k = the layer's parity, so that a layer's partials are
+  // still intact when its one batched reduction runs on the weight-gradient
+  // stream while the data-gradient chain moves on to the next layer.
+  // ev_red[k]: that reduction is done (the layer two further down may reuse
+  // set k); ev_red_live[k]: recorded by the current backward call.
+  void* lnp[2][2] = {};
   size_t lnp_bytes = 0;
-  float* db1p = nullptr;
+  float* db1p[2] = {};
   size_t db1p_bytes = 0;
+  cudaEvent_t ev_red[2] = {};
+  bool ev_red_live[2] = {};
   // column partials of dQKV written by the attention backward kernels (one
   // row per 128-row tile of every sequence), summed into dbqkv on the side
   // stream
-  float* qkvp = nullptr;
+  float* qkvp[2] = {};
   size_t qkvp_bytes = 0;
   // local parameter update (Sec. III): fp32 master weights and state in one
   // allocation, the tensor and chunk tables the update kernel walks
@@ -409,24 +416,24 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   };
   void* ws2 = bf ? s->ws2 : nullptr;
   const size_t ws2b = s->ws2_bytes;
-  // bf16: the column-sum reductions of this layer's bias / LayerNorm-parameter
-  // gradients run on sw too, from partials in buffers of their own
-  int ln_parts = 0, db1_rows = 0;
-  auto ln_reduce = [&](int j, float* dg, float* db, float* dbias) -> sky_status {
-    Timed t(s, sw, P_COLSUM, 0, 3.0 * ln_parts * H * 4.0);
-    return layernorm_bwd_reduce(s->lnp[j], ln_parts, H, dg, db, dbias, sw);
-  };
+  // bf16: the column sums behind this layer's bias and LayerNorm-parameter
+  // gradients (LN2 and LN1 partials per CTA, db1 partials per 32 rows from
+  // the FFN2 data-gradient epilogue, dbqkv partials per 128-row tile from the
+  // attention backward) land in partial buffers of set k and are added up by
+  // one fixed-order launch on sw at the end of the layer.  Set k was last
+  // used by the layer two above; wait for its reduction before reusing it.
+  int ln2_parts = 0, ln1_parts = 0, db1_rows = 0;
+  if (bf && two && s->ev_red_live[k]) SKY_CUDA(cudaStreamWaitEvent(st, s->ev_red[k], 0));
   // a9: LN2 backward -> dU2 (fp32 + dtype), dgamma2, dbeta2, db2
   SKY_TRY(reuse(0));
   {
     Timed t(s, st, P_LN_BWD, 0, (dye + 4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(dY, dy_dt, dY2, Lb.U2, Lb.p[10], Lb.mean2, Lb.rstd2, T, H, dt,
                           bf ? s->dU2_32 : nullptr, s->dU2b, G[10], G[11], G[9],
-                          bf ? s->lnp[0] : s->ws, bf ? s->lnp_bytes : s->ws_bytes, st,
-                          bf ? &ln_parts : nullptr, s->d_status));
+                          bf ? s->lnp[k][0] : s->ws, bf ? s->lnp_bytes : s->ws_bytes, st,
+                          bf ? &ln2_parts : nullptr, s->d_status));
   }
   SKY_TRY(fork(0));
-  if (bf) SKY_TRY(ln_reduce(0, G[10], G[11], G[9]));
   // a10 + a11: dW2 = dU2^T G (on sw, beside the data gradient);
   //            dZ = (dU2 W2) * GELU'(Z);
   //            db1 = sum_rows dZ (fused into the bf16 epilogue; a column-sum pass for fp32)
@@ -438,7 +445,7 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, st, P_GEMM_DGRAD, 2.0 * T * F * H, 0);
     SKY_TRY(gemm::launch_bf16(SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
                               SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr, s->ws, s->ws_bytes,
-                              s->d_status, st, nullptr, s->db1p, s->db1p_bytes, &db1_rows));
+                              s->d_status, st, nullptr, s->db1p[k], s->db1p_bytes, &db1_rows));
   } else {
     SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, F, H, s->dU2b, Lb.p[8], s->dH, false,
                      SKY_EPI_GELU_BWD, nullptr, Lb.Gp, nullptr));
@@ -446,10 +453,6 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     SKY_TRY(column_sum(s->dH, T, F, dt, G[7], s->ws, s->ws_bytes, st));
   }
   SKY_TRY(fork(1));
-  if (bf) {  // db1 = sum of the fused partials
-    Timed t(s, sw, P_COLSUM, 0, 4.0 * db1_rows * F);
-    SKY_CUDA(gemm::reduce_rows_f32(s->db1p, db1_rows, F, G[7], sw));
-  }
   // a12: dX1 = dZ W1 + dU2 (fp32; bf16: dU2 added by the GEMM epilogue, fp32:
   // by the LN1 backward);  dW1 = dZ^T X1
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, F, s->dH, Lb.p[6], s->dP1, true,
@@ -464,12 +467,11 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
     Timed t(s, st, P_LN_BWD, 0, (bf ? 4.0 : 8.0) * T * H + (4.0 + 4.0 + (bf ? e : 0.0)) * T * H + 8.0 * T);
     SKY_TRY(layernorm_bwd(s->dP1, SKY_DTYPE_FP32, bf ? nullptr : static_cast<float*>(s->dU2b),
                           Lb.U1, Lb.p[4], Lb.mean1, Lb.rstd1, T, H, dt, bf ? s->dR[k] : nullptr,
-                          dU1b, G[4], G[5], G[3], bf ? s->lnp[1] : s->ws,
-                          bf ? s->lnp_bytes : s->ws_bytes, st, bf ? &ln_parts : nullptr,
+                          dU1b, G[4], G[5], G[3], bf ? s->lnp[k][1] : s->ws,
+                          bf ? s->lnp_bytes : s->ws_bytes, st, bf ? &ln1_parts : nullptr,
                           s->d_status));
   }
   SKY_TRY(fork(2));
-  if (bf) SKY_TRY(ln_reduce(1, G[4], G[5], G[3]));
   // a14: dctx = dU1 Wo;  dWo = dU1^T ctx
   SKY_TRY(run_gemm(s, st, P_GEMM_DGRAD, SKY_GEMM_XW, T, H, H, dU1b, Lb.p[2], s->dctx, false,
                    SKY_EPI_STORE, nullptr, nullptr, nullptr));
@@ -481,13 +483,34 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   {
     Timed t(s, st, P_ATTN_BWD, 8.0 * H * S * (double)T, e * T * 8.0 * H);
     SKY_TRY(attention_bwd(Lb.QKV, Lb.ctx, s->dctx, Lb.lse, s->d_len, B, S, H, A, dt, s->dqkv,
-                          s->delta, s->d_status, st, bf ? s->qkvp : nullptr));
+                          s->delta, s->d_status, st, bf ? s->qkvp[k] : nullptr));
   }
   SKY_TRY(fork(3));
-  if (bf) {  // dbqkv = the attention kernels' column partials, added in order (on sw)
-    const int rows = B * ceil_div(S, 128);
-    Timed t(s, sw, P_COLSUM, 0, 4.0 * rows * 3.0 * H);
-    SKY_CUDA(gemm::reduce_rows_f32(s->qkvp, rows, 3 * H, G[1], sw));
+  if (bf) {
+    // the layer's eight column reductions in one fixed-order launch on sw:
+    // dgamma2, dbeta2, db2 and dgamma1, dbeta1, dbo from the LayerNorm
+    // partials, db1 from the FFN2 data-gradient partials, dbqkv from the
+    // attention backward's partials
+    const int qkv_rows = B * ceil_div(S, 128);
+    const float* l2 = static_cast<const float*>(s->lnp[k][0]);
+    const float* l1 = static_cast<const float*>(s->lnp[k][1]);
+    ColSegments sg{};
+    sg.seg[0] = {l2, G[10], ln2_parts, H};
+    sg.seg[1] = {l2 + (size_t)ln2_parts * H, G[11], ln2_parts, H};
+    sg.seg[2] = {l2 + 2 * (size_t)ln2_parts * H, G[9], ln2_parts, H};
+    sg.seg[3] = {l1, G[4], ln1_parts, H};
+    sg.seg[4] = {l1 + (size_t)ln1_parts * H, G[5], ln1_parts, H};
+    sg.seg[5] = {l1 + 2 * (size_t)ln1_parts * H, G[3], ln1_parts, H};
+    sg.seg[6] = {s->db1p[k], G[7], db1_rows, F};
+    sg.seg[7] = {s->qkvp[k], G[1], qkv_rows, 3 * H};
+    sg.n = 8;
+    Timed t(s, sw, P_COLSUM, 0,
+            4.0 * (3.0 * (ln2_parts + ln1_parts) * H + (double)db1_rows * F + qkv_rows * 3.0 * H));
+    SKY_TRY(reduce_column_segments(sg, sw));
+    if (two) {
+      SKY_CUDA(cudaEventRecord(s->ev_red[k], sw));
+      s->ev_red_live[k] = true;
+    }
   } else {  // dbqkv = column sums of dQKV
     Timed t(s, sw, P_COLSUM, 0, e * T * 3.0 * H);
     SKY_TRY(column_sum(s->dqkv, T, 3 * H, dt, G[1], s->ws, s->ws_bytes, sw));
@@ -569,6 +592,7 @@ sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
     return SKY_OK;
   };
   for (bool& live : s->ev_out_live) live = false;
+  for (bool& live : s->ev_red_live) live = false;
   if (sw != st) {  // the side stream starts after everything before this call
     SKY_CUDA(cudaEventRecord(s->ev_join, st));
     SKY_CUDA(cudaStreamWaitEvent(sw, s->ev_join, 0));
@@ -699,7 +723,7 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   // db1p | qkvp | status | x32 (bf16)
   const size_t wk = (bf ? 7 : 6) * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
                     align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes +
-                    s->ws2_bytes + 2 * s->lnp_bytes + s->db1p_bytes + s->qkvp_bytes + 256 +
+                    s->ws2_bytes + 4 * s->lnp_bytes + 2 * s->db1p_bytes + 2 * s->qkvp_bytes + 256 +
                     (s->n_slots > 1 ? gb : 0);  // gradient-accumulation scratch (one layer)
   s->ws_bytes_total = wk;
   *total = s->param_bytes + s->grad_bytes + s->stash_bytes + wk;
@@ -811,12 +835,14 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   s->delta = static_cast<float*>(take(lse_b));
   s->ws = take(s->ws_bytes);
   if (s->ws2_bytes) s->ws2 = take(s->ws2_bytes);
-  if (s->lnp_bytes) {
-    s->lnp[0] = take(s->lnp_bytes);
-    s->lnp[1] = take(s->lnp_bytes);
+  for (int k = 0; k < 2; ++k) {
+    if (s->lnp_bytes) {
+      s->lnp[k][0] = take(s->lnp_bytes);
+      s->lnp[k][1] = take(s->lnp_bytes);
+    }
+    if (s->db1p_bytes) s->db1p[k] = static_cast<float*>(take(s->db1p_bytes));
+    if (s->qkvp_bytes) s->qkvp[k] = static_cast<float*>(take(s->qkvp_bytes));
   }
-  if (s->db1p_bytes) s->db1p = static_cast<float*>(take(s->db1p_bytes));
-  if (s->qkvp_bytes) s->qkvp = static_cast<float*>(take(s->qkvp_bytes));
   s->d_status = static_cast<int32_t*>(take(4));
   if (bf) s->x32 = static_cast<float*>(take(t32));
   // further stash slots (parameters and gradients are shared), and the
@@ -837,6 +863,8 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
       ok = cudaEventCreateWithFlags(&s->ev_in[j], cudaEventDisableTiming) == cudaSuccess &&
            cudaEventCreateWithFlags(&s->ev_out[j], cudaEventDisableTiming) == cudaSuccess;
     if (ok) ok = cudaEventCreateWithFlags(&s->ev_join, cudaEventDisableTiming) == cudaSuccess;
+    for (int k = 0; k < 2 && ok; ++k)
+      ok = cudaEventCreateWithFlags(&s->ev_red[k], cudaEventDisableTiming) == cudaSuccess;
     if (!ok) {
       const cudaError_t ce = cudaGetLastError();
       sky_slice_destroy(s);
@@ -858,6 +886,8 @@ sky_status sky_slice_destroy(sky_slice* s) {
     if (s->ev_out[j]) cudaEventDestroy(s->ev_out[j]);
   }
   if (s->ev_join) cudaEventDestroy(s->ev_join);
+  for (int k = 0; k < 2; ++k)
+    if (s->ev_red[k]) cudaEventDestroy(s->ev_red[k]);
   if (s->step_exec) cudaGraphExecDestroy(s->step_exec);
   if (s->cap_stream) cudaStreamDestroy(s->cap_stream);
   if (s->side) cudaStreamDestroy(s->side);
