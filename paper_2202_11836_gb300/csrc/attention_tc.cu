@@ -39,7 +39,9 @@ namespace attn_tc {
 constexpr int BQ = 128, BKV = 64, HD = 64;
 constexpr int Q_BYTES = BQ * HD * 2;    // 16 KiB
 constexpr int KV_BYTES = BKV * HD * 2;  // 8 KiB per K or V tile
-constexpr int NTHR = 192;               // warp 0 TMA, warp 1 MMA, warps 2..5 softmax
+// forward CTA: warp 0 TMA and O += P V issue, warp 1 S = Q K^T issue,
+// warps 2..5 softmax
+constexpr int NTHR = 192;
 constexpr int STAGES = 2;               // dK/dV operand ring
 // The backward kernels run eight softmax warps: warps w and w + 4 share TMEM
 // lane quarter w % 4 and take the low / high 32 columns of each 64-wide tile.
@@ -88,10 +90,11 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
   uint64_t* kv_full = q_full + 1;
   uint64_t* kv_empty = kv_full + F_STAGES;
   uint64_t* s_full = kv_empty + F_STAGES;  // [2]
-  uint64_t* p_full = s_full + 2;           // [2]
+  uint64_t* s_free = s_full + 2;           // [2]
+  uint64_t* p_full = s_free + 2;           // [2]
   uint64_t* pv_done = p_full + 2;          // [2]
-  uint64_t* done = pv_done + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* done = pv_done + 2;            // [2], one per issuing warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 2);
 
   const int qt = blockIdx.x, a = blockIdx.y, b = blockIdx.z;
   const int S = p.S, H = p.H;
@@ -110,14 +113,16 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
     ptx::mbar_init(q_full, 1);
     for (int s = 0; s < F_STAGES; ++s) {
       ptx::mbar_init(&kv_full[s], 1);
-      ptx::mbar_init(&kv_empty[s], 1);
+      ptx::mbar_init(&kv_empty[s], 2);  // S_j has read K_j, P_j V_j has read V_j
     }
     for (int s = 0; s < 2; ++s) {
       ptx::mbar_init(&s_full[s], 1);
+      ptx::mbar_init(&s_free[s], 128);
       ptx::mbar_init(&p_full[s], 128);
       ptx::mbar_init(&pv_done[s], 1);
     }
-    ptx::mbar_init(done, 1);
+    ptx::mbar_init(&done[0], 1);
+    ptx::mbar_init(&done[1], 1);
     ptx::fence_mbar_init();
     ptx::fence_proxy_async_smem();
   }
@@ -132,64 +137,29 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
   const uint32_t tS = tmem, tO = tmem + 128, tP = tmem + 192;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ producer
+    // --------------------------------- producer and O += P V issue (warp 0)
+    // Loads Q and the first F_STAGES K/V tiles, then per tile j: issues
+    // O += P_j V_j once the softmax warps have written P_j, and refills the
+    // ring slot of tile j with tile j + F_STAGES once S_j and P_j V_j have
+    // read it.  (Two threads issue this CTA's MMAs: one thread issues a
+    // tcgen05.mma only about every 100 cycles.)
     if (lane == 0) {
-      ptx::mbar_arrive_expect_tx(q_full, Q_BYTES);
-      ptx::tma_load_2d(smem + F_Q_OFF, &tmQ, q_full, a * HD, row0 + q0);
-      int issued = 0;
-      for (int j = 0; j < n_kt; ++j) {
+      constexpr uint32_t idO = ptx::idesc_bf16_f32(BQ, HD, false, true);
+      const uint32_t skv = ptx::smem_u32(smem + F_KV_OFF);
+      auto load_kv = [&](int j) {
         const int st = j % F_STAGES;
-        const uint32_t ph = (j / F_STAGES) & 1;
-        if (!ptx::mbar_wait(&kv_empty[st], ph ^ 1u, lim, p.status, kWaitHint)) break;
         uint8_t* kv = smem + F_KV_OFF + st * 2 * KV_BYTES;
         ptx::mbar_arrive_expect_tx(&kv_full[st], 2 * KV_BYTES);
         ptx::tma_load_2d(kv, &tmKV, &kv_full[st], H + a * HD, row0 + j * BKV);
         ptx::tma_load_2d(kv + KV_BYTES, &tmKV, &kv_full[st], 2 * H + a * HD, row0 + j * BKV);
-        ++issued;
-      }
-      // drain: bounded waits for the copies still in flight
-      ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint);
-      for (int j = issued - 1; j >= 0 && j >= issued - F_STAGES; --j)
-        ptx::mbar_wait(&kv_full[j % F_STAGES], (j / F_STAGES) & 1, lim, p.status, kWaitHint);
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------- MMA issue
-    if (lane == 0) {
-      constexpr uint32_t idS = ptx::idesc_bf16_f32(BQ, BKV, false, false);
-      constexpr uint32_t idO = ptx::idesc_bf16_f32(BQ, HD, false, true);
-      const uint32_t sq = ptx::smem_u32(smem + F_Q_OFF);
-      const uint32_t skv = ptx::smem_u32(smem + F_KV_OFF);
-      // S_j = Q K_j^T into S buffer j & 1 (K_j already landed)
-      auto mma_s = [&](int j) {
-        const uint32_t sk = skv + (j % F_STAGES) * 2 * KV_BYTES;
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          ptx::tc_mma_f16(tS + (j & 1) * BKV, ptx::smem_desc_sw128(sq + kk * 32, 16, 1024),
-                          ptx::smem_desc_sw128(sk + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
-        ptx::tc_commit(&s_full[j & 1]);
       };
-      auto wait_k = [&](int j) {
-        return ptx::mbar_wait(&kv_full[j % F_STAGES], (j / F_STAGES) & 1, lim, p.status, kWaitHint);
-      };
-      bool ok = ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint) && wait_k(0);
-      if (ok) {
-        ptx::tc_fence_after();
-        mma_s(0);
-      }
-      // S_{s_next} is due next; it goes in while the MMA thread waits for P,
-      // as soon as its K tile has landed
-      int s_next = 1;
-      bool s_done = n_kt <= 1;
-      for (int j = 0; j < n_kt && ok; ++j) {
-        auto s_ready = [&] {
-          return ptx::mbar_try_wait(&kv_full[s_next % F_STAGES], (s_next / F_STAGES) & 1);
-        };
-        auto s_issue = [&] {
-          ptx::tc_fence_after();
-          mma_s(s_next);
-        };
-        if (!ptx::mbar_wait_with(&p_full[j & 1], (j >> 1) & 1, lim, p.status, kWaitHint, s_done, s_ready,
-                                 s_issue))
+      ptx::mbar_arrive_expect_tx(q_full, Q_BYTES);
+      ptx::tma_load_2d(smem + F_Q_OFF, &tmQ, q_full, a * HD, row0 + q0);
+      int issued = 0;
+      for (; issued < n_kt && issued < F_STAGES; ++issued) load_kv(issued);
+      for (int j = 0; j < n_kt; ++j) {
+        if (!ptx::mbar_wait(&p_full[j & 1], (j >> 1) & 1, lim, p.status, kWaitHint)) break;
+        if (!ptx::mbar_wait(&kv_full[j % F_STAGES], (j / F_STAGES) & 1, lim, p.status, kWaitHint))
           break;
         ptx::tc_fence_after();
         const uint32_t sv = skv + (j % F_STAGES) * 2 * KV_BYTES + KV_BYTES;
@@ -200,17 +170,45 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
                                  idO, (j > 0 || kk > 0) ? 1u : 0u);
         ptx::tc_commit(&pv_done[j & 1]);
         ptx::tc_commit(&kv_empty[j % F_STAGES]);
-        if (!s_done) {  // S_{j+1} is needed before P_{j+1} can exist
-          if (!wait_k(s_next)) break;
-          s_issue();
+        if (issued < n_kt) {  // the slot of tile j takes tile j + F_STAGES
+          const int st = issued % F_STAGES;
+          if (!ptx::mbar_wait(&kv_empty[st], ((issued / F_STAGES) & 1) ^ 1u, lim, p.status, kWaitHint))
+            break;
+          load_kv(issued++);
         }
-        // the softmax warps have read S_j (they arrived on p_full[j & 1]
-        // after their TMEM loads), so its buffer takes S_{j+2}
-        s_next = j + 2;
-        s_done = s_next >= n_kt;
       }
-      ptx::tc_commit(done);
-      ptx::mbar_wait(done, 0, lim, p.status, kWaitHint);
+      ptx::tc_commit(&done[1]);
+      ptx::mbar_wait(&done[1], 0, lim, p.status, kWaitHint);
+      // drain: bounded waits for the copies still in flight
+      ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint);
+      for (int j = issued - 1; j >= 0 && j >= issued - F_STAGES; --j)
+        ptx::mbar_wait(&kv_full[j % F_STAGES], (j / F_STAGES) & 1, lim, p.status, kWaitHint);
+    }
+  } else if (warp == 1) {
+    // --------------------------------------------- S = Q K^T issue (warp 1)
+    // S_j goes into buffer j & 1 as soon as K_j has landed and the softmax
+    // warps hold S_{j-2} in registers (s_free)
+    if (lane == 0) {
+      constexpr uint32_t idS = ptx::idesc_bf16_f32(BQ, BKV, false, false);
+      const uint32_t sq = ptx::smem_u32(smem + F_Q_OFF);
+      const uint32_t skv = ptx::smem_u32(smem + F_KV_OFF);
+      bool ok = ptx::mbar_wait(q_full, 0, lim, p.status, kWaitHint);
+      for (int j = 0; j < n_kt && ok; ++j) {
+        if (j >= 2 && !ptx::mbar_wait(&s_free[j & 1], ((j - 2) >> 1) & 1, lim, p.status, kWaitHint))
+          break;
+        if (!ptx::mbar_wait(&kv_full[j % F_STAGES], (j / F_STAGES) & 1, lim, p.status, kWaitHint))
+          break;
+        ptx::tc_fence_after();
+        const uint32_t sk = skv + (j % F_STAGES) * 2 * KV_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          ptx::tc_mma_f16(tS + (j & 1) * BKV, ptx::smem_desc_sw128(sq + kk * 32, 16, 1024),
+                          ptx::smem_desc_sw128(sk + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
+        ptx::tc_commit(&s_full[j & 1]);
+        ptx::tc_commit(&kv_empty[j % F_STAGES]);
+      }
+      ptx::tc_commit(&done[0]);
+      ptx::mbar_wait(&done[0], 0, lim, p.status, kWaitHint);
     }
   } else {
     // --------------------------------------------------- softmax / epilogue
@@ -237,6 +235,9 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
         ptx::tmem_ld_32x32b_x32(tS + (j & 1) * BKV + lane_base + 32, v1);
       }
       ptx::tmem_ld_wait();
+      // S_j is in registers: its buffer may take S_{j+2}
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&s_free[j & 1]);
       const int kbase = j * BKV;
       if (kbase + BKV > len) {  // CTA-uniform: only the last tile holds masked keys
 #pragma unroll
