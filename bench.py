@@ -454,8 +454,9 @@ def run_gpu(args, w):
             "per_layer": {"ms": per_layer_ms, "lengths": "the workload's own (same mask as value)",
                           "pct_bf16_peak": round(100 * per_layer_flops / (per_layer_ms / 1e3)
                                                  / 1e12 / pk["bf16"], 2),
-                          "how": "sky_slice_layer_cost: median over layers of fwd+bwd, CUDA "
-                                 "events per layer, weight-gradient stream joined per layer"},
+                          "how": "sky_slice_layer_cost: median over layers of fwd+bwd; CUDA "
+                                 "events per layer, captured with one pass into a graph and "
+                                 "replayed (per-layer times add up to the pass)"},
             "allocation": allocation_plan(rec),
             "optimizer": optimizer,
             "valid_tokens_per_s": world * int(np.sum(lens)) * args.steps / (ms / 1e3),

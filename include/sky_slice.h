@@ -210,21 +210,24 @@ sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_
 sky_status sky_slice_step_graph_launch(sky_slice* s, void* stream);
 
 /* Measures every layer of the slice (the per-layer benchmark of Sec. IV-B):
- * runs 2 warm-up and `iters` timed forward+backward passes at [B,S] on a
- * fixed input pattern written on the device (parameters as set), records CUDA
- * events around each layer on a stream of its own, and writes the median
- * per-layer times with the analytic FLOPs and the byte counts.
+ * on a fixed input pattern written on the device (parameters as set), runs
+ * 2 forward+backward passes at [B,S] directly, then captures one pass with a
+ * CUDA event around each layer into a CUDA graph on a stream of its own and
+ * replays it 1 + `iters` times (as a step is replayed), and writes the
+ * median per-layer times of the last `iters` replays with the analytic FLOPs
+ * and the byte counts.
  * lens: host int32[B], the valid length of every sequence (each in [1,S]),
  * so that a workload's own padding mask is measured; NULL measures
  * full-length sequences.  fwd_flops / bwd_flops count attention over those
- * lengths.  The weight-gradient stream joins after every layer, so a layer's
- * time includes its own weight gradients (a whole step overlaps them with the
- * next layer's data gradients, so the per-layer sum is an upper bound on the
- * step).  Before it starts, the call waits for all work already enqueued on
+ * lengths.  The layers are timed inside whole forward + backward passes, as a
+ * step runs them: a layer's weight gradients, which run on a second stream,
+ * overlap the next layer's interval, and the slice's first layer takes the
+ * final join, so the per-layer times add up to the passes' time.  Before it
+ * starts, the call waits for all work already enqueued on
  * this slice (its last stream and its weight-gradient stream), because the
  * measurement reuses the slice's stash and workspace.  It allocates its
  * input, output and length buffers (cudaMalloc) and a stream, and frees them
- * on every return path.  n_out must equal layer_end - layer_begin.
+ * and its graph on every return path.  n_out must equal layer_end - layer_begin.
  * Synchronous; overwrites grads, and a following sky_slice_backward needs a
  * new forward (STATE).  Errors: INVALID_ARG (null out, n_out, B or S outside
  * [1, max], iters < 1, a length outside [1,S]), OOM / CUDA (buffers). */

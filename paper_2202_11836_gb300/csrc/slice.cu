@@ -183,6 +183,8 @@ struct sky_slice {
   // gradients on the weight-gradient stream (one layer's worth, reused)
   float* gscr[SKY_NUM_PARAMS] = {};
   bool accumulate = false;
+  // layer_cost: per-layer marks are being captured into a graph
+  bool marks_in_graph = false;
   // batch shape and lengths of the pass in progress (the slot in use)
   int B = 0, S = 0;
   const int32_t* d_len = nullptr;
@@ -543,6 +545,16 @@ sky_status backward_layer(sky_slice* s, int i, const void* dY, sky_dtype dy_dt, 
   return SKY_OK;
 }
 
+// A per-layer timing mark.  Inside a stream capture it becomes an event
+// record node that a replay of the graph records.
+sky_status record_mark(sky_slice* s, cudaEvent_t ev, cudaStream_t st) {
+  if (s->marks_in_graph)
+    SKY_CUDA(cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal));
+  else
+    SKY_CUDA(cudaEventRecord(ev, st));
+  return SKY_OK;
+}
+
 sky_status forward_all(sky_slice* s, const void* x, void* y, cudaStream_t st,
                        std::vector<cudaEvent_t>* marks) {
   const int64_t n = (int64_t)s->B * s->S * s->H;
@@ -568,9 +580,9 @@ sky_status forward_all(sky_slice* s, const void* x, void* y, cudaStream_t st,
     }
   }
   for (int i = 0; i < s->L; ++i) {
-    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i], st));
+    if (marks) SKY_TRY(record_mark(s, (*marks)[2 * i], st));
     SKY_TRY(forward_layer(s, i, i + 1 < s->L ? nullptr : y, st));
-    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
+    if (marks) SKY_TRY(record_mark(s, (*marks)[2 * i + 1], st));
   }
   return SKY_OK;
 }
@@ -581,8 +593,7 @@ sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
   const float* cur2 = nullptr;
   sky_dtype cur_dt = s->cfg.io_fp32 ? SKY_DTYPE_FP32 : s->cfg.dtype;
   // The side stream is used unless kernels are being timed one by one.  It
-  // joins the caller's stream at the end (and after every layer when the
-  // per-layer cost is being measured), so the caller's stream still orders
+  // joins the caller's stream at the end, so the caller's stream still orders
   // everything the backward pass does.
   cudaStream_t sw = (s->side && !s->prof) ? s->side : st;
   auto join = [&]() -> sky_status {
@@ -599,15 +610,19 @@ sky_status backward_all(sky_slice* s, const void* dy, void* dx, cudaStream_t st,
   }
   for (int i = s->L - 1; i >= 0; --i) {
     const int k = (s->L - 1 - i) & 1;
-    if (marks) SKY_CUDA(cudaEventRecord((*marks)[2 * i], st));
+    if (marks) SKY_TRY(record_mark(s, (*marks)[2 * i], st));
     const sky_status rc = backward_layer(s, i, cur, cur_dt, cur2, k, i == 0 ? dx : nullptr, st, sw);
     if (rc != SKY_OK) {
       join();
       return rc;
     }
     if (marks) {
-      SKY_TRY(join());
-      SKY_CUDA(cudaEventRecord((*marks)[2 * i + 1], st));
+      // per-layer marks on the caller's stream only: a layer's weight
+      // gradients on the second stream overlap the next layer's interval, as
+      // in a step, and the slice's first layer (the last one here) takes the
+      // final join, so the per-layer times add up to the backward pass
+      if (i == 0) SKY_TRY(join());
+      SKY_TRY(record_mark(s, (*marks)[2 * i + 1], st));
     }
     cur = s->dP[k];
     cur2 = s->cfg.dtype == SKY_DTYPE_BF16 ? nullptr : s->dR[k];  // bf16: already in dP[k]
@@ -1100,8 +1115,10 @@ struct CostScratch {
   int32_t* len = nullptr;
   cudaStream_t st = nullptr;
   std::vector<cudaEvent_t> ev;
+  cudaGraphExec_t exec = nullptr;
   ~CostScratch() {
     if (st) cudaStreamSynchronize(st);
+    if (exec) cudaGraphExecDestroy(exec);
     for (auto e : ev)
       if (e) cudaEventDestroy(e);
     if (st) cudaStreamDestroy(st);
@@ -1159,13 +1176,45 @@ sky_status sky_slice_layer_cost(sky_slice* s, int32_t B, int32_t S, const int32_
   const bool prof = s->prof;
   s->prof = false;
   sky_status rc = SKY_OK;
-  const int warm = 2;
-  for (int it = 0; it < warm + iters && rc == SKY_OK; ++it) {
+  // two direct passes (one-time set-up happens outside any capture), then
+  // one forward + backward with per-layer marks captured as a graph and
+  // replayed, as a step is
+  for (int it = 0; it < 2 && rc == SKY_OK; ++it) {
+    rc = forward_all(s, cs.x, cs.y, st, nullptr);
+    if (rc == SKY_OK) rc = backward_all(s, cs.dy, cs.dx, st, nullptr);
+    if (rc == SKY_OK && cudaStreamSynchronize(st) != cudaSuccess)
+      rc = cuda_fail(cudaGetLastError(), "sync");
+  }
+  if (rc == SKY_OK) {
+    if (cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+      rc = cuda_fail(cudaGetLastError(), "layer-cost capture");
+  }
+  int64_t captured = 0;
+  if (rc == SKY_OK) {
+    const int64_t n0 = sky_launch_count();
+    s->marks_in_graph = true;
     rc = forward_all(s, cs.x, cs.y, st, &fm);
     if (rc == SKY_OK) rc = backward_all(s, cs.dy, cs.dx, st, &bm);
-    if (rc != SKY_OK) break;
-    if (cudaStreamSynchronize(st) != cudaSuccess) { rc = cuda_fail(cudaGetLastError(), "sync"); break; }
-    if (it < warm) continue;
+    s->marks_in_graph = false;
+    // the captured launches ran nothing yet: they are counted at every replay
+    captured = sky_launch_count() - n0;
+    count_launches(-static_cast<int>(captured));
+    cudaGraph_t graph = nullptr;
+    const cudaError_t ec = cudaStreamEndCapture(st, &graph);
+    if (rc == SKY_OK && ec != cudaSuccess) rc = cuda_fail(ec, "layer-cost capture");
+    if (rc == SKY_OK) {
+      const cudaError_t ei = cudaGraphInstantiate(&cs.exec, graph, 0);
+      if (ei != cudaSuccess) rc = cuda_fail(ei, "layer-cost graph instantiate");
+    }
+    if (graph) cudaGraphDestroy(graph);
+  }
+  for (int it = 0; it < 1 + iters && rc == SKY_OK; ++it) {
+    if (cudaGraphLaunch(cs.exec, st) != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess) {
+      rc = cuda_fail(cudaGetLastError(), "layer-cost replay");
+      break;
+    }
+    count_launches(static_cast<int>(captured));
+    if (it < 1) continue;
     for (int i = 0; i < s->L; ++i) {
       float a = 0, b = 0;
       cudaEventElapsedTime(&a, fm[2 * i], fm[2 * i + 1]);
