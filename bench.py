@@ -368,9 +368,13 @@ def run_gpu(args, w):
     gemm_flops, attn_flops = algorithmic_flops(w, lens)
     pk = peaks()
 
-    # 2. per-kernel CUDA-event timing of the same steps (roofline of the dominant kernel)
+    # 2. per-kernel CUDA-event timing of the same steps (roofline of the
+    # dominant kernel): every kernel in line on the caller's stream between a
+    # pair of events.  (The same timers captured into the step graph and
+    # replayed, sky_slice_step_graph_create with profiling on, read about 2%
+    # slower per GEMM: the event nodes serialise the graph as well.)
     s.set_profiling(True)
-    ms_prof = timed_region(step, max(3, args.steps // 4), 1, sync, barrier, reduce_max, start, stop)
+    timed_region(step, max(3, args.steps // 4), 1, sync, barrier, reduce_max, start, stop)
     stats = s.kernel_stats()
     s.set_profiling(False)
     gemm_ms = sum(v["total_ms"] for k, v in stats.items() if k.startswith("gemm"))
@@ -473,7 +477,9 @@ def run_gpu(args, w):
                          "peak_source": pk["source"] + " (burst bf16: the per-kernel region is "
                                                        "a few steps long; sustained also given)",
                          "traffic": gemm_traffic(w.name), "traffic_unit": "bytes per launch",
-                         "launches": gemm_n},
+                         "launches": gemm_n,
+                         "timing": "CUDA events around every launch, all kernels in line on "
+                                   "the caller's stream"},
             "kernels": kernel_table,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,

@@ -199,11 +199,14 @@ sky_status sky_device_delay(uint64_t ns, void* stream);
  * between launches and keeps all five buffers alive while the graph exists.
  * Replays on one slice must not overlap each other or direct calls on that
  * slice (they share its stash and workspace).  Launches are counted in
- * sky_launch_count at every replay; per-kernel timing does not see them.
- * The graph is freed by the next create and by sky_slice_destroy.
- * Errors: those of sky_slice_forward / sky_slice_backward; STATE if
- * per-kernel timing is on (create) or no graph exists (launch); CUDA if the
- * capture or instantiation fails. */
+ * sky_launch_count at every replay.  With per-kernel timing on at create
+ * (sky_slice_set_profiling), every kernel runs in line on one stream with a
+ * pair of CUDA events around it captured into the graph; each launch of such
+ * a graph then synchronises `stream` and adds the replay's per-kernel times
+ * to the records of sky_slice_kernel_stats (kernel times without host launch
+ * gaps).  The graph is freed by the next create and by sky_slice_destroy.
+ * Errors: those of sky_slice_forward / sky_slice_backward; STATE if no graph
+ * exists (launch); CUDA if the capture or instantiation fails. */
 sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_t* d_len,
                                        int32_t B, int32_t S, void* y, const void* dy, void* dx,
                                        void* stream);

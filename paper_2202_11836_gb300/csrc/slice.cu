@@ -183,8 +183,12 @@ struct sky_slice {
   // gradients on the weight-gradient stream (one layer's worth, reused)
   float* gscr[SKY_NUM_PARAMS] = {};
   bool accumulate = false;
-  // layer_cost: per-layer marks are being captured into a graph
+  // layer_cost / profiled step graph: timing events are being captured
   bool marks_in_graph = false;
+  // per-kernel records of a step graph captured with profiling on, and the
+  // events they use (taken out of the pool, owned until the graph goes)
+  std::vector<sky::ProfRecord> graph_recs;
+  std::vector<cudaEvent_t> graph_events;
   // batch shape and lengths of the pass in progress (the slot in use)
   int B = 0, S = 0;
   const int32_t* d_len = nullptr;
@@ -272,12 +276,18 @@ struct Timed {
     r.cat = cat; r.flops = flops; r.bytes = bytes;
     r.start = next_event(s);
     r.stop = next_event(s);
-    if (r.start) cudaEventRecord(r.start, st);
+    if (r.start) record(r.start);
   }
   ~Timed() {
     if (!s->prof || !r.start || !r.stop) return;
-    cudaEventRecord(r.stop, st);
+    record(r.stop);
     s->recs.push_back(r);
+  }
+  // inside a stream capture the records become event record nodes that every
+  // replay of the graph records
+  void record(cudaEvent_t e) {
+    if (s->marks_in_graph) cudaEventRecordWithFlags(e, st, cudaEventRecordExternal);
+    else cudaEventRecord(e, st);
   }
 };
 
@@ -895,7 +905,11 @@ sky_status sky_slice_destroy(sky_slice* s) {
   ABI_GUARD_BEGIN
   if (!s) return SKY_OK;
   cudaDeviceSynchronize();
+  // the graph first: its nodes use the slice's events
+  if (s->step_exec) cudaGraphExecDestroy(s->step_exec);
+  s->step_exec = nullptr;
   for (auto e : s->event_pool) cudaEventDestroy(e);
+  for (auto e : s->graph_events) cudaEventDestroy(e);
   for (int j = 0; j < 4; ++j) {
     if (s->ev_in[j]) cudaEventDestroy(s->ev_in[j]);
     if (s->ev_out[j]) cudaEventDestroy(s->ev_out[j]);
@@ -903,7 +917,6 @@ sky_status sky_slice_destroy(sky_slice* s) {
   if (s->ev_join) cudaEventDestroy(s->ev_join);
   for (int k = 0; k < 2; ++k)
     if (s->ev_red[k]) cudaEventDestroy(s->ev_red[k]);
-  if (s->step_exec) cudaGraphExecDestroy(s->step_exec);
   if (s->cap_stream) cudaStreamDestroy(s->cap_stream);
   if (s->side) cudaStreamDestroy(s->side);
   if (s->opt_mem) cudaFree(s->opt_mem);
@@ -1051,7 +1064,6 @@ sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_
                                        void* stream) {
   ABI_GUARD_BEGIN
   SKY_CHECK(s, SKY_ERR_INVALID_ARG, "null handle");
-  SKY_CHECK(!s->prof, SKY_ERR_STATE, "per-kernel timing is on; a step graph holds no timers");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   // One step in the ordinary way first: it checks every argument, and any
   // one-time set-up (kernel attributes, occupancy queries) happens outside
@@ -1063,14 +1075,28 @@ sky_status sky_slice_step_graph_create(sky_slice* s, const void* x, const int32_
     SKY_CUDA(cudaGraphExecDestroy(s->step_exec));
     s->step_exec = nullptr;
   }
+  for (auto e : s->graph_events) cudaEventDestroy(e);
+  s->graph_events.clear();
+  s->graph_recs.clear();
+  // the direct step's per-kernel records are not kept
+  s->recs.clear();
+  s->event_next = 0;
   if (!s->cap_stream) SKY_CUDA(cudaStreamCreateWithFlags(&s->cap_stream, cudaStreamNonBlocking));
   cudaStream_t cs = s->cap_stream;
   const int64_t n0 = sky_launch_count();
   SKY_CUDA(cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal));
   s->layers = s->slot_layers[0];
   s->B = B; s->S = S; s->d_len = d_len;
+  s->marks_in_graph = s->prof;
   sky_status rc = forward_all(s, x, y, cs, nullptr);
   if (rc == SKY_OK) rc = backward_all(s, dy, dx, cs, nullptr);
+  s->marks_in_graph = false;
+  if (s->prof) {  // the captured timers now belong to the graph
+    s->graph_recs.swap(s->recs);
+    s->graph_events.assign(s->event_pool.begin(), s->event_pool.begin() + s->event_next);
+    s->event_pool.erase(s->event_pool.begin(), s->event_pool.begin() + s->event_next);
+    s->event_next = 0;
+  }
   cudaGraph_t graph = nullptr;
   const cudaError_t ec = cudaStreamEndCapture(cs, &graph);
   if (rc != SKY_OK) {
@@ -1100,6 +1126,18 @@ sky_status sky_slice_step_graph_launch(sky_slice* s, void* stream) {
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   SKY_CUDA(cudaGraphLaunch(s->step_exec, st));
   count_launches(static_cast<int>(s->step_launches));
+  if (s->prof && !s->graph_recs.empty()) {
+    // a step graph captured with per-kernel timing: add this replay's times
+    SKY_CUDA(cudaStreamSynchronize(st));
+    for (const auto& r : s->graph_recs) {
+      float ms = 0;
+      SKY_CUDA(cudaEventElapsedTime(&ms, r.start, r.stop));
+      s->cat_ms[r.cat] += ms;
+      s->cat_flops[r.cat] += r.flops;
+      s->cat_bytes[r.cat] += r.bytes;
+      s->cat_n[r.cat] += 1;
+    }
+  }
   s->B = s->step_B; s->S = s->step_S; s->d_len = s->step_len;
   s->last_stream = st;
   s->slot_fwd[0] = 1;
