@@ -83,7 +83,9 @@ sky_status sky_attention_fwd(const void* qkv, const int32_t* d_len, int32_t B, i
                              int32_t H, int32_t A, sky_dtype dtype, void* ctx, float* lse,
                              int32_t* d_status, void* stream);
 
-/* Scratch bytes of sky_attention_bwd (the per-row dot(dctx, ctx) terms). */
+/* Scratch bytes of sky_attention_bwd: the per-row terms dot(dctx, ctx) and,
+ * for bf16, 32 bytes per (row, head) of per-query MMA operand rows.  The
+ * workspace must be 16-byte aligned. */
 size_t sky_attention_bwd_workspace_bytes(int32_t B, int32_t S, int32_t H, int32_t A);
 
 /* Attention backward: from dctx [B*S, H] and the forward's qkv, ctx and lse,

@@ -25,9 +25,14 @@ using bf16 = __nv_bfloat16;
 // load of the row is issued before the first product (more bytes in flight
 // per warp); NV == 0: any H that is a multiple of 64, one group at a time.
 // Requires D == 64.
+// Beside delta it writes the per-query terms the tensor-core dK/dV kernel
+// adds inside its score products: xtab[(b*A + a)*2 + 0][s] = lse2 / c and
+// xtab[(b*A + a)*2 + 1][s] = delta (c = log2(e)/sqrt(D)), each negated and
+// split into a bf16 high and low part, as 16-byte rows [hi, lo, 0 x 6].
 template <int NV>
 __global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __restrict__ dctx, int S,
-                                int H, int A, int64_t rows, float* __restrict__ delta) {
+                                int H, int A, int64_t rows, float* __restrict__ delta,
+                                const float* __restrict__ lse, uint4* __restrict__ xtab) {
   pdl_trigger();
   pdl_wait();
   const int64_t row = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
@@ -49,7 +54,20 @@ __global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __rest
     acc += __shfl_xor_sync(0xffffffffu, acc, 1);
     acc += __shfl_xor_sync(0xffffffffu, acc, 2);
     acc += __shfl_xor_sync(0xffffffffu, acc, 4);
-    if ((l & 7) == 0 && col < H) delta[(b * A + col / HD) * S + s] = acc;
+    if ((l & 7) == 0 && col < H) {
+      const int64_t bh = b * A + col / HD;
+      delta[bh * S + s] = acc;
+      auto row16 = [](float x) {  // -x as [hi, lo, 0, ...] in bf16
+        const bf16 hi = __float2bfloat16_rn(-x);
+        const bf16 lo = __float2bfloat16_rn(-x - __bfloat162float(hi));
+        return make_uint4(static_cast<uint32_t>(__bfloat16_as_ushort(hi)) |
+                              (static_cast<uint32_t>(__bfloat16_as_ushort(lo)) << 16),
+                          0u, 0u, 0u);
+      };
+      constexpr float kC = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
+      xtab[(bh * 2) * S + s] = row16(__fdiv_rn(lse[bh * S + s], kC));
+      xtab[(bh * 2 + 1) * S + s] = row16(acc);
+    }
   };
   if constexpr (NV > 0) {
     uint4 x[NV], y[NV];
@@ -212,7 +230,7 @@ sky_status attention_fwd_tc(const void* qkv, const int32_t* lens, int B, int S, 
                             cudaStream_t stream);
 
 sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse, const float* delta,
-                            const int32_t* lens, int B, int S, int H, int A, void* dqkv,
+                            const uint4* xtab, const int32_t* lens, int B, int S, int H, int A, void* dqkv,
                             int32_t* status, uint64_t timeout_ns, cudaStream_t stream,
                             float* colpart);
 
@@ -238,7 +256,10 @@ sky_status attention_fwd(const void* qkv, const int32_t* lens, int B, int S, int
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "attention forward launch");
 }
 
-size_t attention_bwd_ws(int B, int S, int A) { return (size_t)B * A * S * sizeof(float); }
+// delta [B][A][S] floats, then (bf16 path) the dK/dV kernel's per-query rows
+// [B][A][2][S] x 16 bytes, 16-byte aligned.
+static size_t delta_bytes(int B, int S, int A) { return ((size_t)B * A * S * sizeof(float) + 15) & ~(size_t)15; }
+size_t attention_bwd_ws(int B, int S, int A) { return delta_bytes(B, S, A) + (size_t)B * A * 2 * S * 16; }
 
 sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, const float* lse,
                          const int32_t* lens, int B, int S, int H, int A, sky_dtype dt, void* dqkv,
@@ -251,16 +272,17 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
     const auto* c = static_cast<const __nv_bfloat16*>(ctx);
     const auto* dc = static_cast<const __nv_bfloat16*>(dctx);
     const dim3 g(ceil_div(rows * 32, 256)), blk(256);
+    uint4* xtab = reinterpret_cast<uint4*>(reinterpret_cast<char*>(delta) + delta_bytes(B, S, A));
     cudaError_t le;
     switch (H % 256 == 0 ? H / 256 : 0) {
-      case 3: le = launch_pdl(attn::attn_delta_bf16<3>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
-      case 4: le = launch_pdl(attn::attn_delta_bf16<4>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
-      case 8: le = launch_pdl(attn::attn_delta_bf16<8>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
-      default: le = launch_pdl(attn::attn_delta_bf16<0>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta); break;
+      case 3: le = launch_pdl(attn::attn_delta_bf16<3>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta, lse, xtab); break;
+      case 4: le = launch_pdl(attn::attn_delta_bf16<4>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta, lse, xtab); break;
+      case 8: le = launch_pdl(attn::attn_delta_bf16<8>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta, lse, xtab); break;
+      default: le = launch_pdl(attn::attn_delta_bf16<0>, g, blk, 0, stream, 1, c, dc, S, H, A, rows, delta, lse, xtab); break;
     }
     count_launches(1);
     if (le != cudaSuccess) return cuda_fail(le, "attention delta launch");
-    return attention_bwd_tc(qkv, dctx, lse, delta, lens, B, S, H, A, dqkv, status, 2000000000ull,
+    return attention_bwd_tc(qkv, dctx, lse, delta, xtab, lens, B, S, H, A, dqkv, status, 2000000000ull,
                             stream, colpart);
   } else {
     SKY_CHECK(D <= 128, SKY_ERR_UNSUPPORTED, "fp32 attention needs head dim <= 128");

@@ -42,7 +42,6 @@ constexpr int KV_BYTES = BKV * HD * 2;  // 8 KiB per K or V tile
 // forward CTA: warp 0 TMA and O += P V issue, warp 1 S = Q K^T issue,
 // warps 2..5 softmax
 constexpr int NTHR = 192;
-constexpr int STAGES = 2;               // dK/dV operand ring
 // The backward kernels run eight softmax warps: warps w and w + 4 share TMEM
 // lane quarter w % 4 and take the low / high 32 columns of each 64-wide tile.
 constexpr int NSM_B = 256;              // softmax threads in the backward kernels
@@ -346,10 +345,10 @@ constexpr int DQ_SMEM = DQ_BAR_OFF + 256 + 1024;
 
 struct BwdParams {
   int S, H, A;
-  int lse_bulk;  // lse / delta rows may be bulk-copied: S % 4 == 0, 16-byte aligned bases
   const int32_t* lens;
   const float* lse;
   const float* delta;
+  const uint4* xtab;  // dK/dV per-query rows: [B*A][2][S] x 16 bytes (attn_delta_bf16)
   __nv_bfloat16* dqkv;
   // optional: column sums of the stored dQKV, one row per 128-row tile of a
   // sequence: colpart[b * ceil(S/128) + tile][3H]
@@ -623,24 +622,48 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
 // One CTA per 128 keys of (b, a) (tiles at or past len[b] only write zeros);
 // per 64-query tile i over all S queries:
 //   S^T = K Q_i^T, dP^T = V dO_i^T (TMEM); thread = key row:
-//   P^T = exp2(S^T log2(e)/sqrt(D) - lse2_q), dS^T = P^T (dP^T - delta_q) -> smem
-//   dV += P^T dO_i, dK += dS^T Q_i (TMEM); finally dK / sqrt(D), dV -> dQKV.
+//   P^T = exp2(S^T log2(e)/sqrt(D) - lse2_q), dS^T = P^T (dP^T - delta_q),
+//   written back to TMEM over the S^T / dP^T columns they came from;
+//   dV += P^T dO_i, dK += dS^T Q_i with P^T, dS^T as TMEM A operands;
+//   finally dK / sqrt(D), dV -> dQKV.
+// Keeping P^T and dS^T in TMEM takes their 32 KiB of shared-memory stores and
+// the accumulating products' 32 KiB of A-operand reads off the shared-memory
+// port per tile, which the score products' operand reads otherwise saturate.
+// The price is order within a CTA: S^T_{i+1} waits until dV_i has read P^T_i
+// (and dP^T_{i+1} until dK_i has read dS^T_i), so the two CTAs on an SM take
+// turns on the tensor pipe rather than one CTA overlapping itself.
 // The Q_i / dO_i tiles serve both as K-major operands (S^T, dP^T) and as
-// MN-major operands (dK, dV).  As in the dQ kernel, S^T / dP^T are released
-// (s_free) as soon as the softmax warps hold them in registers, so the next
-// tile's S^T, dP^T products overlap the forming of P^T and dS^T.
+// MN-major operands (dK, dV).
 constexpr int BK2 = 128, BQ2 = 64;
 constexpr int KV2_BYTES = BK2 * HD * 2;    // 16 KiB (K or V of 128 keys)
 constexpr int QO2_BYTES = BQ2 * HD * 2;    // 8 KiB  (Q or dO of 64 queries)
-constexpr int PS2_BYTES = BK2 * BQ2 * 2;   // 16 KiB (P^T or dS^T)
+constexpr int KV_STAGES = 3;               // Q / dO ring
 constexpr int KV_K_OFF = 0, KV_V_OFF = KV2_BYTES;
 constexpr int KV_Q_OFF = 2 * KV2_BYTES;
-constexpr int KV_O_OFF = KV_Q_OFF + STAGES * QO2_BYTES;
-constexpr int KV_P_OFF = KV_O_OFF + STAGES * QO2_BYTES;
-constexpr int KV_DS_OFF = KV_P_OFF + PS2_BYTES;
-constexpr int KV_LD_OFF = KV_DS_OFF + PS2_BYTES;   // [STAGES][2][64] floats: lse, delta
-constexpr int KV_BAR_OFF = KV_LD_OFF + STAGES * 2 * BQ2 * 4;
+constexpr int KV_O_OFF = KV_Q_OFF + KV_STAGES * QO2_BYTES;
+// The per-query terms enter the score products as one more K = 16 step:
+// S^T - lse2 / c = [K | E] [Q | X_lse]^T and dP^T - delta = [V | E] [dO | X_delta]^T,
+// with c = log2(e)/sqrt(D), E the 128 x 16 matrix whose first two columns are
+// ones, and X the 64 x 16 per-tile matrix whose first two columns hold the
+// negated term split into a bf16 high part and a bf16 low part (exact to
+// about 2^-17 relative).  The softmax threads then need no per-query loads.
+// E and X are K-major without swizzling, built from 8-row x 16-byte core
+// matrices: a row's K columns 0..7 are 16 contiguous bytes (row groups 128
+// bytes apart), and columns 8..15, all zero, come from one shared zero block
+// (the descriptors' K-direction offset points there).  So an X tile is 64
+// rows of 16 bytes, one bulk copy of the table the delta pre-pass writes.
+constexpr int XROW_BYTES = 16;
+constexpr int X_BYTES = BQ2 * XROW_BYTES;                      // 1 KiB: X of one product
+constexpr int KV_E_OFF = KV_O_OFF + KV_STAGES * QO2_BYTES;     // E: 2 KiB
+constexpr int KV_X_OFF = KV_E_OFF + BK2 * XROW_BYTES;          // [KV_STAGES][2 products] X
+constexpr int KV_Z_OFF = KV_X_OFF + KV_STAGES * 2 * X_BYTES;   // zeros: 2 KiB
+constexpr int KV_RED_OFF = KV_Z_OFF + BK2 * XROW_BYTES;  // [2 halves][4 quarters][64] floats
+constexpr int KV_BAR_OFF = KV_RED_OFF + 2 * 4 * 64 * 4;
+// 91 KiB: more than a third of the SM's shared memory, so at most two CTAs
+// share an SM, as their 256 TMEM columns each require.
 constexpr int KV_SMEM = KV_BAR_OFF + 128 + 1024;
+static_assert(3 * (KV_SMEM + 1024) > 233472 && 2 * (KV_SMEM + 1024) <= 233472,
+              "exactly two dK/dV CTAs per SM");
 
 __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtensorMap tmK,
                                                             const __grid_constant__ CUtensorMap tmQ,
@@ -678,29 +701,30 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
   }
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
-  float* ldst = reinterpret_cast<float*>(smem + KV_LD_OFF);
   uint64_t* kv_full = reinterpret_cast<uint64_t*>(smem + KV_BAR_OFF);
   uint64_t* q_full = kv_full + 1;
-  uint64_t* q_empty = q_full + STAGES;
-  uint64_t* s_full = q_empty + STAGES;
-  uint64_t* s_free = s_full + 1;
-  uint64_t* pds_full = s_free + 1;
-  uint64_t* mm_done = pds_full + 1;
-  uint64_t* done = mm_done + 1;  // [2], one per issuing warp
+  uint64_t* q_empty = q_full + KV_STAGES;
+  uint64_t* st_full = q_empty + KV_STAGES;  // S^T_i complete
+  uint64_t* dpt_full = st_full + 1;         // dP^T_i complete
+  uint64_t* pds_full = dpt_full + 1;        // P^T_i, dS^T_i stored to TMEM
+  uint64_t* dv_done = pds_full + 1;         // dV += P^T_i dO_i complete: S^T columns free
+  uint64_t* dk_done = dv_done + 1;          // dK += dS^T_i Q_i complete: dP^T columns free
+  uint64_t* done = dk_done + 1;             // [2], one per issuing warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 2);
   const int n_qt = (S + BQ2 - 1) / BQ2;
   const uint64_t lim = p.timeout_ns;
 
   if (threadIdx.x == 0) {
     ptx::mbar_init(kv_full, 1);
-    for (int s = 0; s < STAGES; ++s) {
-      ptx::mbar_init(&q_full[s], 32);  // lane 0's expect_tx + 31 lanes' lse/delta stores
-      ptx::mbar_init(&q_empty[s], 2);  // the tile's S^T / dP^T and dV / dK products
+    for (int s = 0; s < KV_STAGES; ++s) {
+      ptx::mbar_init(&q_full[s], 1);  // lane 0's expect_tx (Q_i, dO_i, both X)
+      ptx::mbar_init(&q_empty[s], 2);  // the tile's dV and dK products (each after its score product)
     }
-    ptx::mbar_init(s_full, 1);
-    ptx::mbar_init(s_free, NSM_B);
+    ptx::mbar_init(st_full, 1);
+    ptx::mbar_init(dpt_full, 1);
     ptx::mbar_init(pds_full, NSM_B);
-    ptx::mbar_init(mm_done, 1);
+    ptx::mbar_init(dv_done, 1);
+    ptx::mbar_init(dk_done, 1);
     ptx::mbar_init(&done[0], 1);
     ptx::mbar_init(&done[1], 1);
     ptx::fence_mbar_init();
@@ -710,17 +734,23 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
     ptx::tmem_alloc(tmem_slot, 256);
     ptx::tmem_relinquish();
   }
+  // E: rows [1, 1, 0 x 6] (bf16); the X ring and the zero block: zeros
+  for (int w = threadIdx.x; w < (KV_RED_OFF - KV_E_OFF) / 16; w += NTHR_B)
+    *reinterpret_cast<uint4*>(smem + KV_E_OFF + w * 16) =
+        make_uint4(w < BK2 ? 0x3F803F80u : 0u, 0u, 0u, 0u);
+  ptx::fence_proxy_async_smem();
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // S^T (then P^T, bf16 pairs), dP^T (then dS^T), dV, dK accumulators.  The
+  // column half hf of S^T (queries 32 hf ..) holds that half's P^T in its
+  // first 16 columns, so the two halves never write columns the other reads.
   const uint32_t tST = tmem, tdPT = tmem + 64, tdV = tmem + 128, tdK = tmem + 192;
 
   if (warp == 0) {
     // producer: K, V once; per query tile Q_i, dO_i by TMA and the tile's
-    // log-sum-exp / delta values by bulk copy (or by the warp's lanes when the
-    // rows are not 16-byte aligned), all completing on q_full
-    const bool bulk = p.lse_bulk != 0;
+    // two X matrices by bulk copy, all completing on q_full
     if (lane == 0) {
       ptx::prefetch_tensormap(&tmK);
       ptx::prefetch_tensormap(&tmQ);
@@ -729,98 +759,75 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
       ptx::tma_load_2d(smem + KV_K_OFF, &tmK, kv_full, H + a * HD, row0 + k0);
       ptx::tma_load_2d(smem + KV_V_OFF, &tmK, kv_full, 2 * H + a * HD, row0 + k0);
     }
-    const float* lse_b = p.lse + (static_cast<int64_t>(b) * p.A + a) * S;
-    const float* del_b = p.delta + (static_cast<int64_t>(b) * p.A + a) * S;
+    // this (sequence, head)'s X_lse rows, followed by its X_delta rows
+    const uint4* xs_b = p.xtab + (static_cast<int64_t>(b) * p.A + a) * 2 * S;
     int issued = 0;
-    for (int i = 0; i < n_qt; ++i) {
-      const int st = i & 1;
-      bool ok = true;
-      if (lane == 0) ok = ptx::mbar_wait(&q_empty[st], ((i >> 1) & 1) ^ 1u, lim, p.status, kWaitHint);
-      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
-      float* l2 = ldst + st * 2 * BQ2;
-      const int nq = min(BQ2, S - i * BQ2);  // queries of this tile inside the sequence
-      if (!bulk) {
-        for (int t = lane; t < nq; t += 32) {
-          l2[t] = lse_b[i * BQ2 + t];
-          l2[BQ2 + t] = del_b[i * BQ2 + t];
-        }
-      }
-      if (lane == 0) {
-        const uint32_t lbytes = bulk ? static_cast<uint32_t>(nq) * 4u : 0u;
-        ptx::mbar_arrive_expect_tx(&q_full[st], 2 * QO2_BYTES + 2 * lbytes);
-        ptx::tma_load_2d(smem + KV_Q_OFF + st * QO2_BYTES, &tmQ, &q_full[st], a * HD,
-                         row0 + i * BQ2);
-        ptx::tma_load_2d(smem + KV_O_OFF + st * QO2_BYTES, &tmO, &q_full[st], a * HD,
-                         row0 + i * BQ2);
-        if (bulk) {
-          ptx::bulk_load(l2, lse_b + i * BQ2, lbytes, &q_full[st]);
-          ptx::bulk_load(l2 + BQ2, del_b + i * BQ2, lbytes, &q_full[st]);
-        }
-      } else {
-        ptx::mbar_arrive(&q_full[st]);
-      }
+    for (int i = 0; i < n_qt && lane == 0; ++i) {
+      const int st = i % KV_STAGES;
+      if (!ptx::mbar_wait(&q_empty[st], ((i / KV_STAGES) & 1) ^ 1u, lim, p.status, kWaitHint)) break;
+      const uint32_t xbytes = static_cast<uint32_t>(min(BQ2, S - i * BQ2)) * XROW_BYTES;
+      ptx::mbar_arrive_expect_tx(&q_full[st], 2 * QO2_BYTES + 2 * xbytes);
+      ptx::tma_load_2d(smem + KV_Q_OFF + st * QO2_BYTES, &tmQ, &q_full[st], a * HD, row0 + i * BQ2);
+      ptx::tma_load_2d(smem + KV_O_OFF + st * QO2_BYTES, &tmO, &q_full[st], a * HD, row0 + i * BQ2);
+      uint8_t* x = smem + KV_X_OFF + st * 2 * X_BYTES;
+      ptx::bulk_load(x, xs_b + i * BQ2, xbytes, &q_full[st]);
+      ptx::bulk_load(x + X_BYTES, xs_b + S + i * BQ2, xbytes, &q_full[st]);
       ++issued;
     }
     if (lane == 0) {
       ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint);
-      for (int i = issued - 1; i >= 0 && i >= issued - STAGES; --i)
-        ptx::mbar_wait(&q_full[i & 1], (i >> 1) & 1, lim, p.status, kWaitHint);
+      for (int i = issued - 1; i >= 0 && i >= issued - KV_STAGES; --i)
+        ptx::mbar_wait(&q_full[i % KV_STAGES], (i / KV_STAGES) & 1, lim, p.status, kWaitHint);
     }
-  } else if (warp == 1) {
-    // S^T_i = K Q_i^T and dP^T_i = V dO_i^T, as soon as the softmax warps
-    // hold S^T_{i-1} / dP^T_{i-1} in registers (s_free) and Q_i / dO_i have landed
+  } else if (warp == 1 || warp == 10) {
+    // Warp 1: S^T_i = K Q_i^T, then dV += P^T_i dO_i.  Warp 10: dP^T_i =
+    // V dO_i^T, then dK += dS^T_i Q_i.  Each warp's score product of tile i
+    // goes in once its accumulating product of tile i - 1 has read the
+    // columns it overwrites; the accumulating product once the softmax warps
+    // have stored P^T_i / dS^T_i.
     if (lane == 0) {
+      const bool v_side = warp == 1;
       constexpr uint32_t idS = ptx::idesc_bf16_f32(BK2, BQ2, false, false);
-      const uint32_t sk = ptx::smem_u32(smem + KV_K_OFF), sv = ptx::smem_u32(smem + KV_V_OFF);
+      constexpr uint32_t idG = ptx::idesc_bf16_f32(BK2, HD, false, true);
+      const uint32_t skv = ptx::smem_u32(smem + (v_side ? KV_K_OFF : KV_V_OFF));
+      const uint32_t tscore = v_side ? tST : tdPT, tacc = v_side ? tdV : tdK;
+      uint64_t* score_full = v_side ? st_full : dpt_full;
+      uint64_t* acc_done = v_side ? dv_done : dk_done;
+      // K-major operand of the score product (Q_i or dO_i) and MN-major
+      // operand of the accumulating product (dO_i or Q_i)
+      const int score_off = v_side ? KV_Q_OFF : KV_O_OFF, acc_off = v_side ? KV_O_OFF : KV_Q_OFF;
+      const uint32_t se = ptx::smem_u32(smem + KV_E_OFF), sz = ptx::smem_u32(smem + KV_Z_OFF);
+      const uint32_t sx = ptx::smem_u32(smem + KV_X_OFF + (v_side ? 0 : X_BYTES));
       bool ok = ptx::mbar_wait(kv_full, 0, lim, p.status, kWaitHint);
       for (int i = 0; i < n_qt && ok; ++i) {
-        const int st = i & 1;
-        if (i >= 1 && !ptx::mbar_wait(s_free, (i - 1) & 1, lim, p.status, kWaitHint)) break;
-        if (!ptx::mbar_wait(&q_full[st], (i >> 1) & 1, lim, p.status, kWaitHint)) break;
+        const int st = i % KV_STAGES;
+        if (i >= 1 && !ptx::mbar_wait(acc_done, (i - 1) & 1, lim, p.status, kWaitHint)) break;
+        if (!ptx::mbar_wait(&q_full[st], (i / KV_STAGES) & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
-        const uint32_t sq = ptx::smem_u32(smem + KV_Q_OFF + st * QO2_BYTES);
-        const uint32_t so = ptx::smem_u32(smem + KV_O_OFF + st * QO2_BYTES);
+        const uint32_t sb = ptx::smem_u32(smem + score_off + st * QO2_BYTES);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
-          ptx::tc_mma_f16(tST, ptx::smem_desc_sw128(sk + kk * 32, 16, 1024),
-                          ptx::smem_desc_sw128(sq + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          ptx::tc_mma_f16(tdPT, ptx::smem_desc_sw128(sv + kk * 32, 16, 1024),
-                          ptx::smem_desc_sw128(so + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
-        ptx::tc_commit(s_full);
-        ptx::tc_commit(&q_empty[st]);
-      }
-      ptx::tc_commit(&done[0]);
-      ptx::mbar_wait(&done[0], 0, lim, p.status, kWaitHint);
-    }
-  } else if (warp == 10) {
-    // dV += P^T_i dO_i and dK += dS^T_i Q_i, in tile order, from a warp of
-    // its own so that they go in beside the next tile's score products
-    if (lane == 0) {
-      constexpr uint32_t idG = ptx::idesc_bf16_f32(BK2, HD, false, true);
-      const uint32_t sp = ptx::smem_u32(smem + KV_P_OFF), sds = ptx::smem_u32(smem + KV_DS_OFF);
-      for (int i = 0; i < n_qt; ++i) {
-        const int st = i & 1;
+          ptx::tc_mma_f16(tscore, ptx::smem_desc_sw128(skv + kk * 32, 16, 1024),
+                          ptx::smem_desc_sw128(sb + kk * 32, 16, 1024), idS, kk > 0 ? 1u : 0u);
+        // the per-query term: E X^T
+        const uint32_t sxs = sx + st * 2 * X_BYTES;
+        ptx::tc_mma_f16(tscore, ptx::smem_desc_noswizzle(se, sz - se, 128),
+                        ptx::smem_desc_noswizzle(sxs, sz - sxs, 128), idS, 1u);
+        ptx::tc_commit(score_full);
         if (!ptx::mbar_wait(pds_full, i & 1, lim, p.status, kWaitHint)) break;
-        if (!ptx::mbar_wait(&q_full[st], (i >> 1) & 1, lim, p.status, kWaitHint)) break;
         ptx::tc_fence_after();
-        const uint32_t sq = ptx::smem_u32(smem + KV_Q_OFF + st * QO2_BYTES);
-        const uint32_t so = ptx::smem_u32(smem + KV_O_OFF + st * QO2_BYTES);
+        const uint32_t sa = ptx::smem_u32(smem + acc_off + st * QO2_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < BQ2 / 16; ++kk) {
-          ptx::tc_mma_f16(tdV, ptx::smem_desc_sw128(sp + kk * 32, 16, 1024),
-                          ptx::smem_desc_sw128(so + kk * 2048, 8192, 1024), idG,
-                          (i > 0 || kk > 0) ? 1u : 0u);
-          ptx::tc_mma_f16(tdK, ptx::smem_desc_sw128(sds + kk * 32, 16, 1024),
-                          ptx::smem_desc_sw128(sq + kk * 2048, 8192, 1024), idG,
-                          (i > 0 || kk > 0) ? 1u : 0u);
-        }
-        ptx::tc_commit(mm_done);
+        for (int kk = 0; kk < BQ2 / 16; ++kk)  // queries 16 kk ..: half kk / 2, packed column 8 (kk % 2)
+          ptx::tc_mma_f16_tmem_a(tacc, tscore + (kk >> 1) * 32 + (kk & 1) * 8,
+                                 ptx::smem_desc_sw128(sa + kk * 2048, 8192, 1024), idG,
+                                 (i > 0 || kk > 0) ? 1u : 0u);
+        ptx::tc_commit(acc_done);
         ptx::tc_commit(&q_empty[st]);
       }
-      ptx::tc_commit(&done[1]);
-      ptx::mbar_wait(&done[1], 0, lim, p.status, kWaitHint);
+      uint64_t* fin = &done[v_side ? 0 : 1];
+      ptx::tc_commit(fin);
+      ptx::mbar_wait(fin, 0, lim, p.status, kWaitHint);
     }
   } else {
     const int q4 = warp & 3;
@@ -830,46 +837,33 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
     const bool kvalid = key < len;
     const uint32_t lane_base = static_cast<uint32_t>(q4 * 32) << 16;
     const float sl2 = LOG2E * 0.125f;
-    uint8_t* prow = smem + KV_P_OFF + r * 128;
-    uint8_t* drow = smem + KV_DS_OFF + r * 128;
     bool ok = true;
     auto wait_all = [&](uint64_t* bar, uint32_t parity) {
       const bool mine = ptx::mbar_wait(bar, parity, lim, p.status, kWaitHint);
       return __all_sync(0xffffffffu, mine);
     };
     for (int i = 0; i < n_qt; ++i) {
-      const int st = i & 1;
-      if (!wait_all(&q_full[st], (i >> 1) & 1)) { ok = false; break; }
-      if (!wait_all(s_full, i & 1)) { ok = false; break; }
+      if (!wait_all(st_full, i & 1) || !wait_all(dpt_full, i & 1)) { ok = false; break; }
       ptx::tc_fence_after();
       uint32_t sv[32], dv[32];
       ptx::tmem_ld_32x32b_x32(tST + lane_base + hf * 32, sv);
       ptx::tmem_ld_32x32b_x32(tdPT + lane_base + hf * 32, dv);
       ptx::tmem_ld_wait();
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(s_free);
-      const float* l2 = ldst + st * 2 * BQ2 + hf * 32;
+      // sv = S^T - lse2 / c and dv = dP^T - delta, the terms added by the MMAs
       uint32_t pp[16], dd[16];
 #pragma unroll
-      for (int t = 0; t < 32; t += 4) {
-        // base-2 log-sum-exp / delta of queries t .. t+3: one broadcast 16-byte load each
-        const float4 lq = *reinterpret_cast<const float4*>(l2 + t);
-        const float4 dq = *reinterpret_cast<const float4*>(l2 + BQ2 + t);
-        const float lv[4] = {lq.x, lq.y, lq.z, lq.w};
-        const float dlv[4] = {dq.x, dq.y, dq.z, dq.w};
-        float pt[4], ds[4];
+      for (int t = 0; t < 32; t += 2) {
+        float pt[2], ds[2];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          pt[e] = kvalid ? ptx::ex2_ftz(fmaf(__uint_as_float(sv[t + e]), sl2, -lv[e])) : 0.f;
-          ds[e] = pt[e] * (__uint_as_float(dv[t + e]) - dlv[e]);
+        for (int e = 0; e < 2; ++e) {
+          pt[e] = kvalid ? ptx::ex2_ftz(__uint_as_float(sv[t + e]) * sl2) : 0.f;
+          ds[e] = pt[e] * __uint_as_float(dv[t + e]);
         }
         pp[t >> 1] = ptx::pack_bf16(pt[0], pt[1]);
-        pp[(t >> 1) + 1] = ptx::pack_bf16(pt[2], pt[3]);
         dd[t >> 1] = ptx::pack_bf16(ds[0], ds[1]);
-        dd[(t >> 1) + 1] = ptx::pack_bf16(ds[2], ds[3]);
       }
       const int nq = S - i * BQ2 - hf * 32;  // queries of this half inside the sequence
-      if (nq < 32) {  // warp-uniform: queries past S (their lse / delta slots are stale)
+      if (nq < 32) {  // warp-uniform: queries past S
 #pragma unroll
         for (int t = 0; t < 32; t += 2) {
           const uint32_t keep = (t < nq ? 0x0000ffffu : 0u) | (t + 1 < nq ? 0xffff0000u : 0u);
@@ -877,21 +871,16 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
           dd[t >> 1] &= keep;
         }
       }
-      // P^T / dS^T buffers were last read by the dV / dK products of tile i - 1
-      if (i > 0 && !wait_all(mm_done, (i - 1) & 1)) { ok = false; break; }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int pos = ((hf * 4 + u) ^ (r & 7)) << 4;
-        *reinterpret_cast<uint4*>(prow + pos) = make_uint4(pp[4 * u], pp[4 * u + 1], pp[4 * u + 2], pp[4 * u + 3]);
-        *reinterpret_cast<uint4*>(drow + pos) = make_uint4(dd[4 * u], dd[4 * u + 1], dd[4 * u + 2], dd[4 * u + 3]);
-      }
-      ptx::fence_proxy_async_smem();
+      // over the columns this thread has just read: P^T_i, dS^T_i as bf16 pairs
+      ptx::tmem_st_32x32b_x16(tST + lane_base + hf * 32, pp);
+      ptx::tmem_st_32x32b_x16(tdPT + lane_base + hf * 32, dd);
+      ptx::tmem_st_wait();
       ptx::tc_fence_before();
       ptx::mbar_arrive(pds_full);
     }
     // epilogue: the low-half warps write dK / sqrt(D), the high-half warps dV
-    float* red = reinterpret_cast<float*>(smem + KV_P_OFF);  // [2 halves][4 quarters][64]: P^T is idle
-    if (ok && wait_all(mm_done, (n_qt - 1) & 1)) {
+    float* red = reinterpret_cast<float*>(smem + KV_RED_OFF);  // [2 halves][4 quarters][64]
+    if (ok && wait_all(dv_done, (n_qt - 1) & 1) && wait_all(dk_done, (n_qt - 1) & 1)) {
       ptx::tc_fence_after();
       const uint32_t tacc = hf == 0 ? tdK : tdV;
       const float sc = hf == 0 ? 0.125f : 1.f;
@@ -1001,7 +990,7 @@ sky_status attention_fwd_tc(const void* qkv, const int32_t* lens, int B, int S, 
 
 // Backward launchers (bf16, D = 64): delta must already hold rowsum(dO * O).
 sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse, const float* delta,
-                            const int32_t* lens, int B, int S, int H, int A, void* dqkv,
+                            const uint4* xtab, const int32_t* lens, int B, int S, int H, int A, void* dqkv,
                             int32_t* status, uint64_t timeout_ns, cudaStream_t stream,
                             float* colpart) {
   using namespace attn_tc;
@@ -1016,9 +1005,9 @@ sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse,
   static cudaError_t a2 = cudaFuncSetAttribute(attn_bwd_dkdv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, KV_SMEM);
   if (a1 != cudaSuccess) return cuda_fail(a1, "attention dQ smem attribute");
   if (a2 != cudaSuccess) return cuda_fail(a2, "attention dK/dV smem attribute");
-  const int bulk = (S % 4 == 0) && (reinterpret_cast<uintptr_t>(lse) & 15) == 0 &&
-                   (reinterpret_cast<uintptr_t>(delta) & 15) == 0;
-  BwdParams p{S, H, A, bulk, lens, lse, delta, static_cast<__nv_bfloat16*>(dqkv), colpart, status,
+  SKY_CHECK((reinterpret_cast<uintptr_t>(xtab) & 15) == 0, SKY_ERR_INVALID_ARG,
+            "attention backward workspace must be 16-byte aligned");
+  BwdParams p{S, H, A, lens, lse, delta, xtab, static_cast<__nv_bfloat16*>(dqkv), colpart, status,
               timeout_ns};
   cudaError_t e = launch_pdl(attn_bwd_dkdv_tc, dim3(ceil_div(S, BK2), A, B), dim3(NTHR_B), KV_SMEM,
                              stream, 1, tk128, tq64, to64, p);

@@ -8,6 +8,8 @@ namespace sky {
 
 sky_status attention_fwd(const void* qkv, const int32_t* lens, int B, int S, int H, int A,
                          sky_dtype dt, void* ctx, float* lse, int32_t* status, cudaStream_t st);
+// Scratch of attention_bwd (`delta` below), 16-byte aligned: the per-query
+// delta terms and, for bf16, the dK/dV kernel's per-query MMA operand rows.
 size_t attention_bwd_ws(int B, int S, int A);
 // colpart (bf16 only, optional): column sums of the stored dqkv, one row per
 // 128-row tile of each sequence: colpart[b * ceil(S/128) + tile][3H].

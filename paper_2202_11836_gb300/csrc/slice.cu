@@ -747,7 +747,8 @@ static sky_status plan_slice(sky_slice* s, size_t* total) {
   // dP[2] dR[2] dU2_32 dP1 | dU2b dU1b dctx (bf16) | dH | dqkv | delta | ws | ws2 | lnp[2] |
   // db1p | qkvp | status | x32 (bf16)
   const size_t wk = (bf ? 7 : 6) * t32 + (bf ? 3 : 1) * th + align_up((size_t)T * s->F * s->esz) +
-                    align_up((size_t)T * 3 * s->H * s->esz) + lse + s->ws_bytes +
+                    align_up((size_t)T * 3 * s->H * s->esz) +
+                    align_up(attention_bwd_ws(c.max_batch, c.max_seq, s->A)) + s->ws_bytes +
                     s->ws2_bytes + 4 * s->lnp_bytes + 2 * s->db1p_bytes + 2 * s->qkvp_bytes + 256 +
                     (s->n_slots > 1 ? gb : 0);  // gradient-accumulation scratch (one layer)
   s->ws_bytes_total = wk;
@@ -857,7 +858,7 @@ sky_status sky_slice_create(const sky_slice_config* cfg, sky_slice** out) {
   s->dctx = take(th);
   s->dH = take((size_t)T * s->F * s->esz);
   s->dqkv = take((size_t)T * 3 * s->H * s->esz);
-  s->delta = static_cast<float*>(take(lse_b));
+  s->delta = static_cast<float*>(take(attention_bwd_ws(c.max_batch, c.max_seq, s->A)));
   s->ws = take(s->ws_bytes);
   if (s->ws2_bytes) s->ws2 = take(s->ws2_bytes);
   for (int k = 0; k < 2; ++k) {
