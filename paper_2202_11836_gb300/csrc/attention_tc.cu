@@ -79,6 +79,7 @@ struct FwdParams {
 
 __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ CUtensorMap tmQ,
                                                     const __grid_constant__ CUtensorMap tmKV,
+                                                    const __grid_constant__ CUtensorMap tmOut,
                                                     const FwdParams p) {
   pdl_trigger();
   pdl_wait();
@@ -294,30 +295,37 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
       ptx::tc_fence_before();
       ptx::mbar_arrive(&p_full[j & 1]);
     }
-    // epilogue: O / l -> ctx (bf16), log-sum-exp
+    // epilogue: O / l -> ctx (bf16) as 128-byte-swizzled rows over the Q
+    // tile (the last S product has read it), stored by one TMA that drops the
+    // rows past S; the log-sum-exp directly
     if (ok && wait_all(&pv_done[(n_kt - 1) & 1], ((n_kt - 1) >> 1) & 1)) {
       ptx::tc_fence_after();
       const float inv = 1.f / l;
       const int q = q0 + r;
-      __nv_bfloat16* out = p.ctx + (static_cast<int64_t>(row0) + q) * H + a * HD;
+      const uint32_t orow = ptx::smem_u32(smem + F_Q_OFF) + r * 128;
 #pragma unroll
       for (int c = 0; c < HD / 32; ++c) {
         uint32_t o[32];
         ptx::tmem_ld_32x32b_x32(tO + lane_base + c * 32, o);
         ptx::tmem_ld_wait();
-        if (q < S) {
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            uint32_t w[4];
+        for (int u = 0; u < 4; ++u) {
+          uint32_t w[4];
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
-              w[t] = ptx::pack_bf16(__uint_as_float(o[8 * u + 2 * t]) * inv,
-                                    __uint_as_float(o[8 * u + 2 * t + 1]) * inv);
-            *reinterpret_cast<uint4*>(out + c * 32 + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-          }
+          for (int t = 0; t < 4; ++t)
+            w[t] = ptx::pack_bf16(__uint_as_float(o[8 * u + 2 * t]) * inv,
+                                  __uint_as_float(o[8 * u + 2 * t + 1]) * inv);
+          ptx::st_shared_v4(orow + (((c * 4 + u) ^ (r & 7)) << 4), w[0], w[1], w[2], w[3]);
         }
       }
       if (q < S) p.lse[(static_cast<int64_t>(b) * p.A + a) * S + q] = m + log2f(l);
+    }
+    ptx::fence_proxy_async_smem();  // the staged rows -> the TMA store
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // the four softmax warps
+    if (warp == 2 && lane == 0) {
+      ptx::tma_store_3d(&tmOut, smem + F_Q_OFF, a * HD, q0, b);
+      ptx::bulk_commit_group();
+      ptx::bulk_wait_group_read0();  // before the CTA's memory goes
     }
   }
   ptx::tc_fence_before();
@@ -384,6 +392,7 @@ __device__ __forceinline__ void softmax_warps_sync() {
 __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorMap tmQ,
                                                           const __grid_constant__ CUtensorMap tmKV,
                                                           const __grid_constant__ CUtensorMap tmO,
+                                                          const __grid_constant__ CUtensorMap tmOut,
                                                           const BwdParams p) {
   // Launched right behind the dK/dV kernel, which it does not depend on (it
   // writes the other columns of dQKV): it starts once every dK/dV CTA has
@@ -571,24 +580,24 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
       ptx::tc_fence_before();
       ptx::mbar_arrive(ds_full);
     }
-    // epilogue: each half writes 32 of the 64 dQ columns
+    // epilogue: each half stages 32 of the 64 dQ columns as 128-byte-swizzled
+    // bf16 rows over the Q tile (the last S product has read it); one thread
+    // then stores the tile by TMA, which drops the rows past S
     float* red = reinterpret_cast<float*>(smem + DQ_KV_OFF);  // [4 row quarters][64]: ring is idle
     if (ok && wait_all(dq_done, (n_kt - 1) & 1)) {
       ptx::tc_fence_after();
-      __nv_bfloat16* out = p.dqkv + (static_cast<int64_t>(row0) + q) * (3 * H) + a * HD + hf * 32;
+      const uint32_t orow = ptx::smem_u32(smem + DQ_Q_OFF) + r * 128;
       uint32_t o[32];
       ptx::tmem_ld_32x32b_x32(tdQ + lane_base + hf * 32, o);
       ptx::tmem_ld_wait();
-      if (q < S) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          uint32_t w[4];
+      for (int u = 0; u < 4; ++u) {
+        uint32_t w[4];
 #pragma unroll
-          for (int t = 0; t < 4; ++t)
-            w[t] = ptx::pack_bf16(__uint_as_float(o[8 * u + 2 * t]) * 0.125f,
-                                  __uint_as_float(o[8 * u + 2 * t + 1]) * 0.125f);
-          *reinterpret_cast<uint4*>(out + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-        }
+        for (int t = 0; t < 4; ++t)
+          w[t] = ptx::pack_bf16(__uint_as_float(o[8 * u + 2 * t]) * 0.125f,
+                                __uint_as_float(o[8 * u + 2 * t + 1]) * 0.125f);
+        ptx::st_shared_v4(orow + (((hf * 4 + u) ^ (r & 7)) << 4), w[0], w[1], w[2], w[3]);
       }
       if (p.colpart) {  // column sums of the stored values over this warp's 32 rows
         float v[32];
@@ -600,14 +609,18 @@ __global__ void __maxnreg__(80) attn_bwd_dq_tc(const __grid_constant__ CUtensorM
     } else if (p.colpart) {
       red[q4 * 64 + hf * 32 + lane] = 0.f;
     }
-    if (p.colpart) {  // the four row quarters, added in order, by the quarter-0 warps
-      softmax_warps_sync();
-      if (q4 == 0) {
-        const int c = hf * 32 + lane;
-        const float sum = ((red[c] + red[64 + c]) + red[128 + c]) + red[192 + c];
-        p.colpart[(static_cast<int64_t>(b) * gridDim.x + qt) * (3 * H) + a * HD + c] = sum;
-      }
+    ptx::fence_proxy_async_smem();  // the staged rows -> the TMA store
+    softmax_warps_sync();
+    if (warp == 2 && lane == 0) {
+      ptx::tma_store_3d(&tmOut, smem + DQ_Q_OFF, a * HD, q0, b);
+      ptx::bulk_commit_group();
     }
+    if (p.colpart && q4 == 0) {  // the four row quarters, added in order, by the quarter-0 warps
+      const int c = hf * 32 + lane;
+      const float sum = ((red[c] + red[64 + c]) + red[128 + c]) + red[192 + c];
+      p.colpart[(static_cast<int64_t>(b) * gridDim.x + qt) * (3 * H) + a * HD + c] = sum;
+    }
+    if (warp == 2 && lane == 0) ptx::bulk_wait_group_read0();  // before the CTA's memory goes
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -668,6 +681,7 @@ static_assert(3 * (KV_SMEM + 1024) > 233472 && 2 * (KV_SMEM + 1024) <= 233472,
 __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtensorMap tmK,
                                                             const __grid_constant__ CUtensorMap tmQ,
                                                             const __grid_constant__ CUtensorMap tmO,
+                                                            const __grid_constant__ CUtensorMap tmOut,
                                                             const BwdParams p) {
   // wait first, then let the dQ kernel start: once every CTA here has passed
   // the wait, the delta pre-pass (and everything before it) is complete
@@ -878,30 +892,31 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
       ptx::tc_fence_before();
       ptx::mbar_arrive(pds_full);
     }
-    // epilogue: the low-half warps write dK / sqrt(D), the high-half warps dV
+    // epilogue: the low-half warps stage dK / sqrt(D), the high-half warps dV,
+    // as 128-byte-swizzled bf16 rows over the K / V tiles (the last score
+    // products have read them); one thread then stores both tiles by TMA
+    // through a [B][S][3H] map, which drops the rows past S.
     float* red = reinterpret_cast<float*>(smem + KV_RED_OFF);  // [2 halves][4 quarters][64]
     if (ok && wait_all(dv_done, (n_qt - 1) & 1) && wait_all(dk_done, (n_qt - 1) & 1)) {
       ptx::tc_fence_after();
       const uint32_t tacc = hf == 0 ? tdK : tdV;
       const float sc = hf == 0 ? 0.125f : 1.f;
-      __nv_bfloat16* out = p.dqkv + (static_cast<int64_t>(row0) + key) * rs + (1 + hf) * H + a * HD;
+      const uint32_t orow = ptx::smem_u32(smem + (hf == 0 ? KV_K_OFF : KV_V_OFF)) + r * 128;
       uint32_t o[2][32];
       ptx::tmem_ld_32x32b_x32(tacc + lane_base, o[0]);
       ptx::tmem_ld_32x32b_x32(tacc + lane_base + 32, o[1]);
       ptx::tmem_ld_wait();
-      if (key < S) {
 #pragma unroll
-        for (int c = 0; c < 2; ++c)
+      for (int c = 0; c < 2; ++c)
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            uint32_t w[4];
+        for (int u = 0; u < 4; ++u) {
+          uint32_t w[4];
 #pragma unroll
-            for (int t = 0; t < 4; ++t)
-              w[t] = ptx::pack_bf16(__uint_as_float(o[c][8 * u + 2 * t]) * sc,
-                                    __uint_as_float(o[c][8 * u + 2 * t + 1]) * sc);
-            *reinterpret_cast<uint4*>(out + c * 32 + u * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-          }
-      }
+          for (int t = 0; t < 4; ++t)
+            w[t] = ptx::pack_bf16(__uint_as_float(o[c][8 * u + 2 * t]) * sc,
+                                  __uint_as_float(o[c][8 * u + 2 * t + 1]) * sc);
+          ptx::st_shared_v4(orow + (((c * 4 + u) ^ (r & 7)) << 4), w[0], w[1], w[2], w[3]);
+        }
       if (p.colpart) {  // column sums of the stored values over this warp's 32 rows
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
@@ -916,16 +931,21 @@ __global__ void __maxnreg__(80) attn_bwd_dkdv_tc(const __grid_constant__ CUtenso
       red[(hf * 4 + q4) * 64 + lane] = 0.f;
       red[(hf * 4 + q4) * 64 + 32 + lane] = 0.f;
     }
-    if (p.colpart) {  // the four row quarters, added in order, by the quarter-0 warps
-      softmax_warps_sync();
-      if (q4 == 0) {
-        const float* rh = red + hf * 4 * 64;
-        float* dst = p.colpart + (static_cast<int64_t>(b) * gridDim.x + kt) * rs + (1 + hf) * H + a * HD;
-#pragma unroll
-        for (int c = lane; c < 64; c += 32)
-          dst[c] = ((rh[c] + rh[64 + c]) + rh[128 + c]) + rh[192 + c];
-      }
+    ptx::fence_proxy_async_smem();  // the staged rows -> the TMA store
+    softmax_warps_sync();
+    if (warp == 2 && lane == 0) {
+      ptx::tma_store_3d(&tmOut, smem + KV_K_OFF, H + a * HD, k0, b);
+      ptx::tma_store_3d(&tmOut, smem + KV_V_OFF, 2 * H + a * HD, k0, b);
+      ptx::bulk_commit_group();
     }
+    if (p.colpart && q4 == 0) {  // the four row quarters, added in order, by the quarter-0 warps
+      const float* rh = red + hf * 4 * 64;
+      float* dst = p.colpart + (static_cast<int64_t>(b) * gridDim.x + kt) * rs + (1 + hf) * H + a * HD;
+#pragma unroll
+      for (int c = lane; c < 64; c += 32)
+        dst[c] = ((rh[c] + rh[64 + c]) + rh[128 + c]) + rh[192 + c];
+    }
+    if (warp == 2 && lane == 0) ptx::bulk_wait_group_read0();  // before the CTA's memory goes
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -962,6 +982,21 @@ bool head_map(CUtensorMap* map, const void* base, int64_t T, int W, int rows) {
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
+
+// dQKV as [B][S][3H] bf16 for the dK/dV tile stores: box {64 columns, 128
+// rows of one sequence}, 128B swizzle; rows past S fall outside the tensor.
+bool seq_map(CUtensorMap* map, void* base, int B, int S, int W, int rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(W), static_cast<cuuint64_t>(S),
+                        static_cast<cuuint64_t>(B)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(W) * 2, static_cast<cuuint64_t>(W) * 2 * S};
+  cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(rows), 1u};
+  cuuint32_t estr[3] = {1u, 1u, 1u};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 }  // namespace
 
 }  // namespace attn_tc
@@ -974,16 +1009,18 @@ sky_status attention_fwd_tc(const void* qkv, const int32_t* lens, int B, int S, 
   SKY_CHECK(H == A * HD, SKY_ERR_UNSUPPORTED, "tensor-core attention needs head dim 64");
   SKY_CHECK((reinterpret_cast<uintptr_t>(qkv) & 15) == 0 && (reinterpret_cast<uintptr_t>(ctx) & 15) == 0,
             SKY_ERR_UNSUPPORTED, "attention buffers must be 16-byte aligned");
-  CUtensorMap tq, tkv;
+  CUtensorMap tq, tkv, tout;
   const int64_t T = static_cast<int64_t>(B) * S;
-  SKY_CHECK(head_map(&tq, qkv, T, 3 * H, BQ) && head_map(&tkv, qkv, T, 3 * H, BKV), SKY_ERR_CUDA,
+  SKY_CHECK(head_map(&tq, qkv, T, 3 * H, BQ) && head_map(&tkv, qkv, T, 3 * H, BKV) &&
+                seq_map(&tout, ctx, B, S, H, BQ),
+            SKY_ERR_CUDA,
             "cuTensorMapEncodeTiled failed for the attention operands");
   static cudaError_t attr = cudaFuncSetAttribute(attn_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  F_SMEM);
   if (attr != cudaSuccess) return cuda_fail(attr, "attention smem attribute");
   FwdParams p{S, H, A, lens, static_cast<__nv_bfloat16*>(ctx), lse, status, timeout_ns};
   dim3 grid(ceil_div(S, BQ), A, B);
-  const cudaError_t e = launch_pdl(attn_fwd_tc, grid, dim3(NTHR), F_SMEM, stream, 1, tq, tkv, p);
+  const cudaError_t e = launch_pdl(attn_fwd_tc, grid, dim3(NTHR), F_SMEM, stream, 1, tq, tkv, tout, p);
   count_launches(1);
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "tensor-core attention forward launch");
 }
@@ -996,10 +1033,11 @@ sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse,
   using namespace attn_tc;
   SKY_CHECK(H == A * HD, SKY_ERR_UNSUPPORTED, "tensor-core attention needs head dim 64");
   const int64_t T = static_cast<int64_t>(B) * S;
-  CUtensorMap tq128, tkv64, to128, tk128, tq64, to64;
+  CUtensorMap tq128, tkv64, to128, tk128, tq64, to64, tout;
   SKY_CHECK(head_map(&tq128, qkv, T, 3 * H, BQ) && head_map(&tkv64, qkv, T, 3 * H, BKV) &&
                 head_map(&to128, dctx, T, H, BQ) && head_map(&tk128, qkv, T, 3 * H, BK2) &&
-                head_map(&tq64, qkv, T, 3 * H, BQ2) && head_map(&to64, dctx, T, H, BQ2),
+                head_map(&tq64, qkv, T, 3 * H, BQ2) && head_map(&to64, dctx, T, H, BQ2) &&
+                seq_map(&tout, dqkv, B, S, 3 * H, BK2),
             SKY_ERR_CUDA, "cuTensorMapEncodeTiled failed for the attention backward operands");
   static cudaError_t a1 = cudaFuncSetAttribute(attn_bwd_dq_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, DQ_SMEM);
   static cudaError_t a2 = cudaFuncSetAttribute(attn_bwd_dkdv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, KV_SMEM);
@@ -1010,10 +1048,10 @@ sky_status attention_bwd_tc(const void* qkv, const void* dctx, const float* lse,
   BwdParams p{S, H, A, lens, lse, delta, xtab, static_cast<__nv_bfloat16*>(dqkv), colpart, status,
               timeout_ns};
   cudaError_t e = launch_pdl(attn_bwd_dkdv_tc, dim3(ceil_div(S, BK2), A, B), dim3(NTHR_B), KV_SMEM,
-                             stream, 1, tk128, tq64, to64, p);
+                             stream, 1, tk128, tq64, to64, tout, p);
   if (e == cudaSuccess)
     e = launch_pdl(attn_bwd_dq_tc, dim3(ceil_div(S, BQ), A, B), dim3(NTHR_B), DQ_SMEM, stream, 1,
-                   tq128, tkv64, to128, p);
+                   tq128, tkv64, to128, tout, p);
   count_launches(2);
   return e == cudaSuccess ? SKY_OK : cuda_fail(e, "tensor-core attention backward launch");
 }
