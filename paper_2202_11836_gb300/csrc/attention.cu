@@ -269,6 +269,11 @@ sky_status attention_bwd(const void* qkv, const void* ctx, const void* dctx, con
   const int dblocks = ceil_div(rows * A * 32, 256);
   if (dt == SKY_DTYPE_BF16) {
     SKY_CHECK(D == attn::HD, SKY_ERR_UNSUPPORTED, "bf16 attention needs head dim 64 (got %d)", D);
+    // every kernel below moves 16-byte vectors of these buffers (checked
+    // before the first launch)
+    const auto a16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };
+    SKY_CHECK(a16(qkv) && a16(ctx) && a16(dctx) && a16(dqkv) && a16(delta), SKY_ERR_INVALID_ARG,
+              "bf16 attention backward buffers and workspace must be 16-byte aligned");
     const auto* c = static_cast<const __nv_bfloat16*>(ctx);
     const auto* dc = static_cast<const __nv_bfloat16*>(dctx);
     const dim3 g(ceil_div(rows * 32, 256)), blk(256);

@@ -199,6 +199,27 @@ def test_attention_bad_length_sets_status():
     assert torch.isfinite(ctx.float()).all()
 
 
+def test_attention_bwd_rejects_misaligned_workspace():
+    # checked on the host before any kernel is launched: nothing runs
+    B, S, A = 1, 64, 1
+    H, qkv, dctx, lens = attn_case("bf16", B, S, A, [64])
+    q = to_device(qkv, "bf16")
+    do = to_device(dctx, "bf16")
+    ln = torch.from_numpy(lens).cuda()
+    ctx = torch.zeros((B * S, H), dtype=torch.bfloat16, device="cuda")
+    lse = torch.zeros((B, A, S), dtype=torch.float32, device="cuda")
+    dq = torch.zeros((B * S, 3 * H), dtype=torch.bfloat16, device="cuda")
+    wsb = L.lib().sky_attention_bwd_workspace_bytes(B, S, H, A)
+    ws = torch.empty(wsb + 16, dtype=torch.uint8, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    with pytest.raises(L.SkyError) as e:
+        L.call("sky_attention_bwd", P(q), P(ctx), P(do), P(lse), P(ln), B, S, H, A, 0,
+               P(dq), C.c_void_p(int(ws.data_ptr()) + 4), wsb, P(st), stream())
+    assert e.value.status == L.SKY_ERR_INVALID_ARG
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and not dq.any()
+
+
 @pytest.mark.parametrize("dt", ["bf16", "fp32"])
 @pytest.mark.parametrize("TH", [(300, 768), (257, 1024), (64, 128), (33, 2048)],
                          ids=lambda t: f"T{t[0]}H{t[1]}")
