@@ -10,8 +10,9 @@
 //   O += P_j V_j                   tcgen05.mma M=128 N=64 K=64, A = P_j from
 //                                  TMEM, B = V_j from shared memory -> TMEM
 // Q, K and V come straight out of the packed QKV activations by TMA (one
-// tensor map, per-head column offsets).  Because a thread owns a whole query
-// row, the row max and row sum need no shuffles.
+// tensor map, per-head column offsets), and O / l leaves by TMA from shared
+// memory.  Because a thread owns a whole query row, the row max and row sum
+// need no shuffles.
 //
 // The steps are pipelined inside the CTA: S and P have two TMEM buffers each,
 // so the MMA warp computes S_{j+1} (issued one tile
@@ -339,7 +340,8 @@ __global__ void __launch_bounds__(NTHR, 2) attn_fwd_tc(const __grid_constant__ C
 // ----------------------------------------------------------- backward, dQ
 // One CTA per 128 query rows of (b, a); per 64-key tile j < len:
 //   S = Q K_j^T, dP = dO V_j^T (TMEM); thread = query row:
-//   P = exp2(S log2(e)/sqrt(D) - lse2), dS = P (dP - delta) -> smem (bf16)
+//   P = exp2(S log2(e)/sqrt(D) - lse2), dS = P (dP - delta) -> TMEM as bf16
+//   pairs, the A operand of
 //   dQ += dS K_j (TMEM); finally dQ / sqrt(D) -> dQKV[:, Q block].
 // Pipelining: the softmax warps release S / dP as soon as they hold them in
 // registers (s_free), so S_{j+1} and dP_{j+1} run on the tensor cores while
