@@ -536,7 +536,11 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
   }
 }
 
-// Fixed-order sum of split-K partials: out[i] = sum_s ws[s][i].
+// Fixed-order sum of split-K partials: out[i] = sum_s ws[s][i], added in
+// split order.  SPLITS > 0: every split's load of a vector is issued before
+// the first add (a loop over a run-time count would wait for each load in
+// turn); SPLITS == 0: any count.
+template <int SPLITS>
 __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int splits, int64_t n,
                                      float* __restrict__ out) {
   pdl_trigger();
@@ -544,10 +548,22 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int splits, i
   const int64_t n4 = n / 4;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4;
        i += (int64_t)gridDim.x * blockDim.x) {
-    float4 acc = reinterpret_cast<const float4*>(ws)[i];
-    for (int s = 1; s < splits; ++s) {
-      const float4 v = reinterpret_cast<const float4*>(ws + s * n)[i];
-      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    float4 acc;
+    if constexpr (SPLITS > 0) {
+      float4 v[SPLITS];
+#pragma unroll
+      for (int s = 0; s < SPLITS; ++s) v[s] = reinterpret_cast<const float4*>(ws + s * n)[i];
+      acc = v[0];
+#pragma unroll
+      for (int s = 1; s < SPLITS; ++s) {
+        acc.x += v[s].x; acc.y += v[s].y; acc.z += v[s].z; acc.w += v[s].w;
+      }
+    } else {
+      acc = reinterpret_cast<const float4*>(ws)[i];
+      for (int s = 1; s < splits; ++s) {
+        const float4 v = reinterpret_cast<const float4*>(ws + s * n)[i];
+        acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+      }
     }
     reinterpret_cast<float4*>(out)[i] = acc;
   }
@@ -800,8 +816,17 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   if (p.splits > 1) {
     const int64_t n = static_cast<int64_t>(M) * N;
     const int blocks = static_cast<int>(std::min<int64_t>(ceil_div(n / 4 + 1, 256), sms * 8));
-    e = launch_pdl(splitk_reduce_kernel, dim3(blocks), dim3(256), 0, stream, 1,
-                   static_cast<const float*>(ws), p.splits, n, static_cast<float*>(C));
+    const float* wsf = static_cast<const float*>(ws);
+    float* cf = static_cast<float*>(C);
+    switch (p.splits) {
+      case 2: e = launch_pdl(splitk_reduce_kernel<2>, dim3(blocks), dim3(256), 0, stream, 1, wsf, p.splits, n, cf); break;
+      case 3: e = launch_pdl(splitk_reduce_kernel<3>, dim3(blocks), dim3(256), 0, stream, 1, wsf, p.splits, n, cf); break;
+      case 4: e = launch_pdl(splitk_reduce_kernel<4>, dim3(blocks), dim3(256), 0, stream, 1, wsf, p.splits, n, cf); break;
+      case 5: e = launch_pdl(splitk_reduce_kernel<5>, dim3(blocks), dim3(256), 0, stream, 1, wsf, p.splits, n, cf); break;
+      case 6: e = launch_pdl(splitk_reduce_kernel<6>, dim3(blocks), dim3(256), 0, stream, 1, wsf, p.splits, n, cf); break;
+      case 8: e = launch_pdl(splitk_reduce_kernel<8>, dim3(blocks), dim3(256), 0, stream, 1, wsf, p.splits, n, cf); break;
+      default: e = launch_pdl(splitk_reduce_kernel<0>, dim3(blocks), dim3(256), 0, stream, 1, wsf, p.splits, n, cf); break;
+    }
     count_launches(1);
     if (e != cudaSuccess) return cuda_fail(e, "splitk_reduce launch");
   }
