@@ -52,11 +52,13 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;           // two fp32 accumulators of 128 x 256
 constexpr int NUM_EPI_WARPS = 8;            // two per TMEM lane quarter (default)
 constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
-// CTA-pair variant: per CTA and stage A 128 x 64 + B 128 x 64 (32 KiB), five
-// stages (160 KiB).  Six stages (192 KiB) made most kernels timed alone
-// 1-2 us faster, but the GELU' data-gradient kernel 5 us slower and the
-// whole training step 30-40 us slower; four stages were slower everywhere.
+// CTA-pair variant: per CTA and stage A 128 x 64 + B 128 x 64 (32 KiB).  Six
+// stages (192 KiB) for every epilogue but the GELU' data gradient, which
+// keeps five: with six, its kernel ran 5 us slower (its epilogue prefetches
+// the whole tile's GELU'(z) and competes for bandwidth with the deeper
+// ring), while the others ran 1-2 us faster and the step 0.7% faster.
 constexpr int PAIR_STAGES = 5;
+constexpr int PAIR_STAGES_WIDE = 6;  // all but the GELU' data-gradient epilogue
 constexpr int PAIR_STAGE_BYTES = A_BYTES + (BN / 2) * BK * 2;
 
 // Launch shape per instantiation: epilogue warps (a multiple of 4, one group
@@ -69,7 +71,7 @@ struct Shape {
   static constexpr int EW = EPI == SKY_EPI_BIAS_GELU ? 16 : NUM_EPI_WARPS;
   static constexpr int CW = EW == 16 ? 16 : 32;              // epilogue chunk width (columns)
   static constexpr int THREADS = 64 + 32 * EW;
-  static constexpr int NST = PAIR ? PAIR_STAGES : STAGES;
+  static constexpr int NST = PAIR ? (EPI == SKY_EPI_GELU_BWD ? PAIR_STAGES : PAIR_STAGES_WIDE) : STAGES;
   static constexpr int SBYTES = PAIR ? PAIR_STAGE_BYTES : STAGE_BYTES;
   static constexpr int EPI_OFF = NST * SBYTES;               // per epilogue warp: 32 x CW fp32 staging
   static constexpr int BAR_OFF = EPI_OFF + EW * 32 * CW * 4;
