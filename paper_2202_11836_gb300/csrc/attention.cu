@@ -50,7 +50,8 @@ __global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __rest
     }
     return acc;
   };
-  auto finish = [&](float acc, int col) {
+  // lz: the row's lse of this lane's head, loaded beside ctx / dctx (NV > 0)
+  auto finish = [&](float acc, int col, float lz) {
     acc += __shfl_xor_sync(0xffffffffu, acc, 1);
     acc += __shfl_xor_sync(0xffffffffu, acc, 2);
     acc += __shfl_xor_sync(0xffffffffu, acc, 4);
@@ -65,27 +66,31 @@ __global__ void attn_delta_bf16(const bf16* __restrict__ ctx, const bf16* __rest
                           0u, 0u, 0u);
       };
       constexpr float kC = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
-      xtab[(bh * 2) * S + s] = row16(__fdiv_rn(lse[bh * S + s], kC));
+      xtab[(bh * 2) * S + s] = row16(__fdiv_rn(lz, kC));
       xtab[(bh * 2 + 1) * S + s] = row16(acc);
     }
   };
   if constexpr (NV > 0) {
     uint4 x[NV], y[NV];
+    float lz[NV];
 #pragma unroll
     for (int v = 0; v < NV; ++v) {
       x[v] = *reinterpret_cast<const uint4*>(ctx + row * H + v * 256 + l * 8);
       y[v] = *reinterpret_cast<const uint4*>(dctx + row * H + v * 256 + l * 8);
+      lz[v] = (l & 7) == 0 ? lse[(b * A + (v * 256 + l * 8) / HD) * S + s] : 0.f;
     }
 #pragma unroll
-    for (int v = 0; v < NV; ++v) finish(dot8(x[v], y[v]), v * 256 + l * 8);
+    for (int v = 0; v < NV; ++v) finish(dot8(x[v], y[v]), v * 256 + l * 8, lz[v]);
   } else {
     for (int c0 = 0; c0 < H; c0 += 256) {
       const int col = c0 + l * 8;
-      float acc = 0.f;
-      if (col < H)
+      float acc = 0.f, lz = 0.f;
+      if (col < H) {
         acc = dot8(*reinterpret_cast<const uint4*>(ctx + row * H + col),
                    *reinterpret_cast<const uint4*>(dctx + row * H + col));
-      finish(acc, col);
+        if ((l & 7) == 0) lz = lse[(b * A + col / HD) * S + s];
+      }
+      finish(acc, col, lz);
     }
   }
 }
