@@ -47,9 +47,6 @@ namespace gemm {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;        // 16 KiB
-constexpr int B_BYTES = BN * BK * 2;        // 32 KiB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TMEM_COLS = 2 * BN;           // two fp32 accumulators of 128 x 256
 constexpr int NUM_EPI_WARPS = 8;            // two per TMEM lane quarter (default)
 constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
 // CTA-pair variant: per CTA and stage A 128 x 64 + B 128 x 64 (32 KiB).  Six
@@ -59,20 +56,23 @@ constexpr int MN_CHUNK_BYTES = 64 * BK * 2; // one 64-wide MN-major box: 8 KiB
 // ring), while the others ran 1-2 us faster and the step 0.7% faster.
 constexpr int PAIR_STAGES = 5;
 constexpr int PAIR_STAGES_WIDE = 6;  // all but the GELU' data-gradient epilogue
-constexpr int PAIR_STAGE_BYTES = A_BYTES + (BN / 2) * BK * 2;
 
 // Launch shape per instantiation: epilogue warps (a multiple of 4, one group
 // per TMEM lane quarter), epilogue chunk width, ring stages and shared memory.
 // The bias+GELU epilogue is bound by its own math: it runs 16 warps (four per
 // lane quarter, 64 columns each) on 16-column chunks, which keeps it at about
 // 100 registers a thread (576 threads leave 112).
-template <int EPI, bool PAIR>
+// TBN: the tile's width (256, or 192 for K-major B operands whose output
+// width fills the SM pairs better in 192-wide tiles).
+template <int EPI, bool PAIR, int TBN = BN>
 struct Shape {
   static constexpr int EW = EPI == SKY_EPI_BIAS_GELU ? 16 : NUM_EPI_WARPS;
   static constexpr int CW = EW == 16 ? 16 : 32;              // epilogue chunk width (columns)
   static constexpr int THREADS = 64 + 32 * EW;
   static constexpr int NST = PAIR ? (EPI == SKY_EPI_GELU_BWD ? PAIR_STAGES : PAIR_STAGES_WIDE) : STAGES;
-  static constexpr int SBYTES = PAIR ? PAIR_STAGE_BYTES : STAGE_BYTES;
+  static constexpr int SBYTES = A_BYTES + (PAIR ? TBN / 2 : TBN) * BK * 2;
+  // two fp32 accumulators of 128 x TBN, in a power-of-two TMEM allocation
+  static constexpr int TMEM_ALLOC = 2 * TBN <= 256 ? 256 : 512;
   static constexpr int EPI_OFF = NST * SBYTES;               // per epilogue warp: 32 x CW fp32 staging
   static constexpr int BAR_OFF = EPI_OFF + EW * 32 * CW * 4;
   static constexpr int SMEM = BAR_OFF + 256 /*barriers*/ + 1024 /*alignment slack*/;
@@ -116,15 +116,16 @@ __device__ __forceinline__ float4 ld_nc_f4(const float* p) {
 
 // PAIR: the CTA-pair variant (launched in clusters of two; p.m_tiles counts
 // 256-row tiles).
-template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR>
-__global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
+template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR, int TBN = BN>
+__global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA,
                    const __grid_constant__ CUtensorMap tmB, const Params p) {
-  using SH = Shape<EPI, PAIR>;
+  using SH = Shape<EPI, PAIR, TBN>;
   constexpr int NST = SH::NST;
   constexpr int SBYTES = SH::SBYTES;
   constexpr int EW = SH::EW;
-  constexpr int B_ROWS = PAIR ? BN / 2 : BN;  // B rows (tile columns) this CTA loads
+  constexpr int B_ROWS = PAIR ? TBN / 2 : TBN;  // B rows (tile columns) this CTA loads
+  static_assert(!B_MN || B_ROWS % 64 == 0, "MN-major B is loaded in 64-column boxes");
   constexpr int TILE_M = PAIR ? 2 * BM : BM;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = ptx::smem_u32(smem_raw);
@@ -160,10 +161,10 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
   }
   if (warp == 1) {
     if constexpr (PAIR) {
-      ptx::tmem_alloc_pair(tmem_slot, TMEM_COLS);
+      ptx::tmem_alloc_pair(tmem_slot, SH::TMEM_ALLOC);
       ptx::tmem_relinquish_pair();
     } else {
-      ptx::tmem_alloc(tmem_slot, TMEM_COLS);
+      ptx::tmem_alloc(tmem_slot, SH::TMEM_ALLOC);
       ptx::tmem_relinquish();
     }
   }
@@ -189,7 +190,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
       for (int u = cid; u < units && ok; u += ncl) {
         const int split = u / tiles, rem = u % tiles;
         const int m0 = (rem / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
-        const int n0 = (rem % p.n_tiles) * BN + static_cast<int>(rank) * (BN - B_ROWS);
+        const int n0 = (rem % p.n_tiles) * TBN + static_cast<int>(rank) * (TBN - B_ROWS);
         const int kb0 = split * p.kb_per_split;
         const int kb1 = min(p.k_blocks, kb0 + p.kb_per_split);
         for (int kb = kb0; kb < kb1; ++kb) {
@@ -237,7 +238,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------- MMA issue
     if (lane == 0 && leader) {
-      constexpr uint32_t idesc = ptx::idesc_bf16_f32(TILE_M, BN, A_MN, B_MN);
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(TILE_M, TBN, A_MN, B_MN);
       auto commit = [&](uint64_t* bar) {  // to this barrier in both CTAs of a pair
         if constexpr (PAIR) ptx::tc_commit_pair(bar, 3);
         else ptx::tc_commit(bar);
@@ -256,7 +257,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
                    : ptx::mbar_wait(&tempty[acc], aphase ^ 1u, lim, p.status)))
           break;
         ptx::tc_fence_after();
-        const uint32_t d_tmem = tmem_base + acc * BN;
+        const uint32_t d_tmem = tmem_base + acc * TBN;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!ptx::mbar_wait(&full[stage], phase, lim, p.status)) { ok = false; break; }
           ptx::tc_fence_after();
@@ -291,7 +292,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
     // column half hf of the tile.  Per 32-column chunk: tcgen05.ld (thread =
     // row) -> XOR-swizzled smem tile -> read back so that 8 lanes cover one
     // row's 32 columns, then the fused epilogue and coalesced stores.
-    constexpr int HALF = BN / (EW / 4), CHUNKS = HALF / 32;  // columns of a warp, 32-column chunks
+    constexpr int HALF = TBN / (EW / 4), CHUNKS = HALF / 32;  // columns of a warp, 32-column chunks
     const int q = warp & 3, hf = (warp - 2) >> 2;
     float* stage = reinterpret_cast<float*>(smem + SH::EPI_OFF) + (warp - 2) * 32 * SH::CW;
     const int c4 = lane & 7;          // this lane's 4-column group in a chunk
@@ -301,7 +302,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
     for (int u = cid; u < units; u += ncl) {
       const int split = u / tiles, rem = u % tiles;
       const int m0 = (rem / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
-      const int n0 = (rem % p.n_tiles) * BN + hf * HALF;
+      const int n0 = (rem % p.n_tiles) * TBN + hf * HALF;
       // GELU' input of this warp's whole sub-tile, fetched before the wait
       uint2 pre[EPI == SKY_EPI_GELU_BWD ? CHUNKS : 1][8];
       if constexpr (EPI == SKY_EPI_GELU_BWD) {
@@ -349,7 +350,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
       }
       if (!ptx::mbar_wait(&tfull[acc], aphase, lim, p.status, kSleepNs)) break;
       ptx::tc_fence_after();
-      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN + hf * HALF;
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * TBN + hf * HALF;
       float* outf = OUT_F32 ? static_cast<float*>(p.C) +
                                   static_cast<int64_t>(split) * p.M * static_cast<int64_t>(p.N)
                             : nullptr;
@@ -533,8 +534,8 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR>::THREADS, 1)
   else __syncthreads();
   if (warp == 1) {
     ptx::tc_fence_after();
-    if constexpr (PAIR) ptx::tmem_dealloc_pair(tmem_base, TMEM_COLS);
-    else ptx::tmem_dealloc(tmem_base, TMEM_COLS);
+    if constexpr (PAIR) ptx::tmem_dealloc_pair(tmem_base, SH::TMEM_ALLOC);
+    else ptx::tmem_dealloc(tmem_base, SH::TMEM_ALLOC);
   }
 }
 
@@ -610,11 +611,11 @@ bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, in
 // Launches `units` work units on a persistent grid: one CTA per SM, or for
 // the pair variant one two-CTA cluster per SM pair, capped by how many such
 // clusters the device can hold at once (so the grid is a single wave).
-template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR>
+template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR, int TBN = BN>
 cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
                            const Params& p, cudaStream_t stream) {
-  auto kern = gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32, PAIR>;
-  using SH = Shape<EPI, PAIR>;
+  auto kern = gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32, PAIR, TBN>;
+  using SH = Shape<EPI, PAIR, TBN>;
   static cudaError_t attr =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SH::SMEM);
   if (attr != cudaSuccess) return attr;
@@ -745,16 +746,28 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   const bool a_mn = form == SKY_GEMM_XTW;
   const bool b_mn = form != SKY_GEMM_XWT;
   const bool pair = use_pair(M, epi);
+  // 192-wide pair tiles for K-major B and the plain-store epilogue (bf16 or
+  // fp32 output, bias and residual allowed; no split-K) when the product is
+  // less than one wave of 256-wide tiles and still one wave of 192-wide ones:
+  // more SM pairs then share it.  (Over several waves the narrower tile's
+  // main loop, which reuses each A tile for fewer columns, lost more than
+  // the fuller last wave gained: QKV at T = 8192 took 47.1 instead of 43.1 us.)
+  const int clusters = sms / 2;
+  const int64_t m_t = ceil_div(M, pair ? 2 * BM : BM);
+  const bool may_split = out_f32 && epi == SKY_EPI_STORE && bias == nullptr && resid == nullptr;
+  const bool narrow = pair && form == SKY_GEMM_XWT && epi == SKY_EPI_STORE && !may_split &&
+                      !colsum && !deferred_rows && N % 192 == 0 &&
+                      m_t * ceil_div(N, BN) < clusters && m_t * (N / 192) <= clusters;
+  const int tbn = narrow ? 192 : BN;
   bool ok = a_mn ? make_map(&ta, A, K, M, 64) : make_map(&ta, A, M, K, BM);
-  ok = ok && (b_mn ? make_map(&tb, B, K, N, 64) : make_map(&tb, B, N, K, pair ? BN / 2 : BN));
+  ok = ok && (b_mn ? make_map(&tb, B, K, N, 64) : make_map(&tb, B, N, K, pair ? tbn / 2 : tbn));
   SKY_CHECK(ok, SKY_ERR_CUDA, "cuTensorMapEncodeTiled failed (M=%d N=%d K=%d)", M, N, K);
 
   Params p{};
   p.M = M; p.N = N; p.K = K;
   p.m_tiles = ceil_div(M, pair ? 2 * BM : BM);
-  p.n_tiles = ceil_div(N, BN);
+  p.n_tiles = ceil_div(N, tbn);
   p.k_blocks = ceil_div(K, BK);
-  const bool may_split = out_f32 && epi == SKY_EPI_STORE && bias == nullptr && resid == nullptr;
   p.splits = may_split ? choose_splits(p.m_tiles * p.n_tiles, p.k_blocks, pair ? sms / 2 : sms) : 1;
   if (p.splits > 1) {  // never more partials than the workspace holds
     const size_t cap = ws_bytes / (static_cast<size_t>(M) * N * sizeof(float));
@@ -794,7 +807,10 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
 
   const int units = p.m_tiles * p.n_tiles * p.splits;
   cudaError_t e;
-  if (pair) {
+  if (narrow) {
+    e = out_f32 ? launch_variant<false, false, SKY_EPI_STORE, true, true, 192>(units, sms, ta, tb, p, stream)
+                : launch_variant<false, false, SKY_EPI_STORE, false, true, 192>(units, sms, ta, tb, p, stream);
+  } else if (pair) {
     if (form == SKY_GEMM_XWT)
       e = launch_form<false, false, true>(units, sms, ta, tb, p, epi, out_f32, stream);
     else if (form == SKY_GEMM_XW)

@@ -72,7 +72,10 @@ def test_gemm_store(dt, form, shape):
 
 
 @pytest.mark.parametrize("dt", ["bf16", "fp32"])
-@pytest.mark.parametrize("shape", [(256, 512, 128), (200, 264, 72)], ids=lambda s: "x".join(map(str, s)))
+# (256, 384, 128) and (512, 768, 192) run the 192-wide pair tiles in their
+# plain-store (bias) products
+@pytest.mark.parametrize("shape", [(256, 512, 128), (200, 264, 72), (256, 384, 128), (512, 768, 192)],
+                         ids=lambda s: "x".join(map(str, s)))
 def test_gemm_epilogues(dt, shape):
     M, N, K = shape
     g = np.random.default_rng(11)
