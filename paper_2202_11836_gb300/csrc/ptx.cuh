@@ -37,12 +37,6 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                "r"(bytes)
                : "memory");
 }
-// Raises the transaction count of the current phase without arriving.
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
 // One probe of the phase with the given parity; the thread may be suspended
 // for up to `hint_ns` while the phase is still pending, so waiting threads
 // do not take issue slots from the producer and MMA threads.
