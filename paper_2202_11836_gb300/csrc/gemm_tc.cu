@@ -28,9 +28,9 @@
 // the single-CTA 128 x 256 tile.  The leader CTA's thread issues the MMAs;
 // both CTAs' TMA loads complete on the leader's stage barrier, and the
 // leader's commits arrive on both CTAs' stage-empty and accumulator barriers.
-// Weight gradients
-// (fp32 output) may split the token dimension over CTAs; partials go to a
-// workspace and are summed in a fixed order, so results are deterministic.
+// Weight gradients (fp32 output) may split the token dimension over CTAs;
+// partials go to a workspace and are summed in a fixed order, so results are
+// deterministic.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -114,6 +114,26 @@ __device__ __forceinline__ float4 ld_nc_f4(const float* p) {
   return v;
 }
 
+// ---- work schedule ------------------------------------------------------
+// Every persistent CTA (pair) walks the same list of work units cid, cid +
+// ncl, cid + 2 ncl, ... of the tiles * splits (split-major): unit u is tile
+// u % tiles over the k-blocks of split u / tiles.
+struct Work {
+  int tile, split, kb0, kb1;
+};
+struct Sched {
+  int tiles, units, kbps, kbs, ncl, cid;
+};
+__device__ __forceinline__ bool work_item(const Sched& sched, int it, Work& w) {
+  const int u = sched.cid + it * sched.ncl;
+  if (u >= sched.units) return false;
+  w.split = u / sched.tiles;
+  w.tile = u - w.split * sched.tiles;
+  w.kb0 = w.split * sched.kbps;
+  w.kb1 = min(sched.kbs, w.kb0 + sched.kbps);
+  return true;
+}
+
 // PAIR: the CTA-pair variant (launched in clusters of two; p.m_tiles counts
 // 256-row tiles).
 template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR, int TBN = BN>
@@ -176,9 +196,10 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
   const uint32_t tmem_base = *tmem_slot;
   pdl_wait();  // the set-up above overlapped the previous kernel; its outputs are visible now
 
-  const int tiles = p.m_tiles * p.n_tiles;
-  const int units = tiles * p.splits;
   const uint64_t lim = p.timeout_ns;
+  const Sched sched{p.m_tiles * p.n_tiles, p.m_tiles * p.n_tiles * p.splits, p.kb_per_split,
+                    p.k_blocks, ncl, cid};
+  Work w;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -187,13 +208,10 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
-      for (int u = cid; u < units && ok; u += ncl) {
-        const int split = u / tiles, rem = u % tiles;
-        const int m0 = (rem / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
-        const int n0 = (rem % p.n_tiles) * TBN + static_cast<int>(rank) * (TBN - B_ROWS);
-        const int kb0 = split * p.kb_per_split;
-        const int kb1 = min(p.k_blocks, kb0 + p.kb_per_split);
-        for (int kb = kb0; kb < kb1; ++kb) {
+      for (int it = 0; ok && work_item(sched, it, w); ++it) {
+        const int m0 = (w.tile / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
+        const int n0 = (w.tile % p.n_tiles) * TBN + static_cast<int>(rank) * (TBN - B_ROWS);
+        for (int kb = w.kb0; kb < w.kb1; ++kb) {
           if (!ptx::mbar_wait(&empty[stage], phase ^ 1u, lim, p.status)) { ok = false; break; }
           uint8_t* sa = smem + stage * SBYTES;
           uint8_t* sb = sa + A_BYTES;
@@ -248,17 +266,14 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
       int acc = 0;
       uint32_t aphase = 0;
       bool ok = true;
-      for (int u = cid; u < units && ok; u += ncl) {
-        const int split = u / tiles;
-        const int kb0 = split * p.kb_per_split;
-        const int kb1 = min(p.k_blocks, kb0 + p.kb_per_split);
+      for (int it = 0; ok && work_item(sched, it, w); ++it) {
         // both CTAs' epilogues have drained this accumulator
         if (!(PAIR ? ptx::mbar_wait_cluster(&tempty[acc], aphase ^ 1u, lim, p.status)
                    : ptx::mbar_wait(&tempty[acc], aphase ^ 1u, lim, p.status)))
           break;
         ptx::tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * TBN;
-        for (int kb = kb0; kb < kb1; ++kb) {
+        for (int kb = w.kb0; kb < w.kb1; ++kb) {
           if (!ptx::mbar_wait(&full[stage], phase, lim, p.status)) { ok = false; break; }
           ptx::tc_fence_after();
           const uint32_t sa = ptx::smem_u32(smem + stage * SBYTES);
@@ -270,9 +285,9 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
             const uint64_t bd = B_MN ? ptx::smem_desc_sw128(sb + kk * 2048, MN_CHUNK_BYTES, 1024)
                                      : ptx::smem_desc_sw128(sb + kk * 32, 16, 1024);
             if constexpr (PAIR)
-              ptx::tc_mma_f16_pair(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+              ptx::tc_mma_f16_pair(d_tmem, ad, bd, idesc, (kb > w.kb0 || kk > 0) ? 1u : 0u);
             else
-              ptx::tc_mma_f16(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+              ptx::tc_mma_f16(d_tmem, ad, bd, idesc, (kb > w.kb0 || kk > 0) ? 1u : 0u);
           }
           commit(&empty[stage]);
           if (++stage == NST) { stage = 0; phase ^= 1u; }
@@ -299,10 +314,17 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
     const int rsub = lane >> 3;       // row within each group of 4 rows
     int acc = 0;
     uint32_t aphase = 0;
-    for (int u = cid; u < units; u += ncl) {
-      const int split = u / tiles, rem = u % tiles;
-      const int m0 = (rem / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
-      const int n0 = (rem % p.n_tiles) * TBN + hf * HALF;
+    // hands the accumulator back to the MMA issuer (both CTAs' epilogues arrive
+    // on the leader's barrier)
+    auto release_acc = [&]() {
+      ptx::tc_fence_before();
+      if (leader) ptx::mbar_arrive(&tempty[acc]);
+      else ptx::mbar_arrive_cluster(ptx::mapa_shared(ptx::smem_u32(&tempty[acc]), 0));
+      if (++acc == 2) { acc = 0; aphase ^= 1u; }
+    };
+    for (int it = 0; work_item(sched, it, w); ++it) {
+      const int m0 = (w.tile / p.n_tiles) * TILE_M + static_cast<int>(rank) * BM;
+      const int n0 = (w.tile % p.n_tiles) * TBN + hf * HALF;
       // GELU' input of this warp's whole sub-tile, fetched before the wait
       uint2 pre[EPI == SKY_EPI_GELU_BWD ? CHUNKS : 1][8];
       if constexpr (EPI == SKY_EPI_GELU_BWD) {
@@ -352,7 +374,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
       ptx::tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * TBN + hf * HALF;
       float* outf = OUT_F32 ? static_cast<float*>(p.C) +
-                                  static_cast<int64_t>(split) * p.M * static_cast<int64_t>(p.N)
+                                  static_cast<int64_t>(w.split) * p.M * static_cast<int64_t>(p.N)
                             : nullptr;
       if constexpr (EPI == SKY_EPI_BIAS_GELU) {
         // CW-column chunks: LPR lanes cover a row's CW columns, RPI rows per step
@@ -521,10 +543,7 @@ __global__ void __launch_bounds__(Shape<EPI, PAIR, TBN>::THREADS, 1)
           }
         }
       }
-      ptx::tc_fence_before();
-      if (leader) ptx::mbar_arrive(&tempty[acc]);
-      else ptx::mbar_arrive_cluster(ptx::mapa_shared(ptx::smem_u32(&tempty[acc]), 0));
-      if (++acc == 2) { acc = 0; aphase ^= 1u; }
+      release_acc();
     }
   }
 
@@ -608,21 +627,19 @@ bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, in
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Launches `units` work units on a persistent grid: one CTA per SM, or for
-// the pair variant one two-CTA cluster per SM pair, capped by how many such
-// clusters the device can hold at once (so the grid is a single wave).
+// Launches the product's work units on a persistent grid: one CTA per SM, or
+// for the pair variant one two-CTA cluster per SM pair, capped by how many
+// such clusters the device holds at once (a single wave).
 template <bool A_MN, bool B_MN, int EPI, bool OUT_F32, bool PAIR, int TBN = BN>
-cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
-                           const Params& p, cudaStream_t stream) {
+cudaError_t launch_variant(const Params& p, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
+                           cudaStream_t stream) {
   auto kern = gemm_tc_kernel<A_MN, B_MN, EPI, OUT_F32, PAIR, TBN>;
   using SH = Shape<EPI, PAIR, TBN>;
   static cudaError_t attr =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SH::SMEM);
   if (attr != cudaSuccess) return attr;
-  if constexpr (!PAIR) {
-    const int grid = units < sms ? units : sms;
-    return launch_pdl(kern, dim3(grid), dim3(SH::THREADS), SH::SMEM, stream, 1, ta, tb, p);
-  } else {
+  int ctas = sms;
+  if constexpr (PAIR) {
     static int max_clusters = [&] {
       cudaLaunchConfig_t q = {};
       cudaLaunchAttribute at[1];
@@ -643,27 +660,28 @@ cudaError_t launch_variant(int units, int sms, const CUtensorMap& ta, const CUte
       return n;
     }();
     if (max_clusters < 1) return cudaErrorLaunchOutOfResources;
-    const int clusters = units < max_clusters ? units : max_clusters;
-    return launch_pdl(kern, dim3(2 * clusters), dim3(SH::THREADS), SH::SMEM, stream, 2, ta, tb, p);
+    ctas = max_clusters;
   }
+  const int units = p.m_tiles * p.n_tiles * p.splits;
+  const int grid = units < ctas ? units : ctas;
+  return launch_pdl(kern, dim3((PAIR ? 2 : 1) * grid), dim3(SH::THREADS), SH::SMEM, stream,
+                    PAIR ? 2 : 1, ta, tb, p);
 }
 
 // One instantiation per (operand majorness, epilogue, output type, pairing)
 // keeps every kernel's code to the epilogue it runs.
 template <bool A_MN, bool B_MN, bool PAIR>
-cudaError_t launch_form(int units, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
-                        const Params& p, int epi, bool out_f32, cudaStream_t stream) {
+cudaError_t launch_form(const Params& p, int sms, const CUtensorMap& ta, const CUtensorMap& tb,
+                        int epi, bool out_f32, cudaStream_t stream) {
   if (out_f32)
-    return launch_variant<A_MN, B_MN, SKY_EPI_STORE, true, PAIR>(units, sms, ta, tb, p, stream);
+    return launch_variant<A_MN, B_MN, SKY_EPI_STORE, true, PAIR>(p, sms, ta, tb, stream);
   switch (epi) {
     case SKY_EPI_BIAS_GELU:
-      return launch_variant<A_MN, B_MN, SKY_EPI_BIAS_GELU, false, PAIR>(units, sms, ta, tb, p,
-                                                                        stream);
+      return launch_variant<A_MN, B_MN, SKY_EPI_BIAS_GELU, false, PAIR>(p, sms, ta, tb, stream);
     case SKY_EPI_GELU_BWD:
-      return launch_variant<A_MN, B_MN, SKY_EPI_GELU_BWD, false, PAIR>(units, sms, ta, tb, p,
-                                                                       stream);
+      return launch_variant<A_MN, B_MN, SKY_EPI_GELU_BWD, false, PAIR>(p, sms, ta, tb, stream);
     default:
-      return launch_variant<A_MN, B_MN, SKY_EPI_STORE, false, PAIR>(units, sms, ta, tb, p, stream);
+      return launch_variant<A_MN, B_MN, SKY_EPI_STORE, false, PAIR>(p, sms, ta, tb, stream);
   }
 }
 
@@ -754,6 +772,12 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   // the fuller last wave gained: QKV at T = 8192 took 47.1 instead of 43.1 us.)
   const int clusters = sms / 2;
   const int64_t m_t = ceil_div(M, pair ? 2 * BM : BM);
+  // 192-wide pair tiles for K-major B and the plain-store epilogue when the
+  // product is less than one wave of 256-wide tiles and still one wave of
+  // 192-wide ones: more SM pairs then share it.  (Over several waves the
+  // narrower tile's main loop, which reuses each A tile for fewer columns,
+  // lost more than the fuller last wave gained: QKV at T = 8192 took 47.1
+  // instead of 43.1 us.)
   const bool may_split = out_f32 && epi == SKY_EPI_STORE && bias == nullptr && resid == nullptr;
   const bool narrow = pair && form == SKY_GEMM_XWT && epi == SKY_EPI_STORE && !may_split &&
                       !colsum && !deferred_rows && N % 192 == 0 &&
@@ -765,7 +789,7 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
 
   Params p{};
   p.M = M; p.N = N; p.K = K;
-  p.m_tiles = ceil_div(M, pair ? 2 * BM : BM);
+  p.m_tiles = static_cast<int>(m_t);
   p.n_tiles = ceil_div(N, tbn);
   p.k_blocks = ceil_div(K, BK);
   p.splits = may_split ? choose_splits(p.m_tiles * p.n_tiles, p.k_blocks, pair ? sms / 2 : sms) : 1;
@@ -805,25 +829,24 @@ sky_status launch_bf16(sky_gemm_form form, int M, int N, int K, const void* A, c
   p.timeout_ns = g_timeout_ns;
   p.skip_loads = g_skip_loads;
 
-  const int units = p.m_tiles * p.n_tiles * p.splits;
   cudaError_t e;
   if (narrow) {
-    e = out_f32 ? launch_variant<false, false, SKY_EPI_STORE, true, true, 192>(units, sms, ta, tb, p, stream)
-                : launch_variant<false, false, SKY_EPI_STORE, false, true, 192>(units, sms, ta, tb, p, stream);
+    e = out_f32 ? launch_variant<false, false, SKY_EPI_STORE, true, true, 192>(p, sms, ta, tb, stream)
+                : launch_variant<false, false, SKY_EPI_STORE, false, true, 192>(p, sms, ta, tb, stream);
   } else if (pair) {
     if (form == SKY_GEMM_XWT)
-      e = launch_form<false, false, true>(units, sms, ta, tb, p, epi, out_f32, stream);
+      e = launch_form<false, false, true>(p, sms, ta, tb, epi, out_f32, stream);
     else if (form == SKY_GEMM_XW)
-      e = launch_form<false, true, true>(units, sms, ta, tb, p, epi, out_f32, stream);
+      e = launch_form<false, true, true>(p, sms, ta, tb, epi, out_f32, stream);
     else
-      e = launch_form<true, true, true>(units, sms, ta, tb, p, epi, out_f32, stream);
+      e = launch_form<true, true, true>(p, sms, ta, tb, epi, out_f32, stream);
   } else {
     if (form == SKY_GEMM_XWT)
-      e = launch_form<false, false, false>(units, sms, ta, tb, p, epi, out_f32, stream);
+      e = launch_form<false, false, false>(p, sms, ta, tb, epi, out_f32, stream);
     else if (form == SKY_GEMM_XW)
-      e = launch_form<false, true, false>(units, sms, ta, tb, p, epi, out_f32, stream);
+      e = launch_form<false, true, false>(p, sms, ta, tb, epi, out_f32, stream);
     else
-      e = launch_form<true, true, false>(units, sms, ta, tb, p, epi, out_f32, stream);
+      e = launch_form<true, true, false>(p, sms, ta, tb, epi, out_f32, stream);
   }
   count_launches(1);
   if (e != cudaSuccess) return cuda_fail(e, "gemm_tc_kernel launch");
