@@ -108,6 +108,19 @@ def test_gemm_epilogues(dt, shape):
            L.SKY_EPI_STORE, P(b), None, None, None, 0, None, stream())
     torch.cuda.synchronize()
     assert l2rel(to_host(c32), acc + bias) <= 1e-5
+    # bias into an output of the input type (the QKV projection's form), with
+    # the bias 16-byte aligned and 8 bytes off: the results agree bit for bit
+    outs = []
+    for off in (0, 4 if dt == "bf16" else 2):
+        braw = torch.zeros(N + 8, dtype=td, device="cuda")
+        braw[off:off + N] = b
+        cb = torch.empty((M, N), dtype=td, device="cuda")
+        L.call("sky_gemm", L.SKY_GEMM_XWT, M, N, K, dt_code(dt), P(a), P(w), P(cb), dt_code(dt),
+               L.SKY_EPI_STORE, P(braw[off:off + N]), None, None, None, 0, None, stream())
+        torch.cuda.synchronize()
+        outs.append(to_host(cb))
+        assert l2rel(outs[-1], acc + bias) <= tol_l2
+    assert np.array_equal(outs[0], outs[1])
 
 
 def test_gemm_wgrad_split_deterministic():
