@@ -137,6 +137,11 @@ def test_layernorm_writes_in_bounds(dt, TH):
     L.call("sky_layernorm_fwd", P(a), P(r), P(gam), P(bet), T, H, C.c_float(1e-5), code(dt),
            P(u), P(y32), P(y), P(mean), P(rstd), stream())
     check(u, y32, y, mean, rstd)
+    if dt == "bf16":  # u alone into a bf16 y (the slice's form)
+        y2, m2, r2 = Guarded((T, H), torch.bfloat16), Guarded((T,), torch.float32), Guarded((T,), torch.float32)
+        L.call("sky_layernorm_fwd", P(a), None, P(gam), P(bet), T, H, C.c_float(1e-5), code(dt),
+               None, None, P(y2), P(m2), P(r2), stream())
+        check(y2, m2, r2)
     dy = rand((T, H), dt, 1e-2, seed=10)
     dy2 = rand((T, H), "fp32", 1e-2, seed=11)
     wsb = L.lib().sky_layernorm_bwd_workspace_bytes(T, H)
